@@ -1,0 +1,175 @@
+/*
+ * quartz.h -- C ABI of the GB300 (sm_103a) QuaRTZ W4A4 linear hot path.
+ *
+ * QuaRTZ (arXiv 2509.26436) quantizes activations and weights in two stages:
+ * per-group 8-bit min-max quantization (Section 3, Eq. 1) followed by
+ * Leading Zero Suppression of each 8-bit code to a signed 4-bit code plus a
+ * per-subgroup FLAG (Section 3, Eq. 2).  The linear layer multiplies two such
+ * encoded operands with an integer MMA and applies the per-group 16-bit
+ * scales afterwards (Section 4.4; Appendix C: groups of 64 along K, 16-bit
+ * scales).
+ *
+ * Conventions shared by every entry point
+ *   - All tensor pointers are DEVICE pointers owned by the caller.  The
+ *     library never allocates, frees or synchronises (except
+ *     quartz_device_status, which synchronises the given stream).
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  Every launch is asynchronous on that stream.
+ *   - Every call returns a quartz_status_t (as int32_t).  Arguments are
+ *     validated on the host before anything is launched; on any error
+ *     nothing is launched and no output is touched.
+ *   - Inputs containing NaN or Inf are unsupported (results undefined; the
+ *     kernels do not fault on them).
+ *   - Layouts are row-major and contiguous.  "fp16" means IEEE binary16.
+ */
+#ifndef QUARTZ_H
+#define QUARTZ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    QUARTZ_OK = 0,
+    QUARTZ_ERR_INVALID_ARG = 1,   /* bad size, group size, mode, type or NULL pointer */
+    QUARTZ_ERR_ALIGNMENT = 2,     /* a pointer is not 16-byte aligned */
+    QUARTZ_ERR_UNSUPPORTED = 3,   /* valid per the paper but not built (e.g. group_q != 64) */
+    QUARTZ_ERR_CUDA = 4,          /* a CUDA runtime / driver call failed */
+    QUARTZ_ERR_TIMEOUT = 5,       /* a kernel's bounded wait expired (reported by quartz_device_status) */
+    QUARTZ_ERR_WORKSPACE = 6      /* workspace missing or smaller than quartz_linear_workspace_size */
+} quartz_status_t;
+
+/* Eq. 1 conventions.  The paper's printed Eq. 1 (s = (max-min)/255, clamp to
+ * [-127,127], z = round(-min/s)) is not self-consistent; Appendix A analyses
+ * the symmetric midtread quantizer, which is the default here.
+ *   SYMMETRIC:  s = fp16(max|x| / 127), z = 0, q = clamp(round(x/s), -127, 127)
+ *   ASYMMETRIC: [lo, hi] = [min(min x, 0), max(max x, 0)],
+ *               s = fp16((hi - lo) / 255), z = round(-lo/s) - 128 (stored),
+ *               q = clamp(round(x/s) + z, -127, 127)
+ * round() is round-half-to-even; x/s is evaluated as x * r, r = RN(1/s) in
+ * binary32; a group whose fp16 scale is 0 gets all-zero codes and z = 0. */
+typedef enum { QUARTZ_SYMMETRIC = 0, QUARTZ_ASYMMETRIC = 1 } quartz_mode_t;
+
+typedef enum { QUARTZ_OUT_F16 = 0, QUARTZ_OUT_BF16 = 1, QUARTZ_OUT_F32 = 2 } quartz_out_t;
+
+/* GEMM implementations behind quartz_linear_ex.  TCGEN05 is the product
+ * path (tcgen05 tensor cores, TMEM accumulators); SIMT is a plain CUDA-core
+ * kernel with the same arithmetic, kept as a second on-device path. */
+typedef enum { QUARTZ_ALGO_TCGEN05 = 0, QUARTZ_ALGO_SIMT = 1 } quartz_algo_t;
+
+typedef struct {
+    int32_t group_q; /* min-max quantization group along K; 64 (Appendix C) */
+    int32_t group_s; /* LZS subgroup G_s along K: 8, 16, 32 or 64 (Section 3, Table 1) */
+    int32_t mode;    /* quartz_mode_t */
+} quartz_params_t;
+
+/* One encoded tensor of `rows` rows and `K` columns (Section 4.4: "packed
+ * s4" codes plus "a single flag byte per subgroup").  Buffers are device
+ * memory owned by the caller; sizes in elements:
+ *   codes  uint8 [rows, K/2]        two's-complement 4-bit codes in [-7, 7],
+ *                                   element 2j in the low nibble of byte j
+ *   flags  uint8 [rows, K/group_s]  FLAG of Eq. 2, values 0..4
+ *   scales fp16  [rows, K/group_q]  16-bit scale s of each group (bits)
+ *   zeros  int8  [rows, K/group_q]  stored zero point z (ASYMMETRIC only;
+ *                                   may be NULL in SYMMETRIC mode)
+ *   gsum   int32 [rows, K/group_q]  sum of the decoded values of each group,
+ *                                   sum_k sgn(c_k)(|c_k| << FLAG) (ASYMMETRIC
+ *                                   only; used by the zero-point correction)
+ * Every pointer must be 16-byte aligned. */
+typedef struct {
+    uint8_t *codes;
+    uint8_t *flags;
+    uint16_t *scales;
+    int8_t *zeros;
+    int32_t *gsum;
+    int64_t rows;
+    int64_t K;
+    quartz_params_t p;
+} quartz_encoded_t;
+
+/* Human-readable name of a status code (static storage; never NULL). */
+const char *quartz_status_string(int32_t status);
+
+/* ABI version of this library: (major << 16) | minor. */
+int32_t quartz_version(void);
+
+/* Bytes of each buffer of an encoded [rows, K] tensor, for allocation:
+ * out[0..4] = codes, flags, scales, zeros, gsum.  Returns QUARTZ_OK or
+ * QUARTZ_ERR_INVALID_ARG. */
+int32_t quartz_encoded_sizes(int64_t rows, int64_t K, const quartz_params_t *p, size_t out[5]);
+
+/* Two-stage QuaRTZ encoder, on the fly for activations (Appendix C: "4-bit
+ * compression is applied on-the-fly"): Eq. 1 per group of p->group_q along
+ * K, then Eq. 2 per subgroup of p->group_s, then nibble packing.
+ *   x_f16  fp16 [out->rows, out->K] device, 16-byte aligned
+ *   out    describes the destination: rows, K, p and the buffers above
+ * Requirements: rows >= 0, K > 0, K % 64 == 0, group_q == 64, group_s in
+ * {8,16,32,64}.  rows == 0 is a no-op. */
+int32_t quartz_quantize(const void *x_f16, const quartz_encoded_t *out, void *stream);
+
+/* The same encoder applied to nn.Linear weights [N, K] (one quantization
+ * row per output channel, groups along K).  Weights are encoded once,
+ * offline; the arithmetic is identical to quartz_quantize. */
+int32_t quartz_encode_weights(const void *w_f16, const quartz_encoded_t *out, void *stream);
+
+/* Dequantise an encoded tensor: x_hat = s * (v - z) with the decoded LZS
+ * value v = sgn(c)(|c| << FLAG) (Section 3: "each group has been shifted
+ * equally"), computed in binary32 and rounded once to fp16.
+ *   x_hat_f16  fp16 [e->rows, e->K] device output. */
+int32_t quartz_dequantize(const quartz_encoded_t *e, void *x_hat_f16, void *stream);
+
+/* Workspace bytes quartz_linear needs for an [M, K] x [N, K]^T product
+ * (the operands expanded to the tensor-core input format plus transposed
+ * group scales).  Returns 0 for invalid arguments. */
+size_t quartz_linear_workspace_size(int64_t M, int64_t N, int64_t K, const quartz_params_t *p);
+
+/* W4A4 QuaRTZ linear (Section 4.4 with Appendix C's group scales):
+ *   y[m, n] = sum_g s_a[m,g] s_w[n,g] (P_g[m,n] - z_w[n,g] A_g[m] - z_a[m,g] W_g[n]
+ *                                      + 64 z_a[m,g] z_w[n,g])  (+ bias[n])
+ *   P_g[m, n] = sum_{k in group g} v_a[m,k] v_w[n,k]   (exact integer sum)
+ * where A_g / W_g are the gsum side values (zero in SYMMETRIC mode).
+ *   a          encoded activations [M, K]
+ *   w          encoded weights [N, K] (same K, group_q, group_s and mode)
+ *   bias_f16   fp16 [N] or NULL
+ *   y          [M, N] of y_type (quartz_out_t), 16-byte aligned
+ *   workspace  device scratch of at least quartz_linear_workspace_size bytes,
+ *              16-byte aligned, owned by the caller; contents are scratch
+ * Requirements: N % 8 == 0, K % 64 == 0, M >= 0.  The per-group partials
+ * P_g are exact; the scaled sum is accumulated in binary32 and rounded once
+ * to y_type. */
+int32_t quartz_linear(const quartz_encoded_t *a, const quartz_encoded_t *w, const void *bias_f16,
+                      void *y, int32_t y_type, void *workspace, size_t workspace_bytes,
+                      void *stream);
+
+/* quartz_linear with two extra controls, for verification:
+ *   partials        NULL, or int32 [M, N]: receives P_g[m, n] of group
+ *                   `partials_group` (0 <= partials_group < K/64), the raw
+ *                   integer MMA result before any scale or zero point
+ *   algo            quartz_algo_t: which GEMM kernel runs */
+int32_t quartz_linear_ex(const quartz_encoded_t *a, const quartz_encoded_t *w,
+                         const void *bias_f16, void *y, int32_t y_type, int32_t *partials,
+                         int32_t partials_group, int32_t algo, void *workspace,
+                         size_t workspace_bytes, void *stream);
+
+/* Synchronise `stream`, then read and clear the library's device error word.
+ * Returns QUARTZ_OK, QUARTZ_ERR_TIMEOUT if a kernel gave up on a bounded
+ * wait since the last call (its outputs are then invalid), or
+ * QUARTZ_ERR_CUDA if the stream reports an error. */
+int32_t quartz_device_status(void *stream);
+
+/* Failure-detection self-test: launches one CTA that waits on an mbarrier
+ * nothing ever arrives at, with a bound of `limit_ns` nanoseconds
+ * (1e3 <= limit_ns <= 1e10).  The kernel gives up, records the timeout in
+ * the device error word and returns; quartz_device_status then reports
+ * QUARTZ_ERR_TIMEOUT.  The same bounded-wait routine guards every wait in
+ * the GEMM pipeline. */
+int32_t quartz_selftest_timeout(int64_t limit_ns, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* QUARTZ_H */

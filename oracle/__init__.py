@@ -69,7 +69,7 @@ def _load():
             lib.oracle_dequantize.argtypes = [P, P, P, P, i64, i64, i32, i32, P]
             lib.oracle_group_partials.argtypes = [P, P, i64, i64, i64, i32, P, i64, P]
             lib.oracle_linear.argtypes = [P, P, P, P, P, P, P, P, i64, i64, i64, i32, i32,
-                                          P, P, i64, P, P]
+                                          P, P, i64, P, P, P]
             _lib = lib
     return _lib
 
@@ -227,13 +227,15 @@ def group_partials(va: np.ndarray, vw: np.ndarray, group_q: int = 64, rows=None)
     return P
 
 
-def linear(a: Encoded, w: Encoded, bias16=None, rows=None) -> np.ndarray:
-    """y [n_rows, N] binary64 of the W4A4 linear (selected rows of A)."""
+def linear(a: Encoded, w: Encoded, bias16=None, rows=None, with_abs: bool = False):
+    """y [n_rows, N] binary64 of the W4A4 linear (selected rows of A); with
+    `with_abs` also sum_g |s_a s_w D_g| + |bias| of each output."""
     if a.K != w.K or a.group_q != w.group_q or a.group_s != w.group_s or a.mode != w.mode:
         raise ValueError("operands must share K, group sizes and mode")
     sel = None if rows is None else np.ascontiguousarray(rows, dtype=np.int64)
     nr = a.rows if sel is None else sel.size
     y = np.empty((nr, w.rows), np.float64)
+    yabs = np.empty((nr, w.rows), np.float64) if with_abs else None
     scratch = np.empty((w.rows, w.K), np.int16)
     az = a.zeros if a.mode == ASYMMETRIC else None
     wz = w.zeros if w.mode == ASYMMETRIC else None
@@ -241,5 +243,6 @@ def linear(a: Encoded, w: Encoded, bias16=None, rows=None) -> np.ndarray:
     _check(_load().oracle_linear(_ptr(a.codes), _ptr(a.flags), _ptr(_as_u16(a.scales)), _ptr(az),
                                  _ptr(w.codes), _ptr(w.flags), _ptr(_as_u16(w.scales)), _ptr(wz),
                                  a.rows, w.rows, a.K, a.group_q, a.group_s, _ptr(b), _ptr(sel),
-                                 0 if sel is None else sel.size, _ptr(scratch), _ptr(y)))
-    return y
+                                 0 if sel is None else sel.size, _ptr(scratch), _ptr(y),
+                                 _ptr(yabs)))
+    return (y, yabs) if with_abs else y

@@ -350,13 +350,15 @@ int oracle_group_partials(const int16_t *va, const int16_t *vw, int64_t M, int64
  * evaluated with integer group sums and binary64 scaling.
  * Encoded operands are passed as (codes, flags, scales, zeros); zeros may be
  * NULL (symmetric).  bias is fp16 bits or NULL.  y [n_sel, N] binary64 for
- * the selected rows (rows_sel NULL = all M rows).
+ * the selected rows (rows_sel NULL = all M rows).  When `yabs` is not NULL it
+ * receives sum_g |s_a s_w D_g| + |bias[n]|, the magnitude a rounding error
+ * bound of any evaluation order scales with.
  * ------------------------------------------------------------------------- */
 int oracle_linear(const uint8_t *a_codes, const uint8_t *a_flags, const uint16_t *a_scales,
                   const int8_t *a_zeros, const uint8_t *w_codes, const uint8_t *w_flags,
                   const uint16_t *w_scales, const int8_t *w_zeros, int64_t M, int64_t N,
                   int64_t K, int gq, int gs, const uint16_t *bias, const int64_t *rows_sel,
-                  int64_t n_sel, int16_t *w_scratch /* [N*K] */, double *y)
+                  int64_t n_sel, int16_t *w_scratch /* [N*K] */, double *y, double *yabs)
 {
     int16_t va[65536];
     if (K > 65536 || gq <= 0 || K % gq != 0 || gs <= 0 || gq % gs != 0) return ORACLE_ERR_ARG;
@@ -371,7 +373,7 @@ int oracle_linear(const uint8_t *a_codes, const uint8_t *a_flags, const uint16_t
         if (rc) return rc;
         for (int64_t n = 0; n < N; ++n) {
             const int16_t *vw = w_scratch + n * K;
-            double acc = 0.0;
+            double acc = 0.0, mag = 0.0;
             for (int64_t g = 0; g < G; ++g) {
                 int za = a_zeros ? a_zeros[m * G + g] : 0;
                 int zw = w_zeros ? w_zeros[n * G + g] : 0;
@@ -381,9 +383,14 @@ int oracle_linear(const uint8_t *a_codes, const uint8_t *a_flags, const uint16_t
                 double sa = (double)oracle_half_to_float(a_scales[m * G + g]);
                 double sw = (double)oracle_half_to_float(w_scales[n * G + g]);
                 acc += sa * sw * (double)d;
+                mag += fabs(sa * sw * (double)d);
             }
-            if (bias) acc += (double)oracle_half_to_float(bias[n]);
+            if (bias) {
+                acc += (double)oracle_half_to_float(bias[n]);
+                mag += fabs((double)oracle_half_to_float(bias[n]));
+            }
             y[i * N + n] = acc;
+            if (yabs) yabs[i * N + n] = mag;
         }
     }
     return ORACLE_OK;

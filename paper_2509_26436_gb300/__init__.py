@@ -1,0 +1,165 @@
+"""QuaRTZ W4A4 linear hot path for GB300 (sm_103a).
+
+Python front end of libquartz.so: it only marshals torch CUDA tensors into
+the C ABI of include/quartz.h (device pointers, sizes, the current CUDA
+stream).  Every step of the path (Eq. 1 quantization, Eq. 2 LZS encoding,
+decode, the integer GEMM and the dequant epilogue) runs in the library's
+CUDA kernels.
+
+    e_a = quantize(x)                 # fp16 [M, K] -> encoded activations
+    e_w = encode_weights(w)           # fp16 [N, K] -> encoded weights (offline)
+    y = linear(e_a, e_w, bias)        # fp16 [M, N]
+
+`inputs` (seeded synthetic data) imports nothing from here.
+"""
+from __future__ import annotations
+
+import ctypes as C
+from dataclasses import dataclass
+
+from . import _native as N
+from ._native import (ALGO_SIMT, ALGO_TCGEN05, ASYMMETRIC, OUT_BF16, OUT_F16, OUT_F32,  # noqa: F401
+                      SYMMETRIC, QuartzError)
+
+__all__ = ["Params", "Encoded", "quantize", "encode_weights", "dequantize", "linear",
+           "linear_workspace_size", "empty_encoded", "device_status", "selftest_timeout",
+           "SYMMETRIC", "ASYMMETRIC", "QuartzError"]
+
+
+def _torch():
+    import torch
+    return torch
+
+
+@dataclass(frozen=True)
+class Params:
+    """group_q: min-max group along K (64, Appendix C); group_s: LZS
+    subgroup G_s (8/16/32/64, Section 3); mode: SYMMETRIC or ASYMMETRIC."""
+    group_q: int = 64
+    group_s: int = 16
+    mode: int = SYMMETRIC
+
+    def c(self) -> N.QuartzParams:
+        return N.QuartzParams(self.group_q, self.group_s, self.mode)
+
+
+class Encoded:
+    """An encoded [rows, K] tensor on the GPU (Section 4.4 storage format):
+    codes uint8 [rows, K/2], flags uint8 [rows, K/G_s], scales fp16
+    [rows, K/64], zeros int8 / gsum int32 [rows, K/64] (asymmetric only)."""
+
+    def __init__(self, codes, flags, scales, zeros, gsum, rows, K, params: Params):
+        self.codes, self.flags, self.scales = codes, flags, scales
+        self.zeros, self.gsum = zeros, gsum
+        self.rows, self.K, self.params = rows, K, params
+
+    def c(self) -> N.QuartzEncoded:
+        ptr = lambda t: None if t is None else t.data_ptr()  # noqa: E731
+        return N.QuartzEncoded(ptr(self.codes), ptr(self.flags), ptr(self.scales), ptr(self.zeros),
+                               ptr(self.gsum), self.rows, self.K, self.params.c())
+
+    @property
+    def nbytes(self) -> int:
+        ts = [self.codes, self.flags, self.scales, self.zeros, self.gsum]
+        return sum(t.numel() * t.element_size() for t in ts if t is not None)
+
+
+def empty_encoded(rows: int, K: int, params: Params = Params(), device="cuda") -> Encoded:
+    torch = _torch()
+    sizes = (C.c_size_t * 5)()
+    p = params.c()
+    N.check(N.load().quartz_encoded_sizes(rows, K, C.byref(p), sizes), "quartz_encoded_sizes")
+    G = K // params.group_q
+    codes = torch.empty((rows, K // 2), dtype=torch.uint8, device=device)
+    flags = torch.empty((rows, K // params.group_s), dtype=torch.uint8, device=device)
+    scales = torch.empty((rows, G), dtype=torch.float16, device=device)
+    zeros = gsum = None
+    if params.mode == ASYMMETRIC:
+        zeros = torch.empty((rows, G), dtype=torch.int8, device=device)
+        gsum = torch.empty((rows, G), dtype=torch.int32, device=device)
+    return Encoded(codes, flags, scales, zeros, gsum, rows, K, params)
+
+
+def _stream(stream=None) -> int:
+    torch = _torch()
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return s.cuda_stream
+
+
+def _check_f16(x, name):
+    torch = _torch()
+    if not (x.is_cuda and x.dtype == torch.float16 and x.dim() == 2 and x.is_contiguous()):
+        raise ValueError(f"{name} must be a contiguous 2-D float16 CUDA tensor")
+
+
+def quantize(x, group_s: int = 16, mode: int = SYMMETRIC, out: Encoded | None = None,
+             stream=None, _entry="quartz_quantize") -> Encoded:
+    """Eq. 1 + Eq. 2 on fp16 activations [M, K] (K % 64 == 0)."""
+    _check_f16(x, "x")
+    rows, K = x.shape
+    e = out if out is not None else empty_encoded(rows, K, Params(64, group_s, mode), x.device)
+    ec = e.c()
+    N.check(getattr(N.load(), _entry)(x.data_ptr(), C.byref(ec), _stream(stream)), _entry)
+    return e
+
+
+def encode_weights(w, group_s: int = 16, mode: int = SYMMETRIC, out: Encoded | None = None,
+                   stream=None) -> Encoded:
+    """The same encoder applied to nn.Linear weights [N, K], run offline."""
+    return quantize(w, group_s, mode, out, stream, _entry="quartz_encode_weights")
+
+
+def dequantize(e: Encoded, stream=None):
+    """x_hat = s (v - z) as fp16 [rows, K]."""
+    torch = _torch()
+    y = torch.empty((e.rows, e.K), dtype=torch.float16, device=e.codes.device)
+    ec = e.c()
+    N.check(N.load().quartz_dequantize(C.byref(ec), y.data_ptr(), _stream(stream)), "quartz_dequantize")
+    return y
+
+
+def linear_workspace_size(M: int, N_: int, K: int, params: Params = Params()) -> int:
+    p = params.c()
+    return int(N.load().quartz_linear_workspace_size(M, N_, K, C.byref(p)))
+
+
+_OUT = {"float16": OUT_F16, "bfloat16": OUT_BF16, "float32": OUT_F32}
+
+
+def linear(a: Encoded, w: Encoded, bias=None, out_dtype=None, out=None, workspace=None,
+           partials_group: int | None = None, algo: int = ALGO_TCGEN05, stream=None):
+    """W4A4 QuaRTZ linear: y = dequant(a) @ dequant(w)^T (+ bias), computed as
+    exact integer group partials scaled by the 16-bit group scales.
+
+    Returns y, or (y, partials) when `partials_group` is given (int32 [M, N]
+    raw integer MMA sums of that 64-wide K group)."""
+    torch = _torch()
+    out_dtype = out_dtype or torch.float16
+    M, Nn = a.rows, w.rows
+    dev = a.codes.device
+    y = out if out is not None else torch.empty((M, Nn), dtype=out_dtype, device=dev)
+    y_type = _OUT[str(y.dtype).replace("torch.", "")]
+    if workspace is None:
+        workspace = torch.empty(max(linear_workspace_size(M, Nn, a.K, a.params), 16),
+                                dtype=torch.uint8, device=dev)
+    part = None
+    if partials_group is not None:
+        part = torch.empty((M, Nn), dtype=torch.int32, device=dev)
+    if bias is not None and not (bias.dtype == torch.float16 and bias.is_cuda and bias.numel() == Nn):
+        raise ValueError("bias must be a float16 CUDA tensor of N elements")
+    ac, wc = a.c(), w.c()
+    rc = N.load().quartz_linear_ex(
+        C.byref(ac), C.byref(wc), None if bias is None else bias.data_ptr(), y.data_ptr(), y_type,
+        None if part is None else part.data_ptr(), 0 if partials_group is None else partials_group,
+        algo, workspace.data_ptr(), workspace.numel() * workspace.element_size(), _stream(stream))
+    N.check(rc, "quartz_linear_ex")
+    return y if part is None else (y, part)
+
+
+def device_status(stream=None) -> int:
+    """Synchronise the stream; return (and clear) the library's device status."""
+    return int(N.load().quartz_device_status(_stream(stream)))
+
+
+def selftest_timeout(limit_ns: int, stream=None) -> int:
+    return int(N.load().quartz_selftest_timeout(limit_ns, _stream(stream)))

@@ -1,0 +1,210 @@
+// Host side of the C ABI declared in include/quartz.h: argument validation,
+// workspace carving and kernel launches.  Nothing here allocates device
+// memory or synchronises, except quartz_device_status.
+#include <cstring>
+
+#include "quartz_internal.h"
+
+namespace quartz {
+namespace {
+
+__device__ int g_device_error;
+
+constexpr int kMaxDevices = 64;
+int *g_error_ptr[kMaxDevices] = {};
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int32_t check_params(const quartz_params_t *p)
+{
+    if (!p) return QUARTZ_ERR_INVALID_ARG;
+    if (p->mode != QUARTZ_SYMMETRIC && p->mode != QUARTZ_ASYMMETRIC) return QUARTZ_ERR_INVALID_ARG;
+    if (p->group_s != 8 && p->group_s != 16 && p->group_s != 32 && p->group_s != 64)
+        return QUARTZ_ERR_INVALID_ARG;
+    if (p->group_q <= 0 || p->group_q % p->group_s != 0) return QUARTZ_ERR_INVALID_ARG;
+    if (p->group_q != 64) return QUARTZ_ERR_UNSUPPORTED;
+    return QUARTZ_OK;
+}
+
+int32_t check_shape(int64_t rows, int64_t K, const quartz_params_t *p)
+{
+    const int32_t rc = check_params(p);
+    if (rc) return rc;
+    if (rows < 0 || K <= 0 || K % p->group_q != 0) return QUARTZ_ERR_INVALID_ARG;
+    if (rows > (int64_t(1) << 31) || K > (int64_t(1) << 24)) return QUARTZ_ERR_UNSUPPORTED;
+    return QUARTZ_OK;
+}
+
+int32_t check_encoded(const quartz_encoded_t *e)
+{
+    if (!e) return QUARTZ_ERR_INVALID_ARG;
+    const int32_t rc = check_shape(e->rows, e->K, &e->p);
+    if (rc) return rc;
+    if (e->rows == 0) return QUARTZ_OK;
+    if (!e->codes || !e->flags || !e->scales) return QUARTZ_ERR_INVALID_ARG;
+    if (!aligned16(e->codes) || !aligned16(e->flags) || !aligned16(e->scales))
+        return QUARTZ_ERR_ALIGNMENT;
+    if (e->p.mode == QUARTZ_ASYMMETRIC) {
+        if (!e->zeros || !e->gsum) return QUARTZ_ERR_INVALID_ARG;
+        if (!aligned16(e->zeros) || !aligned16(e->gsum)) return QUARTZ_ERR_ALIGNMENT;
+    }
+    return QUARTZ_OK;
+}
+
+int32_t map_cuda(cudaError_t e) { return e == cudaSuccess ? QUARTZ_OK : QUARTZ_ERR_CUDA; }
+
+}  // namespace
+
+int *device_error_word()
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+    if (!g_error_ptr[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_device_error) != cudaSuccess) return nullptr;
+        g_error_ptr[dev] = static_cast<int *>(p);
+    }
+    return g_error_ptr[dev];
+}
+
+}  // namespace quartz
+
+using namespace quartz;
+
+extern "C" {
+
+const char *quartz_status_string(int32_t status)
+{
+    switch (status) {
+        case QUARTZ_OK: return "QUARTZ_OK";
+        case QUARTZ_ERR_INVALID_ARG: return "QUARTZ_ERR_INVALID_ARG";
+        case QUARTZ_ERR_ALIGNMENT: return "QUARTZ_ERR_ALIGNMENT";
+        case QUARTZ_ERR_UNSUPPORTED: return "QUARTZ_ERR_UNSUPPORTED";
+        case QUARTZ_ERR_CUDA: return "QUARTZ_ERR_CUDA";
+        case QUARTZ_ERR_TIMEOUT: return "QUARTZ_ERR_TIMEOUT";
+        case QUARTZ_ERR_WORKSPACE: return "QUARTZ_ERR_WORKSPACE";
+        default: return "QUARTZ_ERR_UNKNOWN";
+    }
+}
+
+int32_t quartz_version(void) { return (1 << 16) | 0; }
+
+int32_t quartz_encoded_sizes(int64_t rows, int64_t K, const quartz_params_t *p, size_t out[5])
+{
+    if (!out) return QUARTZ_ERR_INVALID_ARG;
+    const int32_t rc = check_shape(rows, K, p);
+    if (rc) return rc;
+    const int64_t G = K / p->group_q;
+    out[0] = static_cast<size_t>(rows * (K / 2));
+    out[1] = static_cast<size_t>(rows * (K / p->group_s));
+    out[2] = static_cast<size_t>(rows * G * 2);
+    out[3] = static_cast<size_t>(rows * G);
+    out[4] = static_cast<size_t>(rows * G * 4);
+    return QUARTZ_OK;
+}
+
+int32_t quartz_quantize(const void *x_f16, const quartz_encoded_t *out, void *stream)
+{
+    int32_t rc = check_encoded(out);
+    if (rc) return rc;
+    if (out->rows == 0) return QUARTZ_OK;
+    if (!x_f16) return QUARTZ_ERR_INVALID_ARG;
+    if (!aligned16(x_f16)) return QUARTZ_ERR_ALIGNMENT;
+    return map_cuda(launch_quantize(x_f16, out, static_cast<cudaStream_t>(stream)));
+}
+
+int32_t quartz_encode_weights(const void *w_f16, const quartz_encoded_t *out, void *stream)
+{
+    return quartz_quantize(w_f16, out, stream);
+}
+
+int32_t quartz_dequantize(const quartz_encoded_t *e, void *x_hat_f16, void *stream)
+{
+    int32_t rc = check_encoded(e);
+    if (rc) return rc;
+    if (e->rows == 0) return QUARTZ_OK;
+    if (!x_hat_f16) return QUARTZ_ERR_INVALID_ARG;
+    if (!aligned16(x_hat_f16)) return QUARTZ_ERR_ALIGNMENT;
+    return map_cuda(launch_dequantize(e, x_hat_f16, static_cast<cudaStream_t>(stream)));
+}
+
+size_t quartz_linear_workspace_size(int64_t M, int64_t N, int64_t K, const quartz_params_t *p)
+{
+    if (check_shape(M, K, p) != QUARTZ_OK || N <= 0 || N % 8 != 0) return 0;
+    return linear_workspace_bytes(M, N, K, p->mode);
+}
+
+int32_t quartz_linear_ex(const quartz_encoded_t *a, const quartz_encoded_t *w,
+                         const void *bias_f16, void *y, int32_t y_type, int32_t *partials,
+                         int32_t partials_group, int32_t algo, void *workspace,
+                         size_t workspace_bytes, void *stream)
+{
+    int32_t rc = check_encoded(a);
+    if (rc) return rc;
+    rc = check_encoded(w);
+    if (rc) return rc;
+    if (a->K != w->K || a->p.group_q != w->p.group_q || a->p.group_s != w->p.group_s ||
+        a->p.mode != w->p.mode)
+        return QUARTZ_ERR_INVALID_ARG;
+    const int64_t M = a->rows, N = w->rows, K = a->K;
+    if (N <= 0 || N % 8 != 0 || N > (int64_t(1) << 24)) return QUARTZ_ERR_INVALID_ARG;
+    if (y_type != QUARTZ_OUT_F16 && y_type != QUARTZ_OUT_BF16 && y_type != QUARTZ_OUT_F32)
+        return QUARTZ_ERR_INVALID_ARG;
+    if (algo != QUARTZ_ALGO_TCGEN05 && algo != QUARTZ_ALGO_SIMT) return QUARTZ_ERR_INVALID_ARG;
+    if (partials && (partials_group < 0 || partials_group >= K / a->p.group_q))
+        return QUARTZ_ERR_INVALID_ARG;
+    if (M * N >= (int64_t(1) << 40)) return QUARTZ_ERR_UNSUPPORTED;
+    if (M == 0) return QUARTZ_OK;
+    if (!y) return QUARTZ_ERR_INVALID_ARG;
+    if (!aligned16(y) || (bias_f16 && !aligned16(bias_f16)) || (partials && !aligned16(partials)))
+        return QUARTZ_ERR_ALIGNMENT;
+    const size_t need = linear_workspace_bytes(M, N, K, a->p.mode);
+    if (!workspace || workspace_bytes < need) return QUARTZ_ERR_WORKSPACE;
+    if (!aligned16(workspace)) return QUARTZ_ERR_ALIGNMENT;
+    int *dev_err = device_error_word();
+    if (!dev_err) return QUARTZ_ERR_CUDA;
+
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    LinearWorkspace ws;
+    linear_workspace_carve(workspace, M, N, K, a->p.mode, &ws);
+    cudaError_t e = launch_expand(a, ws.a_op, ws.a_side, ws.m_pad, 1, s);
+    if (e == cudaSuccess) e = launch_expand(w, ws.w_op, ws.w_side, ws.n_pad, 0, s);
+    if (e != cudaSuccess) return QUARTZ_ERR_CUDA;
+    if (algo == QUARTZ_ALGO_SIMT)
+        e = launch_gemm_simt(ws, M, N, K, a->p.mode, bias_f16, y, y_type, partials, partials_group, s);
+    else
+        e = launch_gemm_tcgen05(ws, M, N, K, a->p.mode, bias_f16, y, y_type, partials,
+                                partials_group, dev_err, s);
+    return map_cuda(e);
+}
+
+int32_t quartz_linear(const quartz_encoded_t *a, const quartz_encoded_t *w, const void *bias_f16,
+                      void *y, int32_t y_type, void *workspace, size_t workspace_bytes,
+                      void *stream)
+{
+    return quartz_linear_ex(a, w, bias_f16, y, y_type, nullptr, 0, QUARTZ_ALGO_TCGEN05, workspace,
+                            workspace_bytes, stream);
+}
+
+int32_t quartz_device_status(void *stream)
+{
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (cudaStreamSynchronize(s) != cudaSuccess) return QUARTZ_ERR_CUDA;
+    int *p = device_error_word();
+    if (!p) return QUARTZ_ERR_CUDA;
+    int v = 0;
+    const int zero = 0;
+    if (cudaMemcpy(&v, p, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return QUARTZ_ERR_CUDA;
+    if (cudaMemcpy(p, &zero, sizeof(int), cudaMemcpyHostToDevice) != cudaSuccess) return QUARTZ_ERR_CUDA;
+    return v == QUARTZ_DEV_TIMEOUT ? QUARTZ_ERR_TIMEOUT : QUARTZ_OK;
+}
+
+int32_t quartz_selftest_timeout(int64_t limit_ns, void *stream)
+{
+    if (limit_ns < 1000 || limit_ns > 10000000000ll) return QUARTZ_ERR_INVALID_ARG;
+    int *dev_err = device_error_word();
+    if (!dev_err) return QUARTZ_ERR_CUDA;
+    return map_cuda(launch_selftest_timeout(limit_ns, dev_err, static_cast<cudaStream_t>(stream)));
+}
+
+}  // extern "C"

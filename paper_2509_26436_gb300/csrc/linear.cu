@@ -1,0 +1,734 @@
+// QuaRTZ W4A4 linear layer for sm_103a (Section 4.4; Appendix C scales).
+//
+// Pipeline of one quartz_linear call:
+//   1. expand: the packed 4-bit codes and per-subgroup FLAGs of both operands
+//      are decoded to v = sgn(c)(|c| << FLAG) and written as fp16 (exact: every
+//      decoded value has at most 3 significant bits and |v| <= 112), together
+//      with the group scales (and zero-point side values) transposed to
+//      [G][rows] fp32 for contiguous per-group access.  This pass is
+//      HBM-bound and touches each operand element once, instead of once per
+//      output tile that reads it.
+//   2. GEMM: a persistent warp-specialised tcgen05 kernel.  One TMA warp
+//      streams 128x64 A and 256x64 W tiles (one 64-wide quantization group
+//      per stage, 128-byte swizzle) into a 4-stage shared-memory ring; one
+//      thread issues kind::f16 MMAs into a fresh fp32 TMEM accumulator for
+//      every group (double-buffered, 2 x 256 columns), so each accumulator
+//      holds exactly P_g = sum_{k in g} v_a v_w; eight epilogue warps read
+//      P_g with tcgen05.ld and fold it into the register-resident output as
+//      y += s_a * (s_w * P_g) with packed f32x2 arithmetic.
+//
+// Exactness of P_g: the products v_a * v_w are integers of magnitude at most
+// 112^2 = 12544 and every partial sum over a group is an integer of
+// magnitude at most 64 * 12544 < 2^20, all exactly representable in the fp32
+// accumulator, so the tensor-core sum equals the integer sum.  (sm_103a has
+// no integer tcgen05 MMA kind; this is why the integer GEMM runs on the f16
+// pipe.)
+#include <cuda.h>
+#include <cuda_fp16.h>
+#include <cuda_bf16.h>
+
+#include "ptx.cuh"
+#include "quartz_internal.h"
+
+namespace quartz {
+namespace {
+
+constexpr int kGroupQ = 64;
+
+// ---------------------------------------------------------------------------
+// 1. expand
+// ---------------------------------------------------------------------------
+template <int GS>
+__global__ void __launch_bounds__(256) expand_kernel(const uint32_t *__restrict__ codes,
+                                                     const uint8_t *__restrict__ flags,
+                                                     int64_t n_chunks, uint4 *__restrict__ op)
+{
+    const int64_t c = static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x;
+    if (c >= n_chunks) return;
+    const uint32_t word = codes[c];
+    const int flag = flags[(c * 8) / GS];
+    const int mul = 1 << flag;
+    uint32_t o[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int c0 = static_cast<int>(word << (28 - 8 * i)) >> 28;
+        const int c1 = static_cast<int>(word << (24 - 8 * i)) >> 28;
+        const __half2 h = __floats2half2_rn(static_cast<float>(c0 * mul), static_cast<float>(c1 * mul));
+        o[i] = *reinterpret_cast<const uint32_t *>(&h);
+    }
+    op[c] = make_uint4(o[0], o[1], o[2], o[3]);
+}
+
+// side[0][g][r] = s[r, g]; asymmetric adds side[1] = z and side[2] =
+// (is_a ? 64 z - gsum : gsum), so that the epilogue's integer correction is
+// P + z_w * (64 z_a - A_g) - z_a * W_g.  Rows in [rows, rows_pad) are 0.
+__global__ void side_kernel(const __half *__restrict__ scales, const int8_t *__restrict__ zeros,
+                            const int32_t *__restrict__ gsum, int64_t rows, int64_t rows_pad,
+                            int G, int nside, int is_a, float *__restrict__ side)
+{
+    const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    const int64_t total = rows_pad * G;
+    if (i >= total) return;
+    const int64_t g = i / rows_pad;
+    const int64_t r = i - g * rows_pad;
+    const bool in = r < rows;
+    side[i] = in ? __half2float(scales[r * G + g]) : 0.f;
+    if (nside > 1) {
+        const float z = in ? static_cast<float>(zeros[r * G + g]) : 0.f;
+        const float gs = in ? static_cast<float>(gsum[r * G + g]) : 0.f;
+        side[total + i] = z;
+        side[2 * total + i] = is_a ? (static_cast<float>(kGroupQ) * z - gs) : gs;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// 2. tcgen05 GEMM
+// ---------------------------------------------------------------------------
+constexpr int BM = 128;
+constexpr int BN = 256;
+constexpr int BK = kGroupQ;
+constexpr int kStages = 4;
+constexpr int kABytes = BM * BK * 2;
+constexpr int kBBytes = BN * BK * 2;
+constexpr int kStageBytes = kABytes + kBBytes;
+constexpr int kEpiWarps = 8;                  // warpgroups 0 and 1
+constexpr int kThreads = (kEpiWarps + 4) * 32;  // warpgroup 2: producer, MMA, 2 idle warps
+constexpr int kProducerWarp = kEpiWarps;
+constexpr int kMmaWarp = kEpiWarps + 1;
+// Register split (setmaxnreg): the launch gives 65536 / 384 -> 168 per
+// thread; warpgroup 2 drops to 56 so the two epilogue warpgroups can hold
+// 224 (2*128*224 + 128*56 = 384*168).
+constexpr uint32_t kRegsEpilogue = 224;
+constexpr uint32_t kRegsControl = 56;
+static_assert(2 * 128 * kRegsEpilogue + 128 * kRegsControl <= kThreads * 168, "register split");
+constexpr uint32_t kTmemCols = 512;   // two fp32 accumulators of 256 columns
+constexpr int kColsPerWarp = BN / 2;  // two warps share each 32-lane TMEM quarter
+
+struct GemmArgs {
+    const float *a_side;  // [nside][G][m_pad]
+    const float *w_side;  // [nside][G][n_pad]
+    int64_t m_pad, n_pad;
+    int M, N, G;
+    int tiles_n, num_tiles;
+    const __half *bias;
+    void *y;
+    int y_type;
+    int32_t *partials;
+    int partials_group;
+    int *dev_err;
+};
+
+template <int NSIDE>
+struct Smem {
+    static constexpr int kOperands = 0;
+    static constexpr int kSide = kStages * kStageBytes;
+    static constexpr int kSideBytes = kEpiWarps * 2 * NSIDE * kColsPerWarp * 4;
+    static constexpr int kBars = kSide + kSideBytes;
+    static constexpr int kNumBars = 2 * kStages + 4 + 1;  // full, empty, acc_full x2, acc_empty x2, drain
+    static constexpr int kMisc = kBars + kNumBars * 8;
+    static constexpr int kTotal = kMisc + 16;
+    static constexpr int kAlloc = kTotal + 1024;  // slack to align the base to 1024 bytes
+};
+
+__device__ __forceinline__ float4 ldg_f4(const float *p)
+{
+    return __ldg(reinterpret_cast<const float4 *>(p));
+}
+
+template <int OUT>
+__device__ __forceinline__ void store_row8(void *y, int64_t off, const float (&v)[8])
+{
+    if (OUT == QUARTZ_OUT_F16) {
+        uint32_t o[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const __half2 h = __floats2half2_rn(v[2 * i], v[2 * i + 1]);
+            o[i] = *reinterpret_cast<const uint32_t *>(&h);
+        }
+        *reinterpret_cast<uint4 *>(static_cast<__half *>(y) + off) = make_uint4(o[0], o[1], o[2], o[3]);
+    } else if (OUT == QUARTZ_OUT_BF16) {
+        uint32_t o[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const __nv_bfloat162 h = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+            o[i] = *reinterpret_cast<const uint32_t *>(&h);
+        }
+        *reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(y) + off) = make_uint4(o[0], o[1], o[2], o[3]);
+    } else {
+        float4 *d = reinterpret_cast<float4 *>(static_cast<float *>(y) + off);
+        d[0] = make_float4(v[0], v[1], v[2], v[3]);
+        d[1] = make_float4(v[4], v[5], v[6], v[7]);
+    }
+}
+
+template <int MODE, int OUT, bool DUMP>
+__global__ void __launch_bounds__(kThreads, 1)
+    gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tmap_a,
+                        const __grid_constant__ CUtensorMap tmap_w, const GemmArgs args)
+{
+    constexpr int NSIDE = (MODE == QUARTZ_ASYMMETRIC) ? 3 : 1;
+    using L = Smem<NSIDE>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const uint32_t smem_base = smem_u32(smem);
+    const uint32_t bar_base = smem_base + L::kBars;
+    auto full_bar = [&](int s) { return bar_base + 8u * s; };
+    auto empty_bar = [&](int s) { return bar_base + 8u * (kStages + s); };
+    auto acc_full_bar = [&](int b) { return bar_base + 8u * (2 * kStages + b); };
+    auto acc_empty_bar = [&](int b) { return bar_base + 8u * (2 * kStages + 2 + b); };
+    const uint32_t drain_bar = bar_base + 8u * (2 * kStages + 4);
+    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(smem + L::kMisc);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + L::kMisc + 4);
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(full_bar(s), 1);
+            mbar_init(empty_bar(s), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(acc_full_bar(b), 1);
+            mbar_init(acc_empty_bar(b), kEpiWarps);
+        }
+        mbar_init(drain_bar, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == kMmaWarp) {
+        tmem_alloc(smem_u32(tmem_holder), kTmemCols);
+        tmem_relinquish();
+    }
+    if (warp == kProducerWarp && lane == 0) {
+        tma_prefetch_desc(&tmap_a);
+        tma_prefetch_desc(&tmap_w);
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_holder;
+    const int G = args.G;
+
+    if (warp >= kEpiWarps) {
+      regs_decrease<kRegsControl>();
+      if (warp == kProducerWarp) {
+        // ------------------------------------------------------------------
+        // TMA producer: one stage = one 64-wide group of A (128 rows) and W
+        // (256 rows).  Rows past M or N are zero-filled by the tensor map.
+        // ------------------------------------------------------------------
+        if (lane == 0) {
+            int it = 0;
+            bool ok = true;
+            for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
+                const int mt = tile / args.tiles_n;
+                const int nt = tile - mt * args.tiles_n;
+                for (int g = 0; g < G; ++g, ++it) {
+                    const int s = it % kStages;
+                    if (it >= kStages &&
+                        !mbar_wait_bounded(empty_bar(s), ((it / kStages) - 1) & 1, abort_flag,
+                                           args.dev_err, kWaitLimitNs)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t sa = smem_base + L::kOperands + s * kStageBytes;
+                    mbar_arrive_expect_tx(full_bar(s), kStageBytes);
+                    tma_load_2d(sa, &tmap_a, g * BK, mt * BM, full_bar(s));
+                    tma_load_2d(sa + kABytes, &tmap_w, g * BK, nt * BN, full_bar(s));
+                }
+            }
+            // Never leave the CTA with copies in flight: wait for the last
+            // load issued into every stage (bounded, even after an abort).
+            int zero = 0;
+            for (int s = 0; s < kStages && s < it; ++s) {
+                const int last = it - 1 - ((it - 1 - s) % kStages);
+                mbar_wait_bounded(full_bar(s), (last / kStages) & 1, &zero, args.dev_err, kWaitLimitNs);
+            }
+        }
+        __syncwarp();
+      } else if (warp == kMmaWarp) {
+        // ------------------------------------------------------------------
+        // MMA issuer: 4 x (M=128, N=256, K=16) kind::f16 MMAs per group into
+        // a fresh accumulator (first MMA overwrites), then two commits: one
+        // frees the operand stage, one hands P_g to the epilogue.
+        // ------------------------------------------------------------------
+        if (lane == 0) {
+            constexpr uint32_t idesc = idesc_f16_f32(BM, BN);
+            int it = 0;
+            bool ok = true;
+            for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
+                for (int g = 0; g < G; ++g, ++it) {
+                    const int s = it % kStages;
+                    const int b = it & 1;
+                    if (!mbar_wait_bounded(full_bar(s), (it / kStages) & 1, abort_flag, args.dev_err,
+                                           kWaitLimitNs)) {
+                        ok = false;
+                        break;
+                    }
+                    if (it >= 2 && !mbar_wait_bounded(acc_empty_bar(b), ((it >> 1) - 1) & 1,
+                                                      abort_flag, args.dev_err, kWaitLimitNs)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t sa = smem_base + L::kOperands + s * kStageBytes;
+                    const uint32_t d = tmem_base + static_cast<uint32_t>(b * BN);
+#pragma unroll
+                    for (int kk = 0; kk < BK / 16; ++kk) {
+                        const uint64_t adesc = sdesc_k_major_sw128(sa + kk * 32);
+                        const uint64_t bdesc = sdesc_k_major_sw128(sa + kABytes + kk * 32);
+                        mma_f16_ss(d, adesc, bdesc, idesc, kk > 0 ? 1u : 0u);
+                    }
+                    mma_commit(empty_bar(s));
+                    mma_commit(acc_full_bar(b));
+                }
+            }
+            // Make sure no MMA is still writing TMEM before it is freed.
+            mma_commit(drain_bar);
+            int zero = 0;
+            mbar_wait_bounded(drain_bar, 0, &zero, args.dev_err, kWaitLimitNs);
+        }
+        __syncwarp();
+      }
+    } else {
+        regs_increase<kRegsEpilogue>();
+        // ------------------------------------------------------------------
+        // Epilogue: warp w owns TMEM lanes 32*(w%4).. (tile rows) and columns
+        // [128*(w/4), +128).  Per group: y += s_a * (s_w * P_g); asymmetric
+        // first corrects P_g by the zero-point terms (exact integers in fp32).
+        // ------------------------------------------------------------------
+        const int quarter = warp & 3;
+        const int colh = warp >> 2;
+        const int row = quarter * 32 + lane;
+        float *wbuf = reinterpret_cast<float *>(smem + L::kSide) + warp * (2 * NSIDE * kColsPerWarp);
+        const int64_t a_plane = args.m_pad * G;
+        const int64_t w_plane = args.n_pad * G;
+
+        int tile = blockIdx.x;
+        int g = 0;
+        // side values of the (tile, g) about to be processed, prefetched one group ahead
+        float4 nxt_w[NSIDE];
+        float nxt_a[NSIDE];
+        auto fetch = [&](int t, int gg) {
+            const int mt = t / args.tiles_n;
+            const int nt = t - mt * args.tiles_n;
+            const int64_t col = static_cast<int64_t>(nt) * BN + colh * kColsPerWarp + 4 * lane;
+            const int64_t r = static_cast<int64_t>(mt) * BM + row;
+#pragma unroll
+            for (int sd = 0; sd < NSIDE; ++sd) {
+                nxt_w[sd] = ldg_f4(args.w_side + sd * w_plane + static_cast<int64_t>(gg) * args.n_pad + col);
+                nxt_a[sd] = __ldg(args.a_side + sd * a_plane + static_cast<int64_t>(gg) * args.m_pad + r);
+            }
+        };
+        if (tile < args.num_tiles) fetch(tile, 0);
+
+        float2 acc[kColsPerWarp / 2];
+        int it = 0;
+        bool ok = true;
+        for (; tile < args.num_tiles && ok; tile += gridDim.x) {
+            const int mt = tile / args.tiles_n;
+            const int nt = tile - mt * args.tiles_n;
+#pragma unroll
+            for (int j = 0; j < kColsPerWarp / 2; ++j) acc[j] = make_float2(0.f, 0.f);
+            for (g = 0; g < G; ++g, ++it) {
+                const int b = it & 1;
+                float *sb = wbuf + b * (NSIDE * kColsPerWarp);
+                float cur_a[NSIDE];
+#pragma unroll
+                for (int sd = 0; sd < NSIDE; ++sd) {
+                    reinterpret_cast<float4 *>(sb + sd * kColsPerWarp)[lane] = nxt_w[sd];
+                    cur_a[sd] = nxt_a[sd];
+                }
+                __syncwarp();
+                {
+                    int nt2 = tile, ng = g + 1;
+                    if (ng == G) {
+                        ng = 0;
+                        nt2 = tile + gridDim.x;
+                    }
+                    if (nt2 < args.num_tiles) fetch(nt2, ng);
+                }
+                if (!mbar_wait_bounded(acc_full_bar(b), (it >> 1) & 1, abort_flag, args.dev_err,
+                                       kWaitLimitNs)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const float2 sa2 = make_float2(cur_a[0], cur_a[0]);
+                const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
+                                       static_cast<uint32_t>(b * BN + colh * kColsPerWarp);
+#pragma unroll
+                for (int c = 0; c < kColsPerWarp / 32; ++c) {
+                    uint32_t r[32];
+                    tmem_ld_32x32b_x32(taddr + c * 32, r);
+                    tmem_wait_ld();
+                    if (DUMP && g == args.partials_group) {
+                        const int64_t m = static_cast<int64_t>(mt) * BM + row;
+                        const int64_t n0 = static_cast<int64_t>(nt) * BN + colh * kColsPerWarp + c * 32;
+                        if (m < args.M) {
+                            for (int j = 0; j < 32; ++j)
+                                if (n0 + j < args.N)
+                                    args.partials[m * args.N + n0 + j] = __float2int_rn(__uint_as_float(r[j]));
+                        }
+                    }
+#pragma unroll
+                    for (int j4 = 0; j4 < 8; ++j4) {
+                        const int col = c * 32 + j4 * 4;
+                        const float4 sw = *reinterpret_cast<const float4 *>(sb + col);
+                        float2 p0 = make_float2(__uint_as_float(r[j4 * 4 + 0]), __uint_as_float(r[j4 * 4 + 1]));
+                        float2 p1 = make_float2(__uint_as_float(r[j4 * 4 + 2]), __uint_as_float(r[j4 * 4 + 3]));
+                        if (MODE == QUARTZ_ASYMMETRIC) {
+                            const float4 zw = *reinterpret_cast<const float4 *>(sb + kColsPerWarp + col);
+                            const float4 gw = *reinterpret_cast<const float4 *>(sb + 2 * kColsPerWarp + col);
+                            const float2 ua = make_float2(cur_a[2], cur_a[2]);
+                            const float2 nza = make_float2(-cur_a[1], -cur_a[1]);
+                            p0 = __ffma2_rn(make_float2(zw.x, zw.y), ua, p0);
+                            p1 = __ffma2_rn(make_float2(zw.z, zw.w), ua, p1);
+                            p0 = __ffma2_rn(nza, make_float2(gw.x, gw.y), p0);
+                            p1 = __ffma2_rn(nza, make_float2(gw.z, gw.w), p1);
+                        }
+                        const float2 t0 = __fmul2_rn(p0, make_float2(sw.x, sw.y));
+                        const float2 t1 = __fmul2_rn(p1, make_float2(sw.z, sw.w));
+                        acc[col / 2] = __ffma2_rn(t0, sa2, acc[col / 2]);
+                        acc[col / 2 + 1] = __ffma2_rn(t1, sa2, acc[col / 2 + 1]);
+                    }
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(acc_empty_bar(b));
+            }
+            if (!ok) break;
+            // ---- store the finished tile row segment ------------------------
+            const int64_t m = static_cast<int64_t>(mt) * BM + row;
+            const int64_t nbase = static_cast<int64_t>(nt) * BN + colh * kColsPerWarp;
+            if (m < args.M) {
+#pragma unroll
+                for (int c8 = 0; c8 < kColsPerWarp / 8; ++c8) {
+                    const int64_t n = nbase + c8 * 8;
+                    if (n < args.N) {
+                        float v[8];
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) {
+                            v[2 * i] = acc[c8 * 4 + i].x;
+                            v[2 * i + 1] = acc[c8 * 4 + i].y;
+                        }
+                        if (args.bias) {
+                            const uint4 braw = __ldg(reinterpret_cast<const uint4 *>(args.bias + n));
+                            const uint32_t bw[4] = {braw.x, braw.y, braw.z, braw.w};
+#pragma unroll
+                            for (int i = 0; i < 4; ++i) {
+                                const float2 bf = __half22float2(*reinterpret_cast<const __half2 *>(&bw[i]));
+                                v[2 * i] = __fadd_rn(v[2 * i], bf.x);
+                                v[2 * i + 1] = __fadd_rn(v[2 * i + 1], bf.y);
+                            }
+                        }
+                        store_row8<OUT>(args.y, m * args.N + n, v);
+                    }
+                }
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == kMmaWarp) {
+        tc_fence_after();
+        tmem_dealloc(tmem_base, kTmemCols);
+    }
+}
+
+// ---------------------------------------------------------------------------
+// 3. SIMT GEMM: same decoded operands, same epilogue arithmetic, CUDA cores.
+//    64x64 output tile per 256-thread block, 4x4 outputs per thread.
+// ---------------------------------------------------------------------------
+template <int MODE, int OUT>
+__global__ void __launch_bounds__(256) gemm_simt_kernel(const __half *__restrict__ a_op,
+                                                        const __half *__restrict__ w_op,
+                                                        const GemmArgs args, int K)
+{
+    __shared__ int16_t sa[64][kGroupQ + 2];
+    __shared__ int16_t sw[64][kGroupQ + 2];
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+    const int m0 = blockIdx.y * 64, n0 = blockIdx.x * 64;
+    float y[4][4] = {};
+    const int64_t a_plane = args.m_pad * args.G;
+    const int64_t w_plane = args.n_pad * args.G;
+    for (int g = 0; g < args.G; ++g) {
+        for (int i = threadIdx.x; i < 64 * kGroupQ; i += 256) {
+            const int r = i / kGroupQ, k = i % kGroupQ;
+            const int64_t kk = static_cast<int64_t>(g) * kGroupQ + k;
+            sa[r][k] = (m0 + r < args.M) ? static_cast<int16_t>(__half2float(a_op[(int64_t)(m0 + r) * K + kk])) : 0;
+            sw[r][k] = (n0 + r < args.N) ? static_cast<int16_t>(__half2float(w_op[(int64_t)(n0 + r) * K + kk])) : 0;
+        }
+        __syncthreads();
+        int p[4][4] = {};
+        for (int k = 0; k < kGroupQ; ++k)
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) p[i][j] += sa[ty * 4 + i][k] * sw[tx * 4 + j][k];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int m = m0 + ty * 4 + i;
+            const float s_a = args.a_side[static_cast<int64_t>(g) * args.m_pad + m];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const int n = n0 + tx * 4 + j;
+                if (m >= args.M || n >= args.N) continue;
+                float P = static_cast<float>(p[i][j]);
+                if (args.partials && g == args.partials_group) args.partials[(int64_t)m * args.N + n] = p[i][j];
+                if (MODE == QUARTZ_ASYMMETRIC) {
+                    const float za = args.a_side[a_plane + (int64_t)g * args.m_pad + m];
+                    const float ua = args.a_side[2 * a_plane + (int64_t)g * args.m_pad + m];
+                    const float zw = args.w_side[w_plane + (int64_t)g * args.n_pad + n];
+                    const float gw = args.w_side[2 * w_plane + (int64_t)g * args.n_pad + n];
+                    P = __fmaf_rn(zw, ua, P);
+                    P = __fmaf_rn(-za, gw, P);
+                }
+                const float t = __fmul_rn(P, args.w_side[static_cast<int64_t>(g) * args.n_pad + n]);
+                y[i][j] = __fmaf_rn(t, s_a, y[i][j]);
+            }
+        }
+        __syncthreads();
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int m = m0 + ty * 4 + i;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int n = n0 + tx * 4 + j;
+            if (m >= args.M || n >= args.N) continue;
+            float v = y[i][j];
+            if (args.bias) v = __fadd_rn(v, __half2float(args.bias[n]));
+            const int64_t off = (int64_t)m * args.N + n;
+            if (OUT == QUARTZ_OUT_F16) static_cast<__half *>(args.y)[off] = __float2half_rn(v);
+            else if (OUT == QUARTZ_OUT_BF16) static_cast<__nv_bfloat16 *>(args.y)[off] = __float2bfloat16_rn(v);
+            else static_cast<float *>(args.y)[off] = v;
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
+size_t align256(size_t v) { return (v + 255) & ~size_t(255); }
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                  const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                  const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_tiled_fn()
+{
+    static EncodeTiledFn fn = nullptr;
+    if (!fn) {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    }
+    return fn;
+}
+
+// K-major fp16 operand [rows, K] read in boxes of [box_rows, 64] with the
+// 128-byte swizzle; out-of-range rows read as zero.
+bool make_operand_map(CUtensorMap *m, const void *base, int64_t rows, int64_t K, int box_rows)
+{
+    EncodeTiledFn fn = encode_tiled_fn();
+    if (!fn) return false;
+    const cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(rows)};
+    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(K) * 2};
+    const cuuint32_t box[2] = {static_cast<cuuint32_t>(BK), static_cast<cuuint32_t>(box_rows)};
+    const cuuint32_t estr[2] = {1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void *>(base), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int num_sms()
+{
+    int dev = 0, n = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    return n > 0 ? n : 1;
+}
+
+template <int MODE, int OUT>
+cudaError_t launch_tc(const CUtensorMap &ta, const CUtensorMap &tw, const GemmArgs &args,
+                      cudaStream_t s)
+{
+    constexpr int NSIDE = (MODE == QUARTZ_ASYMMETRIC) ? 3 : 1;
+    constexpr int smem = Smem<NSIDE>::kAlloc;
+    static_assert(smem <= 227 * 1024, "shared memory budget");
+    auto kern = args.partials ? gemm_tcgen05_kernel<MODE, OUT, true> : gemm_tcgen05_kernel<MODE, OUT, false>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    const int grid = args.num_tiles < num_sms() ? args.num_tiles : num_sms();
+    kern<<<grid, kThreads, smem, s>>>(ta, tw, args);
+    return cudaGetLastError();
+}
+
+template <int MODE>
+cudaError_t launch_tc_out(const CUtensorMap &ta, const CUtensorMap &tw, const GemmArgs &args,
+                          int y_type, cudaStream_t s)
+{
+    switch (y_type) {
+        case QUARTZ_OUT_F16: return launch_tc<MODE, QUARTZ_OUT_F16>(ta, tw, args, s);
+        case QUARTZ_OUT_BF16: return launch_tc<MODE, QUARTZ_OUT_BF16>(ta, tw, args, s);
+        default: return launch_tc<MODE, QUARTZ_OUT_F32>(ta, tw, args, s);
+    }
+}
+
+template <int MODE, int OUT>
+cudaError_t launch_simt(const LinearWorkspace &ws, const GemmArgs &args, int K, cudaStream_t s)
+{
+    dim3 grid(static_cast<unsigned>((args.N + 63) / 64), static_cast<unsigned>((args.M + 63) / 64));
+    gemm_simt_kernel<MODE, OUT><<<grid, 256, 0, s>>>(static_cast<const __half *>(ws.a_op),
+                                                     static_cast<const __half *>(ws.w_op), args, K);
+    return cudaGetLastError();
+}
+
+template <int MODE>
+cudaError_t launch_simt_out(const LinearWorkspace &ws, const GemmArgs &args, int K, int y_type,
+                            cudaStream_t s)
+{
+    switch (y_type) {
+        case QUARTZ_OUT_F16: return launch_simt<MODE, QUARTZ_OUT_F16>(ws, args, K, s);
+        case QUARTZ_OUT_BF16: return launch_simt<MODE, QUARTZ_OUT_BF16>(ws, args, K, s);
+        default: return launch_simt<MODE, QUARTZ_OUT_F32>(ws, args, K, s);
+    }
+}
+
+GemmArgs make_args(const LinearWorkspace &ws, int64_t M, int64_t N, int64_t K, const void *bias,
+                   void *y, int y_type, int32_t *partials, int partials_group, int *dev_err)
+{
+    GemmArgs a;
+    a.a_side = ws.a_side;
+    a.w_side = ws.w_side;
+    a.m_pad = ws.m_pad;
+    a.n_pad = ws.n_pad;
+    a.M = static_cast<int>(M);
+    a.N = static_cast<int>(N);
+    a.G = static_cast<int>(K / kGroupQ);
+    a.tiles_n = static_cast<int>((N + BN - 1) / BN);
+    a.num_tiles = static_cast<int>((M + BM - 1) / BM) * a.tiles_n;
+    a.bias = static_cast<const __half *>(bias);
+    a.y = y;
+    a.y_type = y_type;
+    a.partials = partials;
+    a.partials_group = partials_group;
+    a.dev_err = dev_err;
+    return a;
+}
+
+}  // namespace
+
+size_t linear_workspace_bytes(int64_t M, int64_t N, int64_t K, int mode)
+{
+    const int nside = mode == QUARTZ_ASYMMETRIC ? 3 : 1;
+    const int64_t G = K / kGroupQ;
+    size_t b = align256(static_cast<size_t>(M) * K * 2);
+    b += align256(static_cast<size_t>(N) * K * 2);
+    b += align256(static_cast<size_t>(nside) * G * round_up(M > 0 ? M : 1, BM) * 4);
+    b += align256(static_cast<size_t>(nside) * G * round_up(N, BN) * 4);
+    return b;
+}
+
+void linear_workspace_carve(void *base, int64_t M, int64_t N, int64_t K, int mode,
+                            LinearWorkspace *ws)
+{
+    const int nside = mode == QUARTZ_ASYMMETRIC ? 3 : 1;
+    const int64_t G = K / kGroupQ;
+    uint8_t *p = static_cast<uint8_t *>(base);
+    ws->nside = nside;
+    ws->m_pad = round_up(M > 0 ? M : 1, BM);
+    ws->n_pad = round_up(N, BN);
+    ws->a_op = p;
+    p += align256(static_cast<size_t>(M) * K * 2);
+    ws->w_op = p;
+    p += align256(static_cast<size_t>(N) * K * 2);
+    ws->a_side = reinterpret_cast<float *>(p);
+    p += align256(static_cast<size_t>(nside) * G * ws->m_pad * 4);
+    ws->w_side = reinterpret_cast<float *>(p);
+}
+
+cudaError_t launch_expand(const quartz_encoded_t *e, void *op, float *side, int64_t rows_pad,
+                          int is_a, cudaStream_t s)
+{
+    const int64_t n_chunks = e->rows * e->K / 8;
+    if (n_chunks > 0) {
+        const unsigned blocks = static_cast<unsigned>((n_chunks + 255) / 256);
+        const uint32_t *codes = reinterpret_cast<const uint32_t *>(e->codes);
+        uint4 *o = static_cast<uint4 *>(op);
+        switch (e->p.group_s) {
+            case 8: expand_kernel<8><<<blocks, 256, 0, s>>>(codes, e->flags, n_chunks, o); break;
+            case 16: expand_kernel<16><<<blocks, 256, 0, s>>>(codes, e->flags, n_chunks, o); break;
+            case 32: expand_kernel<32><<<blocks, 256, 0, s>>>(codes, e->flags, n_chunks, o); break;
+            default: expand_kernel<64><<<blocks, 256, 0, s>>>(codes, e->flags, n_chunks, o); break;
+        }
+        cudaError_t err = cudaGetLastError();
+        if (err != cudaSuccess) return err;
+    }
+    const int G = static_cast<int>(e->K / kGroupQ);
+    const int nside = e->p.mode == QUARTZ_ASYMMETRIC ? 3 : 1;
+    const int64_t total = rows_pad * G;
+    side_kernel<<<static_cast<unsigned>((total + 255) / 256), 256, 0, s>>>(
+        reinterpret_cast<const __half *>(e->scales), e->zeros, e->gsum, e->rows, rows_pad, G,
+        nside, is_a, side);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_gemm_tcgen05(const LinearWorkspace &ws, int64_t M, int64_t N, int64_t K,
+                                int mode, const void *bias, void *y, int y_type,
+                                int32_t *partials, int partials_group, int *dev_err,
+                                cudaStream_t s)
+{
+    if (M == 0) return cudaSuccess;
+    CUtensorMap ta, tw;
+    if (!make_operand_map(&ta, ws.a_op, M, K, BM) || !make_operand_map(&tw, ws.w_op, N, K, BN))
+        return cudaErrorInvalidValue;
+    const GemmArgs args = make_args(ws, M, N, K, bias, y, y_type, partials, partials_group, dev_err);
+    return mode == QUARTZ_ASYMMETRIC ? launch_tc_out<QUARTZ_ASYMMETRIC>(ta, tw, args, y_type, s)
+                                     : launch_tc_out<QUARTZ_SYMMETRIC>(ta, tw, args, y_type, s);
+}
+
+cudaError_t launch_gemm_simt(const LinearWorkspace &ws, int64_t M, int64_t N, int64_t K, int mode,
+                             const void *bias, void *y, int y_type, int32_t *partials,
+                             int partials_group, cudaStream_t s)
+{
+    if (M == 0) return cudaSuccess;
+    const GemmArgs args = make_args(ws, M, N, K, bias, y, y_type, partials, partials_group, nullptr);
+    return mode == QUARTZ_ASYMMETRIC
+               ? launch_simt_out<QUARTZ_ASYMMETRIC>(ws, args, static_cast<int>(K), y_type, s)
+               : launch_simt_out<QUARTZ_SYMMETRIC>(ws, args, static_cast<int>(K), y_type, s);
+}
+
+// ---------------------------------------------------------------------------
+// failure-detection self-test: a wait that nothing ever satisfies
+// ---------------------------------------------------------------------------
+namespace {
+__global__ void selftest_timeout_kernel(uint64_t limit_ns, int *dev_err)
+{
+    __shared__ __align__(8) uint64_t bar;
+    __shared__ int abort_flag;
+    if (threadIdx.x == 0) {
+        mbar_init(smem_u32(&bar), 1);
+        abort_flag = 0;
+        fence_mbar_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) mbar_wait_bounded(smem_u32(&bar), 0, &abort_flag, dev_err, limit_ns);
+    __syncthreads();
+}
+}  // namespace
+
+cudaError_t launch_selftest_timeout(int64_t limit_ns, int *dev_err, cudaStream_t s)
+{
+    selftest_timeout_kernel<<<1, 32, 0, s>>>(static_cast<uint64_t>(limit_ns), dev_err);
+    return cudaGetLastError();
+}
+
+}  // namespace quartz

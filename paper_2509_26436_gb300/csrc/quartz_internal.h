@@ -1,0 +1,51 @@
+// Declarations shared by the translation units of libquartz (not installed).
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "../../include/quartz.h"
+
+namespace quartz {
+
+// Values of the library's device error word (0 = no error).
+constexpr int QUARTZ_DEV_OK = 0;
+constexpr int QUARTZ_DEV_TIMEOUT = 1;
+
+// Upper bound on any single mbarrier wait inside a kernel.  No legitimate
+// wait on a healthy GPU comes near it; it only turns a would-be hang into an
+// error status.
+constexpr uint64_t kWaitLimitNs = 2000000000ull;
+
+// Device error word of the current device (see api.cu).
+int *device_error_word();
+
+// Encoder / decoder launches (quantize.cu).  Arguments are pre-validated.
+cudaError_t launch_quantize(const void *x, const quartz_encoded_t *out, cudaStream_t s);
+cudaError_t launch_dequantize(const quartz_encoded_t *e, void *y, cudaStream_t s);
+
+// Linear-layer workspace and launches (linear.cu).
+struct LinearWorkspace {
+    void *a_op;      // fp16 [M, K]  decoded activations, tensor-core input
+    void *w_op;      // fp16 [N, K]  decoded weights
+    float *a_side;   // fp32 [nside][G][Mpad]  scale (and z, gsum when asymmetric)
+    float *w_side;   // fp32 [nside][G][Npad]
+    int64_t m_pad, n_pad;
+    int nside;
+};
+size_t linear_workspace_bytes(int64_t M, int64_t N, int64_t K, int mode);
+void linear_workspace_carve(void *base, int64_t M, int64_t N, int64_t K, int mode,
+                            LinearWorkspace *ws);
+cudaError_t launch_expand(const quartz_encoded_t *e, void *op, float *side, int64_t rows_pad,
+                          int is_a, cudaStream_t s);
+cudaError_t launch_gemm_tcgen05(const LinearWorkspace &ws, int64_t M, int64_t N, int64_t K,
+                                int mode, const void *bias, void *y, int y_type,
+                                int32_t *partials, int partials_group, int *dev_err,
+                                cudaStream_t s);
+cudaError_t launch_gemm_simt(const LinearWorkspace &ws, int64_t M, int64_t N, int64_t K, int mode,
+                             const void *bias, void *y, int y_type, int32_t *partials,
+                             int partials_group, cudaStream_t s);
+cudaError_t launch_selftest_timeout(int64_t limit_ns, int *dev_err, cudaStream_t s);
+
+}  // namespace quartz

@@ -1,0 +1,119 @@
+"""C-ABI checks that need no GPU: the library builds and loads, exports every
+symbol include/quartz.h declares, and rejects bad arguments on the host
+before anything is launched."""
+import ctypes as C
+import os
+import re
+
+import pytest
+
+from paper_2509_26436_gb300 import _native as N
+from paper_2509_26436_gb300 import build as B
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include",
+                      "quartz.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    B.build()
+    return N.load()
+
+
+def _declared():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(quartz_[a-z_0-9]+)\s*\(", src)))
+
+
+def test_header_declares_the_boundary():
+    names = _declared()
+    for required in ("quartz_quantize", "quartz_encode_weights", "quartz_linear",
+                     "quartz_dequantize", "quartz_linear_workspace_size", "quartz_device_status"):
+        assert required in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    for name in _declared():
+        assert hasattr(lib, name), name
+    assert set(_declared()) == set(N.SIGNATURES)
+
+
+def test_status_strings_and_version(lib):
+    assert lib.quartz_status_string(0) == b"QUARTZ_OK"
+    assert lib.quartz_status_string(5) == b"QUARTZ_ERR_TIMEOUT"
+    assert lib.quartz_status_string(99) == b"QUARTZ_ERR_UNKNOWN"
+    assert lib.quartz_version() >> 16 == 1
+
+
+def _enc(rows, K, gs=16, mode=0, ptr=0x1000):
+    return N.QuartzEncoded(ptr, ptr, ptr, ptr, ptr, rows, K, N.QuartzParams(64, gs, mode))
+
+
+def test_encoded_sizes(lib):
+    out = (C.c_size_t * 5)()
+    p = N.QuartzParams(64, 16, 0)
+    assert lib.quartz_encoded_sizes(10, 128, C.byref(p), out) == 0
+    assert list(out) == [10 * 64, 10 * 8, 10 * 2 * 2, 10 * 2, 10 * 2 * 4]
+    p = N.QuartzParams(64, 12, 0)
+    assert lib.quartz_encoded_sizes(10, 128, C.byref(p), out) == N.QUARTZ_ERR_INVALID_ARG
+
+
+def test_host_validation_rejects_before_launch(lib):
+    """Every case here fails in host-side validation; no CUDA call is made."""
+    q = lib.quartz_quantize
+    e = _enc(4, 100)                                   # K not a multiple of 64
+    assert q(0x1000, C.byref(e), None) == N.QUARTZ_ERR_INVALID_ARG
+    e = _enc(4, 128, gs=12)                            # G_s not in {8,16,32,64}
+    assert q(0x1000, C.byref(e), None) == N.QUARTZ_ERR_INVALID_ARG
+    e = N.QuartzEncoded(0x1000, 0x1000, 0x1000, 0, 0, 4, 128, N.QuartzParams(128, 16, 0))
+    assert q(0x1000, C.byref(e), None) == N.QUARTZ_ERR_UNSUPPORTED   # group_q != 64
+    e = _enc(4, 128, mode=7)
+    assert q(0x1000, C.byref(e), None) == N.QUARTZ_ERR_INVALID_ARG
+    e = _enc(4, 128)
+    assert q(0x1001, C.byref(e), None) == N.QUARTZ_ERR_ALIGNMENT
+    assert q(None, C.byref(e), None) == N.QUARTZ_ERR_INVALID_ARG
+    e = _enc(4, 128, ptr=0x1008)
+    assert q(0x1000, C.byref(e), None) == N.QUARTZ_ERR_ALIGNMENT
+    e = N.QuartzEncoded(0x1000, 0x1000, 0x1000, 0, 0, 4, 128, N.QuartzParams(64, 16, 1))
+    assert q(0x1000, C.byref(e), None) == N.QUARTZ_ERR_INVALID_ARG  # asym needs zeros+gsum
+    e = _enc(-1, 128)
+    assert q(0x1000, C.byref(e), None) == N.QUARTZ_ERR_INVALID_ARG
+    assert lib.quartz_dequantize(C.byref(_enc(4, 128)), None, None) == N.QUARTZ_ERR_INVALID_ARG
+
+
+def test_linear_validation(lib):
+    L = lib.quartz_linear_ex
+    a, w = _enc(16, 128), _enc(24, 128)
+    ok = dict(bias=None, y=0x2000, t=0, part=None, pg=0, algo=0, ws=0x3000, wsb=1 << 30)
+
+    def call(a, w, **kw):
+        d = dict(ok, **kw)
+        return L(C.byref(a), C.byref(w), d["bias"], d["y"], d["t"], d["part"], d["pg"], d["algo"],
+                 d["ws"], d["wsb"], None)
+
+    assert call(a, _enc(24, 192)) == N.QUARTZ_ERR_INVALID_ARG           # K mismatch
+    assert call(a, _enc(24, 128, gs=32)) == N.QUARTZ_ERR_INVALID_ARG    # G_s mismatch
+    assert call(a, _enc(20, 128)) == N.QUARTZ_ERR_INVALID_ARG           # N % 8 != 0
+    assert call(a, w, t=3) == N.QUARTZ_ERR_INVALID_ARG                  # output type
+    assert call(a, w, algo=9) == N.QUARTZ_ERR_INVALID_ARG
+    assert call(a, w, part=0x4000, pg=2) == N.QUARTZ_ERR_INVALID_ARG    # group out of range
+    assert call(a, w, y=0x2004) == N.QUARTZ_ERR_ALIGNMENT
+    assert call(a, w, bias=0x2002) == N.QUARTZ_ERR_ALIGNMENT
+    assert call(a, w, wsb=16) == N.QUARTZ_ERR_WORKSPACE
+    assert call(a, w, ws=None) == N.QUARTZ_ERR_WORKSPACE
+    assert call(a, w, y=None) == N.QUARTZ_ERR_INVALID_ARG
+    p = N.QuartzParams(64, 16, 0)
+    assert lib.quartz_linear_workspace_size(16, 24, 128, C.byref(p)) > 16 * 128 * 2 + 24 * 128 * 2
+    assert lib.quartz_linear_workspace_size(16, 20, 128, C.byref(p)) == 0
+    assert lib.quartz_selftest_timeout(10, None) == N.QUARTZ_ERR_INVALID_ARG
+
+
+def test_missing_library_fails_loudly(tmp_path):
+    saved = N._lib
+    try:
+        N._lib = None
+        with pytest.raises(RuntimeError, match="no CPU or fallback"):
+            N.load(str(tmp_path / "libquartz.so"))
+    finally:
+        N._lib = saved

@@ -1,0 +1,164 @@
+"""GPU W4A4 linear parity against the CPU oracle.
+
+* Integer group partials P_g (the MMA result of one 64-wide K group) are
+  compared bit-exactly with the oracle's int64 sums.
+* Outputs are compared with the oracle's binary64 y.  Tolerance, derived
+  from the kernel's arithmetic: P_g is exact; each group term s_a*(s_w*P_g)
+  adds at most two binary32 roundings and the G-term running sum at most G
+  more, so |y_gpu - y| <= (G + 4) * 2^-24 * sum_g |s_a s_w D_g| before the
+  output conversion, which adds a relative 2^-11 (fp16), 2^-8 (bf16) or
+  nothing (fp32).  The test allows the stated relative bounds 1e-3 (fp16),
+  4e-3 (bf16), 1e-5 (fp32) plus that cancellation-aware absolute term.
+"""
+import numpy as np
+import pytest
+
+import oracle as O
+from paper_2509_26436_gb300 import inputs
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+REL = {"float16": 1e-3, "bfloat16": 4e-3, "float32": 1e-5}
+
+
+@pytest.fixture(scope="module")
+def Q():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2509_26436_gb300 as Q
+    return Q
+
+
+def _tol_check(y_gpu, y_ref, y_abs, G, dtype_name):
+    y_gpu = y_gpu.astype(np.float64)
+    tol = REL[dtype_name] * np.abs(y_ref) + (G + 4) * 2.0 ** -24 * y_abs + 2.0 ** -24
+    err = np.abs(y_gpu - y_ref)
+    bad = err > tol
+    assert not bad.any(), (f"{bad.sum()} of {bad.size} outside tolerance; worst "
+                           f"{(err / np.maximum(tol, 1e-30)).max():.3g}x")
+
+
+def _run(Q, xa, xw, gs, mode, bias=None, out_dtype="float16", algo=None, partials_group=None):
+    a = Q.quantize(torch.from_numpy(xa).cuda(), group_s=gs, mode=mode)
+    w = Q.encode_weights(torch.from_numpy(xw).cuda(), group_s=gs, mode=mode)
+    b = None if bias is None else torch.from_numpy(bias).cuda()
+    kw = {}
+    if algo is not None:
+        kw["algo"] = algo
+    r = Q.linear(a, w, b, out_dtype=getattr(torch, out_dtype), partials_group=partials_group, **kw)
+    assert Q.device_status() == 0
+    return r
+
+
+@pytest.mark.parametrize("algo", ["tcgen05", "simt"])
+@pytest.mark.parametrize("out_dtype", ["float16", "bfloat16", "float32"])
+def test_linear_single_layer(Q, algo, out_dtype):
+    """256 tokens x 1152 -> 1152, G_s = 16, symmetric, with bias."""
+    layer = inputs.CONFIG0[0]
+    xa, xw = layer.activations(), layer.weights()
+    bias = inputs.gaussian_weights(1, layer.N, seed=3)[0]
+    alg = Q.ALGO_TCGEN05 if algo == "tcgen05" else Q.ALGO_SIMT
+    y = _run(Q, xa, xw, 16, O.SYMMETRIC, bias, out_dtype, alg)
+    a, w = O.encode(xa, 64, 16), O.encode(xw, 64, 16)
+    ref, rabs = O.linear(a, w, bias, with_abs=True)
+    _tol_check(y.float().cpu().numpy(), ref, rabs, layer.K // 64, out_dtype)
+
+
+@pytest.mark.parametrize("algo", ["tcgen05", "simt"])
+@pytest.mark.parametrize("group", [0, 9, 17])
+def test_group_partials_bit_exact(Q, algo, group):
+    """The integer MMA result of one group equals the oracle's int64 sum."""
+    layer = inputs.CONFIG0[0]
+    xa, xw = layer.activations(), layer.weights()
+    alg = Q.ALGO_TCGEN05 if algo == "tcgen05" else Q.ALGO_SIMT
+    _, part = _run(Q, xa, xw, 16, O.SYMMETRIC, algo=alg, partials_group=group)
+    va = O.decode_values(O.encode(xa, 64, 16))[:, group * 64:(group + 1) * 64]
+    vw = O.decode_values(O.encode(xw, 64, 16))[:, group * 64:(group + 1) * 64]
+    ref = O.group_partials(va, vw, 64)[0]
+    assert np.array_equal(part.cpu().numpy().astype(np.int64), ref)
+
+
+@pytest.mark.parametrize("mode", [O.SYMMETRIC, O.ASYMMETRIC])
+@pytest.mark.parametrize("gs", [8, 32])
+@pytest.mark.parametrize("M,N,K", [(1, 8, 64), (200, 264, 192), (300, 520, 640), (129, 256, 64),
+                                   (1000, 776, 1216), (384, 1024, 256)])
+def test_linear_ragged_shapes(Q, mode, gs, M, N, K):
+    """Several tiles with ragged M and N tails, one-group K, all G_s."""
+    xa = inputs.laplace_activations(M, K, seed=M + N + K)
+    xw = inputs.gaussian_weights(N, K, seed=M * 7 + N)
+    bias = inputs.gaussian_weights(1, N, seed=N)[0]
+    g = (K // 64) // 2
+    y, part = _run(Q, xa, xw, gs, mode, bias, "float32", partials_group=g)
+    a, w = O.encode(xa, 64, gs, mode), O.encode(xw, 64, gs, mode)
+    ref, rabs = O.linear(a, w, bias, with_abs=True)
+    _tol_check(y.cpu().numpy(), ref, rabs, K // 64, "float32")
+    va = O.decode_values(a)[:, g * 64:(g + 1) * 64]
+    vw = O.decode_values(w)[:, g * 64:(g + 1) * 64]
+    assert np.array_equal(part.cpu().numpy().astype(np.int64), O.group_partials(va, vw, 64)[0])
+
+
+def test_linear_asymmetric_conv_activations(Q):
+    """Zero-point path on one-sided post-SiLU im2col activations."""
+    xa = inputs.silu_im2col(1, 64, 16, 16, seed=8)        # [256, 576]
+    xw = inputs.gaussian_weights(320, 576, seed=9)
+    for out_dtype in ("float16", "float32"):
+        y = _run(Q, xa, xw, 16, O.ASYMMETRIC, None, out_dtype)
+        ref, rabs = O.linear(O.encode(xa, 64, 16, O.ASYMMETRIC), O.encode(xw, 64, 16, O.ASYMMETRIC),
+                             with_abs=True)
+        _tol_check(y.float().cpu().numpy(), ref, rabs, 9, out_dtype)
+
+
+def test_linear_zero_rows(Q):
+    a = Q.quantize(torch.empty((0, 128), dtype=torch.float16, device="cuda"))
+    w = Q.encode_weights(torch.randn(16, 128, device="cuda").half())
+    y = Q.linear(a, w)
+    torch.cuda.synchronize()
+    assert y.shape == (0, 16)
+
+
+def _sample_rows(M):
+    return np.unique(np.concatenate([np.arange(4), np.arange(M - 4, M),
+                                     np.linspace(4, M - 5, 8).astype(np.int64)]))
+
+
+FULL_LAYERS = inputs.CONFIG2 + inputs.CONFIG3 + inputs.CONFIG4
+
+
+@pytest.mark.parametrize("layer", FULL_LAYERS, ids=[l.name for l in FULL_LAYERS])
+def test_linear_full_size_sampled(Q, layer):
+    """Full-size layers in the benchmark's launch configuration (G_s = 16,
+    symmetric, fp16 out): codes, one group's integer partials and outputs
+    compared with the oracle on a deterministic sample of token rows."""
+    xa, xw = layer.activations(), layer.weights()
+    G = layer.K // 64
+    g = G // 2
+    a = Q.quantize(torch.from_numpy(xa).cuda(), group_s=16)
+    w = Q.encode_weights(torch.from_numpy(xw).cuda(), group_s=16)
+    y, part = Q.linear(a, w, partials_group=g)
+    assert Q.device_status() == 0
+    rows = _sample_rows(layer.M)
+    rows_t = torch.from_numpy(rows).cuda()
+    ea = O.encode(xa[rows], 64, 16)
+    ew = O.encode(xw, 64, 16)
+    assert np.array_equal(a.codes[rows_t].cpu().numpy(), ea.codes)
+    assert np.array_equal(a.flags[rows_t].cpu().numpy(), ea.flags)
+    assert np.array_equal(w.codes.cpu().numpy(), ew.codes)
+    ref, rabs = O.linear(ea, ew, with_abs=True)
+    _tol_check(y[rows_t].float().cpu().numpy(), ref, rabs, G, "float16")
+    va = O.decode_values(ea)[:, g * 64:(g + 1) * 64]
+    vw = O.decode_values(ew)[:, g * 64:(g + 1) * 64]
+    assert np.array_equal(part[rows_t].cpu().numpy().astype(np.int64), O.group_partials(va, vw, 64)[0])
+
+
+def test_bounded_wait_reports_timeout(Q):
+    """Failure detection without a fault: a kernel waits on an mbarrier that
+    nothing arrives at, gives up after 1 ms and the host reads the status;
+    the context stays usable."""
+    assert Q.device_status() == 0
+    assert Q.selftest_timeout(1_000_000) == 0
+    assert Q.device_status() == 5          # QUARTZ_ERR_TIMEOUT
+    assert Q.device_status() == 0          # cleared
+    x = torch.randn(4, 64, device="cuda").half()
+    Q.quantize(x)
+    assert Q.device_status() == 0
