@@ -1,0 +1,364 @@
+#!/usr/bin/env python
+"""Benchmark of the QuaRTZ W4A4 hot path on FLUX.1-schnell-shaped block linears.
+
+One step = the whole hot path over one batch: for each of the four MM-DiT
+block linears (QKV 3072->9216, proj 3072->3072, MLP 3072->12288 and
+12288->3072, M = (4096 + 512) tokens x batch 4 = 18432), quantize + LZS-encode
+the fp16 activations (Eq. 1, Eq. 2), expand the codes and run the tcgen05
+GEMM with its dequant epilogue (Section 4.4).  Weights are encoded once,
+offline, outside the timed region (as the paper's PTQ does).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Prints one JSON line (rank 0).  `value` is W4A4 linear TOPS of the whole job
+(2*M*N*K summed over the layers, per step, over the device-timed step
+time); the encode GB/s of the quantize kernel is reported beside it.  The
+inputs (~0.8 GB of fp16 activations per step) exceed the 129 MB L2, so no
+flush is needed between steps.  Multi-GPU runs are independent replicas
+(the path shards by token rows with no exchange): weak scaling.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "QuaRTZ W4A4 linear TOPS (% of roofline); LZS encode GB/s (% of HBM peak)"
+GROUP_Q, GROUP_S = 64, 16
+FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS = 6800.0, 1900.0
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=300)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
+    p.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline leg")
+    return p.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), float(d["bf16_tflops"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS, "fallback"
+
+
+def dist_env():
+    return (int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)),
+            int(os.environ.get("LOCAL_RANK", 0)))
+
+
+def layer_config(layers):
+    return {"workload": "flux1_schnell_mmdit_block_linears", "tokens": layers[0].M,
+            "layers": [f"{l.name}:{l.K}->{l.N}" for l in layers], "group_q": GROUP_Q,
+            "group_s": GROUP_S, "mode": "symmetric", "out": "f16",
+            "inputs": "seeded synthetic Laplace(0,0.05), 0.1% channels x50; weights N(0,0.02)",
+            "l2": "activations per step 0.8 GB > 129 MB L2, no flush"}
+
+
+def encode_bytes_per_elem(gs=GROUP_S):
+    """Algorithmic HBM bytes of the encoder per element: fp16 in, 4-bit code,
+    one FLAG byte per G_s, one fp16 scale per 64 (symmetric)."""
+    return 2.0 + 0.5 + 1.0 / gs + 2.0 / GROUP_Q
+
+
+# --------------------------------------------------------------------------
+# clocks during the timed region
+# --------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("index,pci.bus_id,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index):
+        self.dev = device_index
+        self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        self.p = None
+
+    def __enter__(self):
+        try:
+            self.p = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}",
+                                       "--format=csv,noheader,nounits", "-lms", "100"],
+                                      stdout=self.f, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.p = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        if self.p is not None:
+            time.sleep(0.15)
+            self.p.terminate()
+            self.p.wait()
+
+    def summary(self, bus_id=None):
+        self.f.flush()
+        self.f.seek(0)
+        rows = [[c.strip() for c in line.split(",")] for line in self.f if line.count(",") >= 9]
+        os.unlink(self.f.name)
+        if bus_id:
+            mine = [r for r in rows if r[1].lower().endswith(bus_id.lower()[-12:])]
+            rows = mine or rows
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"], "samples": 0}
+        idx = {r[0] for r in rows}
+        if len(idx) > 1:
+            rows = [r for r in rows if r[0] == str(self.dev)] or rows
+        sm = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        smax = [float(r[3]) for r in rows if r[3].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in rows for n, v in zip(names, r[6:10]) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None, "reasons": reasons,
+                "samples": len(rows),
+                "power_w_max": max((float(r[4]) for r in rows
+                                    if r[4].replace(".", "").isdigit()), default=None)}
+
+
+# --------------------------------------------------------------------------
+# CPU oracle baseline (a bounded sample of the same workload)
+# --------------------------------------------------------------------------
+def oracle_sample(layers, rows_per_layer, xs=None, ws=None):
+    """Time the oracle on `rows_per_layer` token rows of every layer:
+    encode (Eq. 1 + Eq. 2) of those rows plus the W4A4 linear for them.
+    Weights are encoded before timing, like the GPU path.  Returns
+    (seconds, ops, elements)."""
+    import numpy as np
+
+    import oracle as O
+    enc_w, xa_s = [], []
+    for i, l in enumerate(layers):
+        w = ws[i] if ws is not None else l.weights()
+        enc_w.append(O.encode(w, GROUP_Q, GROUP_S))
+        x = xs[i] if xs is not None else l.activations()
+        sel = np.linspace(0, l.M - 1, rows_per_layer).astype(np.int64)
+        xa_s.append(np.ascontiguousarray(x[sel]))
+    t0 = time.perf_counter()
+    ops = 0
+    for l, x, ew in zip(layers, xa_s, enc_w):
+        ea = O.encode(x, GROUP_Q, GROUP_S)
+        O.linear(ea, ew)
+        ops += 2 * x.shape[0] * l.N * l.K
+    return time.perf_counter() - t0, ops
+
+
+def run_reference(args):
+    from paper_2509_26436_gb300 import inputs
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    layers = inputs.CONFIG4
+    rows = 2
+    xs = [l.activations() for l in layers]
+    ws = [l.weights() for l in layers]
+    times = []
+    total_ops = 0
+    for i in range(args.warmup + args.steps):
+        t, ops = oracle_sample(layers, rows, xs, ws)
+        if i >= args.warmup:
+            times.append(t)
+            total_ops = ops
+    t_step = sum(times) / len(times)
+    value = total_ops / t_step / 1e12
+    sample = (f"{rows} token rows of each of the 4 FLUX block linears per step (encode + linear), "
+              "single-threaded plain C oracle, weights encoded before timing")
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_step * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64/f64",
+        "data": "synthetic", "config": layer_config(layers),
+        "cpu_baseline": {"value": value, "unit": "TOPS", "cores": 1, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "TOPS", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+# --------------------------------------------------------------------------
+# our path
+# --------------------------------------------------------------------------
+def run_ours(args):
+    import numpy as np
+    import torch
+
+    import paper_2509_26436_gb300 as Q
+    from paper_2509_26436_gb300 import inputs
+
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    hbm_peak, tc_peak, peak_src = peaks()
+    layers = inputs.CONFIG4
+
+    # ---- inputs (seeded, host) -> pinned host + device ---------------------
+    xs = [l.activations() for l in layers]
+    ws = [l.weights() for l in layers]
+    x_host = [torch.from_numpy(x).pin_memory() for x in xs]
+    x_dev = [h.to(dev) for h in x_host]
+    enc_w = [Q.encode_weights(torch.from_numpy(w).to(dev), group_s=GROUP_S) for w in ws]
+    enc_a = [Q.empty_encoded(l.M, l.K, Q.Params(GROUP_Q, GROUP_S), dev) for l in layers]
+    y_dev = [torch.empty((l.M, l.N), dtype=torch.float16, device=dev) for l in layers]
+    ws_bytes = max(Q.linear_workspace_size(l.M, l.N, l.K) for l in layers)
+    workspace = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+    torch.cuda.synchronize()
+    assert Q.device_status() == 0
+
+    nl = len(layers)
+    ev = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
+
+    def step(rec=None):
+        for i in range(nl):
+            if rec is not None:
+                rec["q"][i][0].record(stream)
+            Q.quantize(x_dev[i], out=enc_a[i], group_s=GROUP_S)
+            if rec is not None:
+                rec["q"][i][1].record(stream)
+            Q.linear(enc_a[i], enc_w[i], out=y_dev[i], workspace=workspace,
+                     gemm_events=None if rec is None else rec["g"][i])
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    assert Q.device_status() == 0
+
+    # per-kernel durations: every step records events around the quantize
+    # kernel and around the GEMM kernel of every layer
+    recs = [{"q": [(ev(), ev()) for _ in range(nl)], "g": [(ev(), ev()) for _ in range(nl)]}
+            for _ in range(args.steps)]
+    bus = None
+    try:
+        bus = torch.cuda.get_device_properties(dev).pci_bus_id
+    except AttributeError:
+        pass
+    t0, t1 = ev(), ev()
+    barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        t0.record(stream)
+        for k in range(args.steps):
+            step(recs[k])
+        t1.record(stream)
+        torch.cuda.synchronize()
+    barrier()
+    clocks = clk.summary(bus)
+    status = Q.device_status()
+    assert status == 0, f"device status {status}"
+    t_step = t0.elapsed_time(t1) / 1e3 / args.steps
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([t_step], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        t_step = float(t.item())
+
+    ops_step = sum(l.ops for l in layers)
+    value = world * ops_step / t_step / 1e12
+    gemm_ms = [statistics.mean(r["g"][i][0].elapsed_time(r["g"][i][1]) for r in recs)
+               for i in range(nl)]
+    quant_ms = [statistics.mean(r["q"][i][0].elapsed_time(r["q"][i][1]) for r in recs)
+                for i in range(nl)]
+    gemm_tflops = sum(l.ops for l in layers) / (sum(gemm_ms) / 1e3) / 1e12
+    elems = sum(l.M * l.K for l in layers)
+    enc_gbs = elems * encode_bytes_per_elem() / (sum(quant_ms) / 1e3) / 1e9
+    launches_per_step = nl * (1 + 5)   # quantize; expand A, side A, expand W, side W, GEMM
+
+    # ---- end to end through the public API with host buffers ---------------
+    e2e = None
+    if not args.no_e2e:
+        y_host = [torch.empty((l.M, l.N), dtype=torch.float16).pin_memory() for l in layers]
+        e_steps = max(3, min(args.steps // 10, 20))
+
+        def e2e_step():
+            for i in range(nl):
+                x_dev[i].copy_(x_host[i], non_blocking=True)
+                Q.quantize(x_dev[i], out=enc_a[i], group_s=GROUP_S)
+                Q.linear(enc_a[i], enc_w[i], out=y_dev[i], workspace=workspace)
+                y_host[i].copy_(y_dev[i], non_blocking=True)
+
+        for _ in range(2):
+            e2e_step()
+        torch.cuda.synchronize()
+        barrier()
+        a0, a1 = ev(), ev()
+        a0.record(stream)
+        for _ in range(e_steps):
+            e2e_step()
+        a1.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        te = a0.elapsed_time(a1) / 1e3 / e_steps
+        if world > 1:
+            import torch.distributed as dist
+            t = torch.tensor([te], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            te = float(t.item())
+        e2e = {"value": world * ops_step / te / 1e12, "unit": "TOPS",
+               "h2d_bytes_per_step": sum(x.numel() * 2 for x in x_host),
+               "d2h_bytes_per_step": sum(l.M * l.N * 2 for l in layers), "steps": e_steps,
+               "ms_per_step": te * 1e3}
+
+    # ---- CPU oracle baseline (rank 0 only, N = 1) ---------------------------
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        rows = 4
+        t, ops = oracle_sample(layers, rows, xs, ws)
+        cpu = {"value": ops / t / 1e12, "unit": "TOPS", "cores": 1, "kind": "oracle",
+               "sample": f"{rows} token rows of each of the 4 layers (encode + linear), "
+                         f"{t:.1f} s single-threaded plain C"}
+
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    if rank != 0:
+        return
+    out = {
+        "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": t_step * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f16", "data": "synthetic",
+        "config": layer_config(layers),
+        "roofline": {"bound": "tensor", "achieved": gemm_tflops, "peak": tc_peak,
+                     "unit": "TFLOP/s", "frac": gemm_tflops / tc_peak, "traffic": None,
+                     "kernel": "gemm_tcgen05_kernel", "peak_source": f"{peak_src} bf16 burst",
+                     "per_layer_ms": gemm_ms},
+        "encode": {"kernel": "quantize_kernel", "gbs": enc_gbs, "peak_gbs": hbm_peak,
+                   "frac": enc_gbs / hbm_peak, "bytes_per_elem": encode_bytes_per_elem(),
+                   "per_layer_ms": quant_ms, "peak_source": peak_src},
+        "clocks": clocks,
+        "gpu_launches": launches_per_step * args.steps,
+        "e2e": e2e,
+        "cpu_baseline": cpu,
+    }
+    print(json.dumps(out), flush=True)
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

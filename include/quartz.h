@@ -144,15 +144,26 @@ int32_t quartz_linear(const quartz_encoded_t *a, const quartz_encoded_t *w, cons
                       void *y, int32_t y_type, void *workspace, size_t workspace_bytes,
                       void *stream);
 
-/* quartz_linear with two extra controls, for verification:
- *   partials        NULL, or int32 [M, N]: receives P_g[m, n] of group
- *                   `partials_group` (0 <= partials_group < K/64), the raw
- *                   integer MMA result before any scale or zero point
- *   algo            quartz_algo_t: which GEMM kernel runs */
+/* Extra controls of quartz_linear_ex (all optional; zero-initialise):
+ *   partials          NULL, or int32 [M, N] device buffer that receives
+ *                     P_g[m, n] of group `partials_group` (0 <= g < K/64), the
+ *                     raw integer MMA result before any scale or zero point
+ *   algo              quartz_algo_t: which GEMM kernel runs
+ *   gemm_event_begin  NULL, or a cudaEvent_t recorded on `stream` right before
+ *   gemm_event_end    / right after the GEMM kernel (after operand expansion),
+ *                     so a caller can time the GEMM kernel alone */
+typedef struct {
+    int32_t *partials;
+    int32_t partials_group;
+    int32_t algo;
+    void *gemm_event_begin;
+    void *gemm_event_end;
+} quartz_linear_opts_t;
+
+/* quartz_linear with the controls above (opts may be NULL = defaults). */
 int32_t quartz_linear_ex(const quartz_encoded_t *a, const quartz_encoded_t *w,
-                         const void *bias_f16, void *y, int32_t y_type, int32_t *partials,
-                         int32_t partials_group, int32_t algo, void *workspace,
-                         size_t workspace_bytes, void *stream);
+                         const void *bias_f16, void *y, int32_t y_type, void *workspace,
+                         size_t workspace_bytes, const quartz_linear_opts_t *opts, void *stream);
 
 /* Synchronise `stream`, then read and clear the library's device error word.
  * Returns QUARTZ_OK, QUARTZ_ERR_TIMEOUT if a kernel gave up on a bounded

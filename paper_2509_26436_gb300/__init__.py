@@ -127,12 +127,14 @@ _OUT = {"float16": OUT_F16, "bfloat16": OUT_BF16, "float32": OUT_F32}
 
 
 def linear(a: Encoded, w: Encoded, bias=None, out_dtype=None, out=None, workspace=None,
-           partials_group: int | None = None, algo: int = ALGO_TCGEN05, stream=None):
+           partials_group: int | None = None, algo: int = ALGO_TCGEN05, stream=None,
+           gemm_events=None):
     """W4A4 QuaRTZ linear: y = dequant(a) @ dequant(w)^T (+ bias), computed as
     exact integer group partials scaled by the 16-bit group scales.
 
     Returns y, or (y, partials) when `partials_group` is given (int32 [M, N]
-    raw integer MMA sums of that 64-wide K group)."""
+    raw integer MMA sums of that 64-wide K group).  `gemm_events` = a pair
+    of torch.cuda.Event recorded around the GEMM kernel alone."""
     torch = _torch()
     out_dtype = out_dtype or torch.float16
     M, Nn = a.rows, w.rows
@@ -148,10 +150,14 @@ def linear(a: Encoded, w: Encoded, bias=None, out_dtype=None, out=None, workspac
     if bias is not None and not (bias.dtype == torch.float16 and bias.is_cuda and bias.numel() == Nn):
         raise ValueError("bias must be a float16 CUDA tensor of N elements")
     ac, wc = a.c(), w.c()
+    opts = N.QuartzLinearOpts(None if part is None else part.data_ptr(),
+                              0 if partials_group is None else partials_group, algo,
+                              None if gemm_events is None else gemm_events[0].cuda_event,
+                              None if gemm_events is None else gemm_events[1].cuda_event)
     rc = N.load().quartz_linear_ex(
         C.byref(ac), C.byref(wc), None if bias is None else bias.data_ptr(), y.data_ptr(), y_type,
-        None if part is None else part.data_ptr(), 0 if partials_group is None else partials_group,
-        algo, workspace.data_ptr(), workspace.numel() * workspace.element_size(), _stream(stream))
+        workspace.data_ptr(), workspace.numel() * workspace.element_size(), C.byref(opts),
+        _stream(stream))
     N.check(rc, "quartz_linear_ex")
     return y if part is None else (y, part)
 

@@ -45,6 +45,11 @@ class QuartzEncoded(C.Structure):
                 ("rows", C.c_int64), ("K", C.c_int64), ("p", QuartzParams)]
 
 
+class QuartzLinearOpts(C.Structure):
+    _fields_ = [("partials", _P), ("partials_group", C.c_int32), ("algo", C.c_int32),
+                ("gemm_event_begin", _P), ("gemm_event_end", _P)]
+
+
 SIGNATURES = {
     "quartz_status_string": (C.c_char_p, [_I32]),
     "quartz_version": (_I32, []),
@@ -56,7 +61,7 @@ SIGNATURES = {
     "quartz_linear": (_I32, [C.POINTER(QuartzEncoded), C.POINTER(QuartzEncoded), _P, _P, _I32,
                              _P, _SZ, _P]),
     "quartz_linear_ex": (_I32, [C.POINTER(QuartzEncoded), C.POINTER(QuartzEncoded), _P, _P, _I32,
-                                _P, _I32, _I32, _P, _SZ, _P]),
+                                _P, _SZ, C.POINTER(QuartzLinearOpts), _P]),
     "quartz_device_status": (_I32, [_P]),
     "quartz_selftest_timeout": (_I32, [_I64, _P]),
 }

@@ -135,10 +135,15 @@ size_t quartz_linear_workspace_size(int64_t M, int64_t N, int64_t K, const quart
 }
 
 int32_t quartz_linear_ex(const quartz_encoded_t *a, const quartz_encoded_t *w,
-                         const void *bias_f16, void *y, int32_t y_type, int32_t *partials,
-                         int32_t partials_group, int32_t algo, void *workspace,
-                         size_t workspace_bytes, void *stream)
+                         const void *bias_f16, void *y, int32_t y_type, void *workspace,
+                         size_t workspace_bytes, const quartz_linear_opts_t *opts, void *stream)
 {
+    quartz_linear_opts_t o;
+    std::memset(&o, 0, sizeof(o));
+    if (opts) o = *opts;
+    int32_t *partials = o.partials;
+    const int32_t partials_group = o.partials_group;
+    const int32_t algo = o.algo;
     int32_t rc = check_encoded(a);
     if (rc) return rc;
     rc = check_encoded(w);
@@ -170,11 +175,15 @@ int32_t quartz_linear_ex(const quartz_encoded_t *a, const quartz_encoded_t *w,
     cudaError_t e = launch_expand(a, ws.a_op, ws.a_side, ws.m_pad, 1, s);
     if (e == cudaSuccess) e = launch_expand(w, ws.w_op, ws.w_side, ws.n_pad, 0, s);
     if (e != cudaSuccess) return QUARTZ_ERR_CUDA;
+    if (o.gemm_event_begin && cudaEventRecord(static_cast<cudaEvent_t>(o.gemm_event_begin), s) != cudaSuccess)
+        return QUARTZ_ERR_CUDA;
     if (algo == QUARTZ_ALGO_SIMT)
         e = launch_gemm_simt(ws, M, N, K, a->p.mode, bias_f16, y, y_type, partials, partials_group, s);
     else
         e = launch_gemm_tcgen05(ws, M, N, K, a->p.mode, bias_f16, y, y_type, partials,
                                 partials_group, dev_err, s);
+    if (e == cudaSuccess && o.gemm_event_end)
+        e = cudaEventRecord(static_cast<cudaEvent_t>(o.gemm_event_end), s);
     return map_cuda(e);
 }
 
@@ -182,8 +191,7 @@ int32_t quartz_linear(const quartz_encoded_t *a, const quartz_encoded_t *w, cons
                       void *y, int32_t y_type, void *workspace, size_t workspace_bytes,
                       void *stream)
 {
-    return quartz_linear_ex(a, w, bias_f16, y, y_type, nullptr, 0, QUARTZ_ALGO_TCGEN05, workspace,
-                            workspace_bytes, stream);
+    return quartz_linear_ex(a, w, bias_f16, y, y_type, workspace, workspace_bytes, nullptr, stream);
 }
 
 int32_t quartz_device_status(void *stream)

@@ -89,8 +89,9 @@ def test_linear_validation(lib):
 
     def call(a, w, **kw):
         d = dict(ok, **kw)
-        return L(C.byref(a), C.byref(w), d["bias"], d["y"], d["t"], d["part"], d["pg"], d["algo"],
-                 d["ws"], d["wsb"], None)
+        o = N.QuartzLinearOpts(d["part"], d["pg"], d["algo"], None, None)
+        return L(C.byref(a), C.byref(w), d["bias"], d["y"], d["t"], d["ws"], d["wsb"], C.byref(o),
+                 None)
 
     assert call(a, _enc(24, 192)) == N.QUARTZ_ERR_INVALID_ARG           # K mismatch
     assert call(a, _enc(24, 128, gs=32)) == N.QUARTZ_ERR_INVALID_ARG    # G_s mismatch
