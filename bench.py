@@ -44,6 +44,7 @@ def parse():
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
     p.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline leg")
+    p.add_argument("--layers", default="", help="comma-separated subset of layer names (profiling)")
     return p.parse_args()
 
 
@@ -68,6 +69,16 @@ def layer_config(layers):
             "group_s": GROUP_S, "mode": "symmetric", "out": "f16",
             "inputs": "seeded synthetic Laplace(0,0.05), 0.1% channels x50; weights N(0,0.02)",
             "l2": "activations per step 0.8 GB > 129 MB L2, no flush"}
+
+
+def select_layers(all_layers, names):
+    if not names:
+        return list(all_layers)
+    want = names.split(",")
+    sel = [l for l in all_layers if l.name in want]
+    if len(sel) != len(want):
+        raise SystemExit(f"unknown layer in {names}; have {[l.name for l in all_layers]}")
+    return sel
 
 
 def encode_bytes_per_elem(gs=GROUP_S):
@@ -132,17 +143,19 @@ class ClockSampler:
 # --------------------------------------------------------------------------
 # CPU oracle baseline (a bounded sample of the same workload)
 # --------------------------------------------------------------------------
-def oracle_sample(layers, rows_per_layer, xs=None, ws=None):
-    """Time the oracle on `rows_per_layer` token rows of every layer:
-    encode (Eq. 1 + Eq. 2) of those rows plus the W4A4 linear for them.
-    Weights are encoded before timing, like the GPU path.  Returns
-    (seconds, ops, elements)."""
+def oracle_sample(layers, rows_per_layer, xs=None, ws=None, cols_per_layer=None):
+    """Time the oracle on `rows_per_layer` token rows of every layer (and the
+    first `cols_per_layer` output channels, or all): encode (Eq. 1 + Eq. 2)
+    of those rows plus the W4A4 linear for them.  Weights are encoded before
+    timing, like the GPU path.  Returns (seconds, ops)."""
     import numpy as np
 
     import oracle as O
     enc_w, xa_s = [], []
     for i, l in enumerate(layers):
         w = ws[i] if ws is not None else l.weights()
+        if cols_per_layer is not None:
+            w = np.ascontiguousarray(w[:cols_per_layer])
         enc_w.append(O.encode(w, GROUP_Q, GROUP_S))
         x = xs[i] if xs is not None else l.activations()
         sel = np.linspace(0, l.M - 1, rows_per_layer).astype(np.int64)
@@ -152,7 +165,7 @@ def oracle_sample(layers, rows_per_layer, xs=None, ws=None):
     for l, x, ew in zip(layers, xa_s, enc_w):
         ea = O.encode(x, GROUP_Q, GROUP_S)
         O.linear(ea, ew)
-        ops += 2 * x.shape[0] * l.N * l.K
+        ops += 2 * x.shape[0] * ew.rows * l.K
     return time.perf_counter() - t0, ops
 
 
@@ -161,21 +174,22 @@ def run_reference(args):
     rank, world, _ = dist_env()
     if rank != 0:
         return
-    layers = inputs.CONFIG4
-    rows = 2
+    layers = select_layers(inputs.CONFIG4, args.layers)
+    rows, cols = 1, 1024
     xs = [l.activations() for l in layers]
     ws = [l.weights() for l in layers]
     times = []
     total_ops = 0
     for i in range(args.warmup + args.steps):
-        t, ops = oracle_sample(layers, rows, xs, ws)
+        t, ops = oracle_sample(layers, rows, xs, ws, cols)
         if i >= args.warmup:
             times.append(t)
             total_ops = ops
     t_step = sum(times) / len(times)
     value = total_ops / t_step / 1e12
-    sample = (f"{rows} token rows of each of the 4 FLUX block linears per step (encode + linear), "
-              "single-threaded plain C oracle, weights encoded before timing")
+    sample = (f"{rows} token row x the first {cols} output channels of each of the 4 FLUX block "
+              "linears per step (encode + linear), single-threaded plain C oracle, weights "
+              "encoded before timing")
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_step * 1e3,
@@ -204,7 +218,7 @@ def run_ours(args):
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=dev)
     hbm_peak, tc_peak, peak_src = peaks()
-    layers = inputs.CONFIG4
+    layers = select_layers(inputs.CONFIG4, args.layers)
 
     # ---- inputs (seeded, host) -> pinned host + device ---------------------
     xs = [l.activations() for l in layers]
@@ -321,7 +335,7 @@ def run_ours(args):
     # ---- CPU oracle baseline (rank 0 only, N = 1) ---------------------------
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
-        rows = 4
+        rows = 8
         t, ops = oracle_sample(layers, rows, xs, ws)
         cpu = {"value": ops / t / 1e12, "unit": "TOPS", "cores": 1, "kind": "oracle",
                "sample": f"{rows} token rows of each of the 4 layers (encode + linear), "
