@@ -150,6 +150,13 @@ def linear(a: Encoded, w: Encoded, bias=None, out_dtype=None, out=None, workspac
     if bias is not None and not (bias.dtype == torch.float16 and bias.is_cuda and bias.numel() == Nn):
         raise ValueError("bias must be a float16 CUDA tensor of N elements")
     ac, wc = a.c(), w.c()
+    if gemm_events is not None:
+        # torch creates events lazily and tracks their recording itself: a
+        # first record through torch creates them; the library then
+        # re-records them around the GEMM launch on the same stream.
+        s_ = stream if stream is not None else torch.cuda.current_stream()
+        for e in gemm_events:
+            e.record(s_)
     opts = N.QuartzLinearOpts(None if part is None else part.data_ptr(),
                               0 if partials_group is None else partials_group, algo,
                               None if gemm_events is None else gemm_events[0].cuda_event,

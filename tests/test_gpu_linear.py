@@ -162,3 +162,21 @@ def test_bounded_wait_reports_timeout(Q):
     x = torch.randn(4, 64, device="cuda").half()
     Q.quantize(x)
     assert Q.device_status() == 0
+
+
+def test_gemm_events_bracket_the_gemm_kernel(Q):
+    """The events quartz_linear_ex records sit around the GEMM launch only:
+    they measure a positive time no longer than the whole call."""
+    layer = inputs.CONFIG0[0]
+    a = Q.quantize(torch.from_numpy(layer.activations()).cuda())
+    w = Q.encode_weights(torch.from_numpy(layer.weights()).cuda())
+    g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    for _ in range(3):
+        c0.record()
+        Q.linear(a, w, gemm_events=(g0, g1))
+        c1.record()
+    torch.cuda.synchronize()
+    t_gemm, t_call = g0.elapsed_time(g1), c0.elapsed_time(c1)
+    assert 0 < t_gemm <= t_call
+    assert Q.device_status() == 0
