@@ -91,25 +91,33 @@ constexpr int kStages = 4;
 constexpr int kABytes = BM * BK * 2;
 constexpr int kBBytes = BN * BK * 2;
 constexpr int kStageBytes = kABytes + kBBytes;
-constexpr int kEpiWarps = 8;                  // warpgroups 0 and 1
-constexpr int kThreads = (kEpiWarps + 4) * 32;  // warpgroup 2: producer, MMA, 2 idle warps
+// Warpgroups 0-3 dequantise (16 warps: four per 32-lane TMEM quarter, 64
+// columns each); warpgroup 4 holds the TMA producer, the MMA issuer and two
+// idle warps.  The dequant epilogue is the throughput-critical part (two fp32
+// operations per output element per group, as many cycles as the MMAs), so it
+// gets four warps per scheduler to hide FMA and shared-memory latency.
+constexpr int kEpiWarps = 16;
+constexpr int kThreads = (kEpiWarps + 4) * 32;
 constexpr int kProducerWarp = kEpiWarps;
 constexpr int kMmaWarp = kEpiWarps + 1;
-// Register split (setmaxnreg): the launch gives 65536 / 384 -> 168 per
-// thread; warpgroup 2 drops to 56 so the two epilogue warpgroups can hold
-// 224 (2*128*224 + 128*56 = 384*168).
-constexpr uint32_t kRegsEpilogue = 224;
-constexpr uint32_t kRegsControl = 56;
-static_assert(2 * 128 * kRegsEpilogue + 128 * kRegsControl <= kThreads * 168, "register split");
+constexpr int kColsPerWarp = BN / 4;
+// Register split (setmaxnreg): 640 threads launch with 96 registers each;
+// warpgroup 4 drops to 32 so the epilogue warpgroups can hold 112
+// (512*112 + 128*32 = 61440 = 640*96).
+constexpr uint32_t kRegsLaunch = 96;
+constexpr uint32_t kRegsEpilogue = 112;
+constexpr uint32_t kRegsControl = 32;
+static_assert(kEpiWarps * 32 * kRegsEpilogue + 128 * kRegsControl <= kThreads * kRegsLaunch,
+              "register split exceeds the launch allocation");
 constexpr uint32_t kTmemCols = 512;   // two fp32 accumulators of 256 columns
-constexpr int kColsPerWarp = BN / 2;  // two warps share each 32-lane TMEM quarter
+constexpr int kRasterM = 8;           // tiles are visited in bands of 8 M-tiles
 
 struct GemmArgs {
     const float *a_side;  // [nside][G][m_pad]
     const float *w_side;  // [nside][G][n_pad]
     int64_t m_pad, n_pad;
     int M, N, G;
-    int tiles_n, num_tiles;
+    int tiles_m, tiles_n, num_tiles;
     const __half *bias;
     void *y;
     int y_type;
@@ -129,6 +137,19 @@ struct Smem {
     static constexpr int kTotal = kMisc + 16;
     static constexpr int kAlloc = kTotal + 1024;  // slack to align the base to 1024 bytes
 };
+
+// Tile visiting order: bands of kRasterM M-tiles, N-tiles inside a band, so
+// the CTAs resident at one time share few A row-blocks and W column-blocks
+// and both stay in L2.
+__device__ __forceinline__ void tile_coords(int tile, const GemmArgs &a, int &mt, int &nt)
+{
+    const int band = tile / (kRasterM * a.tiles_n);
+    const int m0 = band * kRasterM;
+    const int gm = min(kRasterM, a.tiles_m - m0);
+    const int r = tile - band * kRasterM * a.tiles_n;
+    mt = m0 + r % gm;
+    nt = r / gm;
+}
 
 __device__ __forceinline__ float4 ldg_f4(const float *p)
 {
@@ -159,6 +180,17 @@ __device__ __forceinline__ void store_row8(void *y, int64_t off, const float (&v
         d[0] = make_float4(v[0], v[1], v[2], v[3]);
         d[1] = make_float4(v[4], v[5], v[6], v[7]);
     }
+}
+
+template <int OUT>
+__device__ __forceinline__ void store_pair(void *y, int64_t off, float2 v)
+{
+    if (OUT == QUARTZ_OUT_F16)
+        *reinterpret_cast<__half2 *>(static_cast<__half *>(y) + off) = __floats2half2_rn(v.x, v.y);
+    else if (OUT == QUARTZ_OUT_BF16)
+        *reinterpret_cast<__nv_bfloat162 *>(static_cast<__nv_bfloat16 *>(y) + off) = __floats2bfloat162_rn(v.x, v.y);
+    else
+        *reinterpret_cast<float2 *>(static_cast<float *>(y) + off) = v;
 }
 
 template <int MODE, int OUT, bool DUMP>
@@ -221,8 +253,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             int it = 0;
             bool ok = true;
             for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
-                const int mt = tile / args.tiles_n;
-                const int nt = tile - mt * args.tiles_n;
+                int mt, nt;
+                tile_coords(tile, args, mt, nt);
                 for (int g = 0; g < G; ++g, ++it) {
                     const int s = it % kStages;
                     if (it >= kStages &&
@@ -293,104 +325,125 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else {
         regs_increase<kRegsEpilogue>();
         // ------------------------------------------------------------------
-        // Epilogue: warp w owns TMEM lanes 32*(w%4).. (tile rows) and columns
-        // [128*(w/4), +128).  Per group: y += s_a * (s_w * P_g); asymmetric
-        // first corrects P_g by the zero-point terms (exact integers in fp32).
+        // Epilogue.  Warp w reads TMEM lanes [32*(w%4), +32) (tile rows) and
+        // columns [64*(w/4), +64) with the 16x256b shape, so thread t holds
+        // rows 32*(w%4) + t/4 + {0, 8, 16, 24} and, in every 8-column block,
+        // the column pair 2*(t%4) + {0, 1}: 4 rows x 16 columns.  Per group:
+        // y += s_a * (s_w * P_g) on column pairs with f32x2 arithmetic;
+        // asymmetric first corrects P_g by the zero-point terms (exact
+        // integers in fp32).  The 64 column side values of the next group are
+        // prefetched into registers (16 lanes x float4) and staged per warp in
+        // shared memory; each thread then reads only its 8 column pairs.
         // ------------------------------------------------------------------
         const int quarter = warp & 3;
-        const int colh = warp >> 2;
-        const int row = quarter * 32 + lane;
+        const int slot = warp >> 2;
+        const int trow = lane >> 2;          // row offset inside each 8-row band
+        const int tcol = 2 * (lane & 3);     // column offset inside each 8-column block
         float *wbuf = reinterpret_cast<float *>(smem + L::kSide) + warp * (2 * NSIDE * kColsPerWarp);
         const int64_t a_plane = args.m_pad * G;
         const int64_t w_plane = args.n_pad * G;
 
-        int tile = blockIdx.x;
-        int g = 0;
-        // side values of the (tile, g) about to be processed, prefetched one group ahead
+        // prefetch cursor: the (tile, group) whose side values are fetched next
+        int p_tile = blockIdx.x, p_g = 0;
+        const float *p_w = nullptr, *p_a = nullptr;
+        auto cursor_tile = [&]() {
+            int mt, nt;
+            tile_coords(p_tile, args, mt, nt);
+            p_w = args.w_side + static_cast<int64_t>(nt) * BN + slot * kColsPerWarp + 4 * (lane & 15);
+            p_a = args.a_side + static_cast<int64_t>(mt) * BM + quarter * 32 + trow;
+        };
         float4 nxt_w[NSIDE];
-        float nxt_a[NSIDE];
-        auto fetch = [&](int t, int gg) {
-            const int mt = t / args.tiles_n;
-            const int nt = t - mt * args.tiles_n;
-            const int64_t col = static_cast<int64_t>(nt) * BN + colh * kColsPerWarp + 4 * lane;
-            const int64_t r = static_cast<int64_t>(mt) * BM + row;
+        float nxt_a[NSIDE][4];
+        auto fetch_advance = [&]() {
+            if (p_tile >= args.num_tiles) return;
 #pragma unroll
             for (int sd = 0; sd < NSIDE; ++sd) {
-                nxt_w[sd] = ldg_f4(args.w_side + sd * w_plane + static_cast<int64_t>(gg) * args.n_pad + col);
-                nxt_a[sd] = __ldg(args.a_side + sd * a_plane + static_cast<int64_t>(gg) * args.m_pad + r);
+                nxt_w[sd] = ldg_f4(p_w + sd * w_plane);
+#pragma unroll
+                for (int k = 0; k < 4; ++k) nxt_a[sd][k] = __ldg(p_a + sd * a_plane + 8 * k);
+            }
+            if (++p_g == G) {
+                p_g = 0;
+                p_tile += gridDim.x;
+                if (p_tile < args.num_tiles) cursor_tile();
+            } else {
+                p_w += args.n_pad;
+                p_a += args.m_pad;
             }
         };
-        if (tile < args.num_tiles) fetch(tile, 0);
+        if (p_tile < args.num_tiles) cursor_tile();
+        fetch_advance();
 
-        float2 acc[kColsPerWarp / 2];
+        // acc[k][i] = output pair (row trow + 8k, columns 8i + tcol + {0,1})
+        float2 acc[4][kColsPerWarp / 8];
         int it = 0;
         bool ok = true;
-        for (; tile < args.num_tiles && ok; tile += gridDim.x) {
-            const int mt = tile / args.tiles_n;
-            const int nt = tile - mt * args.tiles_n;
+        for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
+            int mt, nt;
+            tile_coords(tile, args, mt, nt);
 #pragma unroll
-            for (int j = 0; j < kColsPerWarp / 2; ++j) acc[j] = make_float2(0.f, 0.f);
-            for (g = 0; g < G; ++g, ++it) {
+            for (int k = 0; k < 4; ++k)
+#pragma unroll
+                for (int i = 0; i < kColsPerWarp / 8; ++i) acc[k][i] = make_float2(0.f, 0.f);
+            for (int g = 0; g < G; ++g, ++it) {
                 const int b = it & 1;
                 float *sb = wbuf + b * (NSIDE * kColsPerWarp);
-                float cur_a[NSIDE];
+                float cur_a[NSIDE][4];
 #pragma unroll
                 for (int sd = 0; sd < NSIDE; ++sd) {
-                    reinterpret_cast<float4 *>(sb + sd * kColsPerWarp)[lane] = nxt_w[sd];
-                    cur_a[sd] = nxt_a[sd];
+                    if (lane < kColsPerWarp / 4)
+                        reinterpret_cast<float4 *>(sb + sd * kColsPerWarp)[lane] = nxt_w[sd];
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) cur_a[sd][k] = nxt_a[sd][k];
                 }
                 __syncwarp();
-                {
-                    int nt2 = tile, ng = g + 1;
-                    if (ng == G) {
-                        ng = 0;
-                        nt2 = tile + gridDim.x;
-                    }
-                    if (nt2 < args.num_tiles) fetch(nt2, ng);
-                }
+                fetch_advance();
                 if (!mbar_wait_bounded(acc_full_bar(b), (it >> 1) & 1, abort_flag, args.dev_err,
                                        kWaitLimitNs)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                const float2 sa2 = make_float2(cur_a[0], cur_a[0]);
-                const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
-                                       static_cast<uint32_t>(b * BN + colh * kColsPerWarp);
+                const uint32_t tbase = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
+                                       static_cast<uint32_t>(b * BN + slot * kColsPerWarp);
 #pragma unroll
-                for (int c = 0; c < kColsPerWarp / 32; ++c) {
-                    uint32_t r[32];
-                    tmem_ld_32x32b_x32(taddr + c * 32, r);
-                    tmem_wait_ld();
-                    if (DUMP && g == args.partials_group) {
-                        const int64_t m = static_cast<int64_t>(mt) * BM + row;
-                        const int64_t n0 = static_cast<int64_t>(nt) * BN + colh * kColsPerWarp + c * 32;
-                        if (m < args.M) {
-                            for (int j = 0; j < 32; ++j)
-                                if (n0 + j < args.N)
-                                    args.partials[m * args.N + n0 + j] = __float2int_rn(__uint_as_float(r[j]));
-                        }
-                    }
+                for (int h = 0; h < 2; ++h) {            // lanes +0 / +16 of the quarter
 #pragma unroll
-                    for (int j4 = 0; j4 < 8; ++j4) {
-                        const int col = c * 32 + j4 * 4;
-                        const float4 sw = *reinterpret_cast<const float4 *>(sb + col);
-                        float2 p0 = make_float2(__uint_as_float(r[j4 * 4 + 0]), __uint_as_float(r[j4 * 4 + 1]));
-                        float2 p1 = make_float2(__uint_as_float(r[j4 * 4 + 2]), __uint_as_float(r[j4 * 4 + 3]));
-                        if (MODE == QUARTZ_ASYMMETRIC) {
-                            const float4 zw = *reinterpret_cast<const float4 *>(sb + kColsPerWarp + col);
-                            const float4 gw = *reinterpret_cast<const float4 *>(sb + 2 * kColsPerWarp + col);
-                            const float2 ua = make_float2(cur_a[2], cur_a[2]);
-                            const float2 nza = make_float2(-cur_a[1], -cur_a[1]);
-                            p0 = __ffma2_rn(make_float2(zw.x, zw.y), ua, p0);
-                            p1 = __ffma2_rn(make_float2(zw.z, zw.w), ua, p1);
-                            p0 = __ffma2_rn(nza, make_float2(gw.x, gw.y), p0);
-                            p1 = __ffma2_rn(nza, make_float2(gw.z, gw.w), p1);
+                    for (int c = 0; c < 2; ++c) {        // columns +0 / +32 of the slice
+                        uint32_t r[16];
+                        tmem_ld_16x256b_x4(tbase + (static_cast<uint32_t>(16 * h) << 16) + 32 * c, r);
+                        tmem_wait_ld(r);
+                        if (DUMP && g == args.partials_group) {
+#pragma unroll
+                            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                                for (int e = 0; e < 4; ++e) {
+                                    const int64_t m = static_cast<int64_t>(mt) * BM + quarter * 32 + 16 * h + trow + 8 * (e >> 1);
+                                    const int64_t n = static_cast<int64_t>(nt) * BN + slot * kColsPerWarp + 32 * c + 8 * i + tcol + (e & 1);
+                                    if (m < args.M && n < args.N)
+                                        args.partials[m * args.N + n] = __float2int_rn(__uint_as_float(r[4 * i + e]));
+                                }
                         }
-                        const float2 t0 = __fmul2_rn(p0, make_float2(sw.x, sw.y));
-                        const float2 t1 = __fmul2_rn(p1, make_float2(sw.z, sw.w));
-                        acc[col / 2] = __ffma2_rn(t0, sa2, acc[col / 2]);
-                        acc[col / 2 + 1] = __ffma2_rn(t1, sa2, acc[col / 2 + 1]);
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) {
+                            const int col = 32 * c + 8 * i + tcol;
+                            const float2 sw = *reinterpret_cast<const float2 *>(sb + col);
+#pragma unroll
+                            for (int e = 0; e < 2; ++e) {   // rows +0 / +8 of this lane half
+                                const int k = 2 * h + e;
+                                float2 p = make_float2(__uint_as_float(r[4 * i + 2 * e]),
+                                                       __uint_as_float(r[4 * i + 2 * e + 1]));
+                                if (MODE == QUARTZ_ASYMMETRIC) {
+                                    const float2 zw = *reinterpret_cast<const float2 *>(sb + kColsPerWarp + col);
+                                    const float2 gw = *reinterpret_cast<const float2 *>(sb + 2 * kColsPerWarp + col);
+                                    p = __ffma2_rn(zw, make_float2(cur_a[2][k], cur_a[2][k]), p);
+                                    p = __ffma2_rn(make_float2(-cur_a[1][k], -cur_a[1][k]), gw, p);
+                                }
+                                const float2 t = __fmul2_rn(p, sw);
+                                acc[k][4 * c + i] = __ffma2_rn(t, make_float2(cur_a[0][k], cur_a[0][k]),
+                                                               acc[k][4 * c + i]);
+                            }
+                        }
                     }
                 }
                 tc_fence_before();
@@ -398,32 +451,22 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (lane == 0) mbar_arrive(acc_empty_bar(b));
             }
             if (!ok) break;
-            // ---- store the finished tile row segment ------------------------
-            const int64_t m = static_cast<int64_t>(mt) * BM + row;
-            const int64_t nbase = static_cast<int64_t>(nt) * BN + colh * kColsPerWarp;
-            if (m < args.M) {
+            // ---- store the finished tile: 4 rows x 8 column pairs per thread ----
 #pragma unroll
-                for (int c8 = 0; c8 < kColsPerWarp / 8; ++c8) {
-                    const int64_t n = nbase + c8 * 8;
-                    if (n < args.N) {
-                        float v[8];
+            for (int k = 0; k < 4; ++k) {
+                const int64_t m = static_cast<int64_t>(mt) * BM + quarter * 32 + trow + 8 * k;
+                if (m >= args.M) continue;
 #pragma unroll
-                        for (int i = 0; i < 4; ++i) {
-                            v[2 * i] = acc[c8 * 4 + i].x;
-                            v[2 * i + 1] = acc[c8 * 4 + i].y;
-                        }
-                        if (args.bias) {
-                            const uint4 braw = __ldg(reinterpret_cast<const uint4 *>(args.bias + n));
-                            const uint32_t bw[4] = {braw.x, braw.y, braw.z, braw.w};
-#pragma unroll
-                            for (int i = 0; i < 4; ++i) {
-                                const float2 bf = __half22float2(*reinterpret_cast<const __half2 *>(&bw[i]));
-                                v[2 * i] = __fadd_rn(v[2 * i], bf.x);
-                                v[2 * i + 1] = __fadd_rn(v[2 * i + 1], bf.y);
-                            }
-                        }
-                        store_row8<OUT>(args.y, m * args.N + n, v);
+                for (int i = 0; i < kColsPerWarp / 8; ++i) {
+                    const int64_t n = static_cast<int64_t>(nt) * BN + slot * kColsPerWarp + 8 * i + tcol;
+                    if (n >= args.N) continue;
+                    float2 v = acc[k][i];
+                    if (args.bias) {
+                        const float2 bf = __half22float2(*reinterpret_cast<const __half2 *>(args.bias + n));
+                        v.x = __fadd_rn(v.x, bf.x);
+                        v.y = __fadd_rn(v.y, bf.y);
                     }
+                    store_pair<OUT>(args.y, m * args.N + n, v);
                 }
             }
         }
@@ -614,7 +657,8 @@ GemmArgs make_args(const LinearWorkspace &ws, int64_t M, int64_t N, int64_t K, c
     a.N = static_cast<int>(N);
     a.G = static_cast<int>(K / kGroupQ);
     a.tiles_n = static_cast<int>((N + BN - 1) / BN);
-    a.num_tiles = static_cast<int>((M + BM - 1) / BM) * a.tiles_n;
+    a.tiles_m = static_cast<int>((M + BM - 1) / BM);
+    a.num_tiles = a.tiles_m * a.tiles_n;
     a.bias = static_cast<const __half *>(bias);
     a.y = y;
     a.y_type = y_type;

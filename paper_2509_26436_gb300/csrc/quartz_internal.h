@@ -5,7 +5,7 @@
 #include <cstdint>
 #include <cuda_runtime.h>
 
-#include "../../include/quartz.h"
+#include "quartz.h"
 
 namespace quartz {
 
