@@ -165,6 +165,28 @@ int32_t quartz_linear_ex(const quartz_encoded_t *a, const quartz_encoded_t *w,
                          const void *bias_f16, void *y, int32_t y_type, void *workspace,
                          size_t workspace_bytes, const quartz_linear_opts_t *opts, void *stream);
 
+/* Scratch-free variant of quartz_linear, for callers that cannot allocate
+ * device memory (for example a plugin inside a host framework that owns all
+ * device memory through its own pool and forbids side allocations, or code on
+ * a latency-critical path where a cudaMalloc could synchronise the device).
+ * The paper has no counterpart to this entry point; it only changes where
+ * the scratch workspace lives.
+ *
+ * Same arguments, arithmetic and results as quartz_linear without the
+ * workspace arguments.  The workspace is a library-owned device array of
+ * QUARTZ_NOALLOC_SCRATCH_BYTES that every GPU loading the library holds until
+ * the process exits; the call allocates and frees nothing.
+ *   - Problems whose quartz_linear_workspace_size exceeds the array are
+ *     rejected with QUARTZ_ERR_WORKSPACE before anything is launched.
+ *   - The first call on a device looks up the array's device address with
+ *     that device current; make that first call before any stream capture.
+ *   - All calls on a device share the array and it keeps the last call's
+ *     contents.  Calls that overlap on the GPU (e.g. on two unordered
+ *     streams) race on it; serialise them. */
+#define QUARTZ_NOALLOC_SCRATCH_BYTES ((size_t)32 << 20)
+int32_t quartz_linear_noalloc(const quartz_encoded_t *a, const quartz_encoded_t *w,
+                              const void *bias_f16, void *y, int32_t y_type, void *stream);
+
 /* Synchronise `stream`, then read and clear the library's device error word.
  * Returns QUARTZ_OK, QUARTZ_ERR_TIMEOUT if a kernel gave up on a bounded
  * wait since the last call (its outputs are then invalid), or
