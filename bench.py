@@ -58,6 +58,25 @@ def peaks():
         return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS, "fallback"
 
 
+def gemm_traffic():
+    """DRAM bytes per GEMM launch from the committed ncu summary, if it was
+    taken on the GEMM source as it is now (else None)."""
+    import hashlib
+    csrc = os.path.join(ROOT, "paper_2509_26436_gb300", "csrc")
+    h = hashlib.sha256()
+    for f in ("linear.cu", "ptx.cuh"):
+        with open(os.path.join(csrc, f), "rb") as fh:
+            h.update(fh.read())
+    try:
+        with open(os.path.join(ROOT, "profiles", "gemm_tcgen05_flux_block.md")) as fh:
+            kv = dict(line.split(": ", 1) for line in fh if line.startswith(("gemm_source_sha16", "dram_bytes")))
+    except OSError:
+        return None
+    if kv.get("gemm_source_sha16", "").strip() != h.hexdigest()[:16]:
+        return None
+    return float(kv["dram_bytes_per_launch"])
+
+
 def dist_env():
     return (int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)),
             int(os.environ.get("LOCAL_RANK", 0)))
@@ -335,7 +354,7 @@ def run_ours(args):
     # ---- CPU oracle baseline (rank 0 only, N = 1) ---------------------------
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
-        rows = 8
+        rows = 128
         t, ops = oracle_sample(layers, rows, xs, ws)
         cpu = {"value": ops / t / 1e12, "unit": "TOPS", "cores": 1, "kind": "oracle",
                "sample": f"{rows} token rows of each of the 4 layers (encode + linear), "
@@ -352,7 +371,7 @@ def run_ours(args):
         "scaling": "weak", "vs_baseline": None, "dtype": "f16", "data": "synthetic",
         "config": layer_config(layers),
         "roofline": {"bound": "tensor", "achieved": gemm_tflops, "peak": tc_peak,
-                     "unit": "TFLOP/s", "frac": gemm_tflops / tc_peak, "traffic": None,
+                     "unit": "TFLOP/s", "frac": gemm_tflops / tc_peak, "traffic": gemm_traffic(),
                      "kernel": "gemm_tcgen05_kernel", "peak_source": f"{peak_src} bf16 burst",
                      "per_layer_ms": gemm_ms},
         "encode": {"kernel": "quantize_kernel", "gbs": enc_gbs, "peak_gbs": hbm_peak,
