@@ -38,13 +38,34 @@ constexpr int kGroupQ = 64;
 // ---------------------------------------------------------------------------
 // 1. expand
 // ---------------------------------------------------------------------------
+// Row order of the expanded weight operand: inside every block of 16 rows,
+// W row 4a + b is stored at position 4b + a (a 4x4 transposition; the map is
+// its own inverse).  The GEMM's TMEM column j then holds output column
+// perm16(j), which makes the four TMEM columns a thread reads with the
+// 16x128b shape four consecutive output columns.
+__host__ __device__ __forceinline__ int64_t perm16(int64_t r)
+{
+    return (r & ~int64_t(15)) | ((r & 3) << 2) | ((r >> 2) & 3);
+}
+
 template <int GS>
 __global__ void __launch_bounds__(256) expand_kernel(const uint32_t *__restrict__ codes,
                                                      const uint8_t *__restrict__ flags,
-                                                     int64_t n_chunks, uint4 *__restrict__ op)
+                                                     int64_t n_chunks, int64_t chunks_per_row,
+                                                     int64_t n_chunks_pad, int permute,
+                                                     uint4 *__restrict__ op)
 {
     const int64_t c = static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x;
-    if (c >= n_chunks) return;
+    if (c >= n_chunks_pad) return;
+    int64_t dst = c;
+    if (permute) {
+        const int64_t r = c / chunks_per_row;
+        dst = perm16(r) * chunks_per_row + (c - r * chunks_per_row);
+    }
+    if (c >= n_chunks) {  // padding rows up to a multiple of 16
+        op[dst] = make_uint4(0, 0, 0, 0);
+        return;
+    }
     const uint32_t word = codes[c];
     const int flag = flags[(c * 8) / GS];
     const int mul = 1 << flag;
@@ -56,7 +77,7 @@ __global__ void __launch_bounds__(256) expand_kernel(const uint32_t *__restrict_
         const __half2 h = __floats2half2_rn(static_cast<float>(c0 * mul), static_cast<float>(c1 * mul));
         o[i] = *reinterpret_cast<const uint32_t *>(&h);
     }
-    op[c] = make_uint4(o[0], o[1], o[2], o[3]);
+    op[dst] = make_uint4(o[0], o[1], o[2], o[3]);
 }
 
 // side[0][g][r] = s[r, g]; asymmetric adds side[1] = z and side[2] =
@@ -179,6 +200,22 @@ __device__ __forceinline__ void store_row8(void *y, int64_t off, const float (&v
         float4 *d = reinterpret_cast<float4 *>(static_cast<float *>(y) + off);
         d[0] = make_float4(v[0], v[1], v[2], v[3]);
         d[1] = make_float4(v[4], v[5], v[6], v[7]);
+    }
+}
+
+template <int OUT>
+__device__ __forceinline__ void store_quad(void *y, int64_t off, float4 v)
+{
+    if (OUT == QUARTZ_OUT_F16) {
+        const __half2 a = __floats2half2_rn(v.x, v.y), b = __floats2half2_rn(v.z, v.w);
+        *reinterpret_cast<uint2 *>(static_cast<__half *>(y) + off) =
+            make_uint2(*reinterpret_cast<const uint32_t *>(&a), *reinterpret_cast<const uint32_t *>(&b));
+    } else if (OUT == QUARTZ_OUT_BF16) {
+        const __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y), b = __floats2bfloat162_rn(v.z, v.w);
+        *reinterpret_cast<uint2 *>(static_cast<__nv_bfloat16 *>(y) + off) =
+            make_uint2(*reinterpret_cast<const uint32_t *>(&a), *reinterpret_cast<const uint32_t *>(&b));
+    } else {
+        *reinterpret_cast<float4 *>(static_cast<float *>(y) + off) = v;
     }
 }
 
@@ -326,19 +363,22 @@ __global__ void __launch_bounds__(kThreads, 1)
         regs_increase<kRegsEpilogue>();
         // ------------------------------------------------------------------
         // Epilogue.  Warp w reads TMEM lanes [32*(w%4), +32) (tile rows) and
-        // columns [64*(w/4), +64) with the 16x256b shape, so thread t holds
-        // rows 32*(w%4) + t/4 + {0, 8, 16, 24} and, in every 8-column block,
-        // the column pair 2*(t%4) + {0, 1}: 4 rows x 16 columns.  Per group:
-        // y += s_a * (s_w * P_g) on column pairs with f32x2 arithmetic;
-        // asymmetric first corrects P_g by the zero-point terms (exact
-        // integers in fp32).  The 64 column side values of the next group are
-        // prefetched into registers (16 lanes x float4) and staged per warp in
-        // shared memory; each thread then reads only its 8 column pairs.
+        // TMEM columns [64*(w/4), +64) with the 16x128b shape: per 16-column
+        // chunk, thread t holds TMEM columns t%4 + {0,4,8,12} of lanes t/4 and
+        // t/4 + 8 (and t/4 + 16, t/4 + 24 from the second lane half).  With
+        // the weight rows transposed inside each 16-row block, those four TMEM
+        // columns are the four consecutive output columns 4*(t%4) + {0..3},
+        // so one 16-byte shared load gives their scales (each used for four
+        // rows) and the stores are 4-wide.  Per group, y += s_a * (s_w * P_g)
+        // on (row, row + 8) pairs with f32x2 arithmetic (asymmetric first adds
+        // the exact integer zero-point terms to P_g).  Side values of the next
+        // group are prefetched one group ahead into registers and staged per
+        // warp in shared memory.
         // ------------------------------------------------------------------
         const int quarter = warp & 3;
         const int slot = warp >> 2;
         const int trow = lane >> 2;          // row offset inside each 8-row band
-        const int tcol = 2 * (lane & 3);     // column offset inside each 8-column block
+        const int tq = 4 * (lane & 3);       // first of this thread's 4 output columns in a 16-column chunk
         float *wbuf = reinterpret_cast<float *>(smem + L::kSide) + warp * (2 * NSIDE * kColsPerWarp);
         const int64_t a_plane = args.m_pad * G;
         const int64_t w_plane = args.n_pad * G;
@@ -374,17 +414,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (p_tile < args.num_tiles) cursor_tile();
         fetch_advance();
 
-        // acc[k][i] = output pair (row trow + 8k, columns 8i + tcol + {0,1})
-        float2 acc[4][kColsPerWarp / 8];
+        // acc[h][j]: output column 16*(j/4) + tq + j%4 of this warp's slice,
+        // rows trow + 16h (.x) and trow + 16h + 8 (.y)
+        float2 acc[2][16];
         int it = 0;
         bool ok = true;
         for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
             int mt, nt;
             tile_coords(tile, args, mt, nt);
 #pragma unroll
-            for (int k = 0; k < 4; ++k)
+            for (int h = 0; h < 2; ++h)
 #pragma unroll
-                for (int i = 0; i < kColsPerWarp / 8; ++i) acc[k][i] = make_float2(0.f, 0.f);
+                for (int j = 0; j < 16; ++j) acc[h][j] = make_float2(0.f, 0.f);
             for (int g = 0; g < G; ++g, ++it) {
                 const int b = it & 1;
                 float *sb = wbuf + b * (NSIDE * kColsPerWarp);
@@ -407,42 +448,41 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t tbase = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
                                        static_cast<uint32_t>(b * BN + slot * kColsPerWarp);
 #pragma unroll
-                for (int h = 0; h < 2; ++h) {            // lanes +0 / +16 of the quarter
+                for (int chunk = 0; chunk < 4; ++chunk) {    // 16-column chunks of the slice
+                    uint32_t r[16];
+                    tmem_ld_16x128b_x4_pair(tbase + 16 * chunk, tbase + (16u << 16) + 16 * chunk, r);
+                    tmem_wait_ld(r);
+                    const float4 sw = *reinterpret_cast<const float4 *>(sb + 16 * chunk + tq);
+                    const float swv[4] = {sw.x, sw.y, sw.z, sw.w};
+                    float4 zw4 = make_float4(0.f, 0.f, 0.f, 0.f), gw4 = zw4;
+                    if (MODE == QUARTZ_ASYMMETRIC) {
+                        zw4 = *reinterpret_cast<const float4 *>(sb + kColsPerWarp + 16 * chunk + tq);
+                        gw4 = *reinterpret_cast<const float4 *>(sb + 2 * kColsPerWarp + 16 * chunk + tq);
+                    }
+                    const float zwv[4] = {zw4.x, zw4.y, zw4.z, zw4.w};
+                    const float gwv[4] = {gw4.x, gw4.y, gw4.z, gw4.w};
 #pragma unroll
-                    for (int c = 0; c < 2; ++c) {        // columns +0 / +32 of the slice
-                        uint32_t r[16];
-                        tmem_ld_16x256b_x4(tbase + (static_cast<uint32_t>(16 * h) << 16) + 32 * c, r);
-                        tmem_wait_ld(r);
-                        if (DUMP && g == args.partials_group) {
-#pragma unroll
-                            for (int i = 0; i < 4; ++i)
-#pragma unroll
-                                for (int e = 0; e < 4; ++e) {
-                                    const int64_t m = static_cast<int64_t>(mt) * BM + quarter * 32 + 16 * h + trow + 8 * (e >> 1);
-                                    const int64_t n = static_cast<int64_t>(nt) * BN + slot * kColsPerWarp + 32 * c + 8 * i + tcol + (e & 1);
-                                    if (m < args.M && n < args.N)
-                                        args.partials[m * args.N + n] = __float2int_rn(__uint_as_float(r[4 * i + e]));
-                                }
-                        }
+                    for (int h = 0; h < 2; ++h) {
 #pragma unroll
                         for (int i = 0; i < 4; ++i) {
-                            const int col = 32 * c + 8 * i + tcol;
-                            const float2 sw = *reinterpret_cast<const float2 *>(sb + col);
-#pragma unroll
-                            for (int e = 0; e < 2; ++e) {   // rows +0 / +8 of this lane half
-                                const int k = 2 * h + e;
-                                float2 p = make_float2(__uint_as_float(r[4 * i + 2 * e]),
-                                                       __uint_as_float(r[4 * i + 2 * e + 1]));
-                                if (MODE == QUARTZ_ASYMMETRIC) {
-                                    const float2 zw = *reinterpret_cast<const float2 *>(sb + kColsPerWarp + col);
-                                    const float2 gw = *reinterpret_cast<const float2 *>(sb + 2 * kColsPerWarp + col);
-                                    p = __ffma2_rn(zw, make_float2(cur_a[2][k], cur_a[2][k]), p);
-                                    p = __ffma2_rn(make_float2(-cur_a[1][k], -cur_a[1][k]), gw, p);
+                            float2 p = make_float2(__uint_as_float(r[8 * h + 2 * i]), __uint_as_float(r[8 * h + 2 * i + 1]));
+                            if (DUMP && g == args.partials_group) {
+                                const int64_t m = static_cast<int64_t>(mt) * BM + quarter * 32 + 16 * h + trow;
+                                const int64_t n = static_cast<int64_t>(nt) * BN + slot * kColsPerWarp + 16 * chunk + tq + i;
+                                if (n < args.N) {
+                                    if (m < args.M) args.partials[m * args.N + n] = __float2int_rn(p.x);
+                                    if (m + 8 < args.M) args.partials[(m + 8) * args.N + n] = __float2int_rn(p.y);
                                 }
-                                const float2 t = __fmul2_rn(p, sw);
-                                acc[k][4 * c + i] = __ffma2_rn(t, make_float2(cur_a[0][k], cur_a[0][k]),
-                                                               acc[k][4 * c + i]);
                             }
+                            if (MODE == QUARTZ_ASYMMETRIC) {
+                                const float2 ua = make_float2(cur_a[2][2 * h], cur_a[2][2 * h + 1]);
+                                const float2 nza = make_float2(-cur_a[1][2 * h], -cur_a[1][2 * h + 1]);
+                                p = __ffma2_rn(make_float2(zwv[i], zwv[i]), ua, p);
+                                p = __ffma2_rn(nza, make_float2(gwv[i], gwv[i]), p);
+                            }
+                            const float2 t = __fmul2_rn(p, make_float2(swv[i], swv[i]));
+                            acc[h][4 * chunk + i] = __ffma2_rn(t, make_float2(cur_a[0][2 * h], cur_a[0][2 * h + 1]),
+                                                               acc[h][4 * chunk + i]);
                         }
                     }
                 }
@@ -451,24 +491,34 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (lane == 0) mbar_arrive(acc_empty_bar(b));
             }
             if (!ok) break;
-            // ---- store the finished tile: 4 rows x 8 column pairs per thread ----
+            // ---- store: 4 rows x 4 chunks of 4 consecutive columns per thread ----
 #pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                const int64_t m = static_cast<int64_t>(mt) * BM + quarter * 32 + trow + 8 * k;
-                if (m >= args.M) continue;
+            for (int h = 0; h < 2; ++h)
 #pragma unroll
-                for (int i = 0; i < kColsPerWarp / 8; ++i) {
-                    const int64_t n = static_cast<int64_t>(nt) * BN + slot * kColsPerWarp + 8 * i + tcol;
-                    if (n >= args.N) continue;
-                    float2 v = acc[k][i];
-                    if (args.bias) {
-                        const float2 bf = __half22float2(*reinterpret_cast<const __half2 *>(args.bias + n));
-                        v.x = __fadd_rn(v.x, bf.x);
-                        v.y = __fadd_rn(v.y, bf.y);
+                for (int e = 0; e < 2; ++e) {
+                    const int64_t m = static_cast<int64_t>(mt) * BM + quarter * 32 + 16 * h + 8 * e + trow;
+                    if (m >= args.M) continue;
+#pragma unroll
+                    for (int chunk = 0; chunk < 4; ++chunk) {
+                        const int64_t n = static_cast<int64_t>(nt) * BN + slot * kColsPerWarp + 16 * chunk + tq;
+                        if (n >= args.N) continue;
+                        float4 v;
+                        v.x = e ? acc[h][4 * chunk + 0].y : acc[h][4 * chunk + 0].x;
+                        v.y = e ? acc[h][4 * chunk + 1].y : acc[h][4 * chunk + 1].x;
+                        v.z = e ? acc[h][4 * chunk + 2].y : acc[h][4 * chunk + 2].x;
+                        v.w = e ? acc[h][4 * chunk + 3].y : acc[h][4 * chunk + 3].x;
+                        if (args.bias) {
+                            const uint2 braw = __ldg(reinterpret_cast<const uint2 *>(args.bias + n));
+                            const float2 b0 = __half22float2(*reinterpret_cast<const __half2 *>(&braw.x));
+                            const float2 b1 = __half22float2(*reinterpret_cast<const __half2 *>(&braw.y));
+                            v.x = __fadd_rn(v.x, b0.x);
+                            v.y = __fadd_rn(v.y, b0.y);
+                            v.z = __fadd_rn(v.z, b1.x);
+                            v.w = __fadd_rn(v.w, b1.y);
+                        }
+                        store_quad<OUT>(args.y, m * args.N + n, v);
                     }
-                    store_pair<OUT>(args.y, m * args.N + n, v);
                 }
-            }
         }
     }
 
@@ -501,7 +551,7 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const __half *__restrict
             const int r = i / kGroupQ, k = i % kGroupQ;
             const int64_t kk = static_cast<int64_t>(g) * kGroupQ + k;
             sa[r][k] = (m0 + r < args.M) ? static_cast<int16_t>(__half2float(a_op[(int64_t)(m0 + r) * K + kk])) : 0;
-            sw[r][k] = (n0 + r < args.N) ? static_cast<int16_t>(__half2float(w_op[(int64_t)(n0 + r) * K + kk])) : 0;
+            sw[r][k] = (n0 + r < args.N) ? static_cast<int16_t>(__half2float(w_op[perm16(n0 + r) * K + kk])) : 0;
         }
         __syncthreads();
         int p[4][4] = {};
@@ -675,7 +725,7 @@ size_t linear_workspace_bytes(int64_t M, int64_t N, int64_t K, int mode)
     const int nside = mode == QUARTZ_ASYMMETRIC ? 3 : 1;
     const int64_t G = K / kGroupQ;
     size_t b = align256(static_cast<size_t>(M) * K * 2);
-    b += align256(static_cast<size_t>(N) * K * 2);
+    b += align256(static_cast<size_t>(round_up(N, 16)) * K * 2);
     b += align256(static_cast<size_t>(nside) * G * round_up(M > 0 ? M : 1, BM) * 4);
     b += align256(static_cast<size_t>(nside) * G * round_up(N, BN) * 4);
     return b;
@@ -693,7 +743,7 @@ void linear_workspace_carve(void *base, int64_t M, int64_t N, int64_t K, int mod
     ws->a_op = p;
     p += align256(static_cast<size_t>(M) * K * 2);
     ws->w_op = p;
-    p += align256(static_cast<size_t>(N) * K * 2);
+    p += align256(static_cast<size_t>(round_up(N, 16)) * K * 2);
     ws->a_side = reinterpret_cast<float *>(p);
     p += align256(static_cast<size_t>(nside) * G * ws->m_pad * 4);
     ws->w_side = reinterpret_cast<float *>(p);
@@ -702,16 +752,20 @@ void linear_workspace_carve(void *base, int64_t M, int64_t N, int64_t K, int mod
 cudaError_t launch_expand(const quartz_encoded_t *e, void *op, float *side, int64_t rows_pad,
                           int is_a, cudaStream_t s)
 {
-    const int64_t n_chunks = e->rows * e->K / 8;
-    if (n_chunks > 0) {
-        const unsigned blocks = static_cast<unsigned>((n_chunks + 255) / 256);
+    const int64_t cpr = e->K / 8;
+    const int64_t n_chunks = e->rows * cpr;
+    // the weight operand is row-permuted and padded to a multiple of 16 rows
+    const int64_t n_chunks_pad = is_a ? n_chunks : round_up(e->rows, 16) * cpr;
+    if (n_chunks_pad > 0) {
+        const unsigned blocks = static_cast<unsigned>((n_chunks_pad + 255) / 256);
         const uint32_t *codes = reinterpret_cast<const uint32_t *>(e->codes);
         uint4 *o = static_cast<uint4 *>(op);
+        const int perm = is_a ? 0 : 1;
         switch (e->p.group_s) {
-            case 8: expand_kernel<8><<<blocks, 256, 0, s>>>(codes, e->flags, n_chunks, o); break;
-            case 16: expand_kernel<16><<<blocks, 256, 0, s>>>(codes, e->flags, n_chunks, o); break;
-            case 32: expand_kernel<32><<<blocks, 256, 0, s>>>(codes, e->flags, n_chunks, o); break;
-            default: expand_kernel<64><<<blocks, 256, 0, s>>>(codes, e->flags, n_chunks, o); break;
+            case 8: expand_kernel<8><<<blocks, 256, 0, s>>>(codes, e->flags, n_chunks, cpr, n_chunks_pad, perm, o); break;
+            case 16: expand_kernel<16><<<blocks, 256, 0, s>>>(codes, e->flags, n_chunks, cpr, n_chunks_pad, perm, o); break;
+            case 32: expand_kernel<32><<<blocks, 256, 0, s>>>(codes, e->flags, n_chunks, cpr, n_chunks_pad, perm, o); break;
+            default: expand_kernel<64><<<blocks, 256, 0, s>>>(codes, e->flags, n_chunks, cpr, n_chunks_pad, perm, o); break;
         }
         cudaError_t err = cudaGetLastError();
         if (err != cudaSuccess) return err;
@@ -732,7 +786,7 @@ cudaError_t launch_gemm_tcgen05(const LinearWorkspace &ws, int64_t M, int64_t N,
 {
     if (M == 0) return cudaSuccess;
     CUtensorMap ta, tw;
-    if (!make_operand_map(&ta, ws.a_op, M, K, BM) || !make_operand_map(&tw, ws.w_op, N, K, BN))
+    if (!make_operand_map(&ta, ws.a_op, M, K, BM) || !make_operand_map(&tw, ws.w_op, round_up(N, 16), K, BN))
         return cudaErrorInvalidValue;
     const GemmArgs args = make_args(ws, M, N, K, bias, y, y_type, partials, partials_group, dev_err);
     return mode == QUARTZ_ASYMMETRIC ? launch_tc_out<QUARTZ_ASYMMETRIC>(ta, tw, args, y_type, s)

@@ -212,18 +212,19 @@ __device__ __forceinline__ void tmem_wait_ld(uint32_t (&r)[16])
                  : "memory");
 }
 
-// 16 lanes x (4 x 256 bits) of TMEM.  For every 8-column block i (0..3),
-// thread t receives r[4i+0..1] = (lane t/4, columns 8i + 2(t%4) + {0,1}) and
-// r[4i+2..3] = (lane t/4 + 8, the same columns), relative to `taddr`.
-__device__ __forceinline__ void tmem_ld_16x256b_x4(uint32_t taddr, uint32_t (&r)[16])
+// Two loads of 16 lanes x (4 x 128 bits) of TMEM, at t0 and t1.  For every
+// 4-column block i (0..3) of the load at t0, thread t receives r[2i] = (lane
+// t/4, column 4i + t%4) and r[2i+1] = (lane t/4 + 8, the same column); the
+// load at t1 fills r[8..15] the same way.
+__device__ __forceinline__ void tmem_ld_16x128b_x4_pair(uint32_t t0, uint32_t t1, uint32_t (&r)[16])
 {
     asm volatile(
-        "tcgen05.ld.sync.aligned.16x256b.x4.b32 "
-        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        "tcgen05.ld.sync.aligned.16x128b.x4.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%16];\n\t"
+        "tcgen05.ld.sync.aligned.16x128b.x4.b32 {%8,%9,%10,%11,%12,%13,%14,%15}, [%17];"
         : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
           "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
           "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-        : "r"(taddr)
+        : "r"(t0), "r"(t1)
         : "memory");
 }
 
