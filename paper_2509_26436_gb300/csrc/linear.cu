@@ -80,9 +80,18 @@ __global__ void __launch_bounds__(256) expand_kernel(const uint32_t *__restrict_
     op[dst] = make_uint4(o[0], o[1], o[2], o[3]);
 }
 
-// side[0][g][r] = s[r, g]; asymmetric adds side[1] = z and side[2] =
+// Position of activation row r in its group's side-value row: inside every
+// block of 32 rows, row 8a + b sits at 4b + a, so that the four rows
+// b + {0, 8, 16, 24} one epilogue thread scales are one 16-byte vector.
+__host__ __device__ __forceinline__ int64_t perm32(int64_t r)
+{
+    return (r & ~int64_t(31)) | ((r & 7) << 2) | ((r >> 3) & 3);
+}
+
+// side[0][g][.] = s[r, g]; asymmetric adds side[1] = z and side[2] =
 // (is_a ? 64 z - gsum : gsum), so that the epilogue's integer correction is
 // P + z_w * (64 z_a - A_g) - z_a * W_g.  Rows in [rows, rows_pad) are 0.
+// Weight rows are stored in natural order, activation rows at perm32(r).
 __global__ void side_kernel(const __half *__restrict__ scales, const int8_t *__restrict__ zeros,
                             const int32_t *__restrict__ gsum, int64_t rows, int64_t rows_pad,
                             int G, int nside, int is_a, float *__restrict__ side)
@@ -92,13 +101,14 @@ __global__ void side_kernel(const __half *__restrict__ scales, const int8_t *__r
     if (i >= total) return;
     const int64_t g = i / rows_pad;
     const int64_t r = i - g * rows_pad;
+    const int64_t o = g * rows_pad + (is_a ? perm32(r) : r);
     const bool in = r < rows;
-    side[i] = in ? __half2float(scales[r * G + g]) : 0.f;
+    side[o] = in ? __half2float(scales[r * G + g]) : 0.f;
     if (nside > 1) {
         const float z = in ? static_cast<float>(zeros[r * G + g]) : 0.f;
         const float gs = in ? static_cast<float>(gsum[r * G + g]) : 0.f;
-        side[total + i] = z;
-        side[2 * total + i] = is_a ? (static_cast<float>(kGroupQ) * z - gs) : gs;
+        side[total + o] = z;
+        side[2 * total + o] = is_a ? (static_cast<float>(kGroupQ) * z - gs) : gs;
     }
 }
 
@@ -147,13 +157,19 @@ struct GemmArgs {
     int *dev_err;
 };
 
+// Shared memory: the operand stages, then a ring of side-value slots (one
+// group's NSIDE x BM activation and NSIDE x BN weight values each, copied by
+// the producer and released by the epilogue), then the mbarriers.
 template <int NSIDE>
 struct Smem {
     static constexpr int kOperands = 0;
     static constexpr int kSide = kStages * kStageBytes;
-    static constexpr int kSideBytes = kEpiWarps * 2 * NSIDE * kColsPerWarp * 4;
-    static constexpr int kBars = kSide + kSideBytes;
-    static constexpr int kNumBars = 2 * kStages + 4 + 1;  // full, empty, acc_full x2, acc_empty x2, drain
+    static constexpr int kSideSlots = NSIDE == 1 ? 8 : 4;
+    static constexpr int kSideABytes = NSIDE * BM * 4;
+    static constexpr int kSideSlotBytes = NSIDE * (BM + BN) * 4;
+    static constexpr int kBars = kSide + kSideSlots * kSideSlotBytes;
+    // full, empty, acc_full x2, acc_empty x2, drain, side_full, side_empty
+    static constexpr int kNumBars = 2 * kStages + 4 + 1 + 2 * kSideSlots;
     static constexpr int kMisc = kBars + kNumBars * 8;
     static constexpr int kTotal = kMisc + 16;
     static constexpr int kAlloc = kTotal + 1024;  // slack to align the base to 1024 bytes
@@ -172,37 +188,6 @@ __device__ __forceinline__ void tile_coords(int tile, const GemmArgs &a, int &mt
     nt = r / gm;
 }
 
-__device__ __forceinline__ float4 ldg_f4(const float *p)
-{
-    return __ldg(reinterpret_cast<const float4 *>(p));
-}
-
-template <int OUT>
-__device__ __forceinline__ void store_row8(void *y, int64_t off, const float (&v)[8])
-{
-    if (OUT == QUARTZ_OUT_F16) {
-        uint32_t o[4];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const __half2 h = __floats2half2_rn(v[2 * i], v[2 * i + 1]);
-            o[i] = *reinterpret_cast<const uint32_t *>(&h);
-        }
-        *reinterpret_cast<uint4 *>(static_cast<__half *>(y) + off) = make_uint4(o[0], o[1], o[2], o[3]);
-    } else if (OUT == QUARTZ_OUT_BF16) {
-        uint32_t o[4];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const __nv_bfloat162 h = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
-            o[i] = *reinterpret_cast<const uint32_t *>(&h);
-        }
-        *reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(y) + off) = make_uint4(o[0], o[1], o[2], o[3]);
-    } else {
-        float4 *d = reinterpret_cast<float4 *>(static_cast<float *>(y) + off);
-        d[0] = make_float4(v[0], v[1], v[2], v[3]);
-        d[1] = make_float4(v[4], v[5], v[6], v[7]);
-    }
-}
-
 template <int OUT>
 __device__ __forceinline__ void store_quad(void *y, int64_t off, float4 v)
 {
@@ -217,17 +202,6 @@ __device__ __forceinline__ void store_quad(void *y, int64_t off, float4 v)
     } else {
         *reinterpret_cast<float4 *>(static_cast<float *>(y) + off) = v;
     }
-}
-
-template <int OUT>
-__device__ __forceinline__ void store_pair(void *y, int64_t off, float2 v)
-{
-    if (OUT == QUARTZ_OUT_F16)
-        *reinterpret_cast<__half2 *>(static_cast<__half *>(y) + off) = __floats2half2_rn(v.x, v.y);
-    else if (OUT == QUARTZ_OUT_BF16)
-        *reinterpret_cast<__nv_bfloat162 *>(static_cast<__nv_bfloat16 *>(y) + off) = __floats2bfloat162_rn(v.x, v.y);
-    else
-        *reinterpret_cast<float2 *>(static_cast<float *>(y) + off) = v;
 }
 
 template <int MODE, int OUT, bool DUMP>
@@ -249,6 +223,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto acc_full_bar = [&](int b) { return bar_base + 8u * (2 * kStages + b); };
     auto acc_empty_bar = [&](int b) { return bar_base + 8u * (2 * kStages + 2 + b); };
     const uint32_t drain_bar = bar_base + 8u * (2 * kStages + 4);
+    auto side_full_bar = [&](int s) { return bar_base + 8u * (2 * kStages + 5 + s); };
+    auto side_empty_bar = [&](int s) { return bar_base + 8u * (2 * kStages + 5 + L::kSideSlots + s); };
     uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(smem + L::kMisc);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + L::kMisc + 4);
 
@@ -262,6 +238,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(acc_empty_bar(b), kEpiWarps);
         }
         mbar_init(drain_bar, 1);
+        for (int s = 0; s < L::kSideSlots; ++s) {
+            mbar_init(side_full_bar(s), 1);
+            mbar_init(side_empty_bar(s), kEpiWarps);
+        }
         *abort_flag = 0;
         fence_mbar_init();
     }
@@ -285,14 +265,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ------------------------------------------------------------------
         // TMA producer: one stage = one 64-wide group of A (128 rows) and W
         // (256 rows).  Rows past M or N are zero-filled by the tensor map.
+        // The group's side values (scales; asymmetric also zero-point terms)
+        // go by bulk copy into their own ring slot, which the epilogue frees.
         // ------------------------------------------------------------------
         if (lane == 0) {
-            int it = 0;
+            constexpr int S = L::kSideSlots;
+            const int64_t a_plane = args.m_pad * G;
+            const int64_t w_plane = args.n_pad * G;
+            int it = 0;       // groups whose operand copies were issued
+            int it_side = 0;  // groups whose side-value copies were issued
             bool ok = true;
             for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
                 int mt, nt;
                 tile_coords(tile, args, mt, nt);
-                for (int g = 0; g < G; ++g, ++it) {
+                for (int g = 0; g < G; ++g) {
                     const int s = it % kStages;
                     if (it >= kStages &&
                         !mbar_wait_bounded(empty_bar(s), ((it / kStages) - 1) & 1, abort_flag,
@@ -304,14 +290,38 @@ __global__ void __launch_bounds__(kThreads, 1)
                     mbar_arrive_expect_tx(full_bar(s), kStageBytes);
                     tma_load_2d(sa, &tmap_a, g * BK, mt * BM, full_bar(s));
                     tma_load_2d(sa + kABytes, &tmap_w, g * BK, nt * BN, full_bar(s));
+                    ++it;
+
+                    const int ss = it_side % S;
+                    if (it_side >= S && !mbar_wait_bounded(side_empty_bar(ss), ((it_side / S) - 1) & 1,
+                                                           abort_flag, args.dev_err, kWaitLimitNs)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t sd_dst = smem_base + L::kSide + ss * L::kSideSlotBytes;
+                    mbar_arrive_expect_tx(side_full_bar(ss), L::kSideSlotBytes);
+                    const float *src_a = args.a_side + static_cast<int64_t>(g) * args.m_pad + static_cast<int64_t>(mt) * BM;
+                    const float *src_w = args.w_side + static_cast<int64_t>(g) * args.n_pad + static_cast<int64_t>(nt) * BN;
+#pragma unroll
+                    for (int sd = 0; sd < NSIDE; ++sd) {
+                        bulk_load(sd_dst + sd * BM * 4, src_a + sd * a_plane, BM * 4, side_full_bar(ss));
+                        bulk_load(sd_dst + L::kSideABytes + sd * BN * 4, src_w + sd * w_plane, BN * 4,
+                                  side_full_bar(ss));
+                    }
+                    ++it_side;
                 }
             }
             // Never leave the CTA with copies in flight: wait for the last
-            // load issued into every stage (bounded, even after an abort).
+            // load issued into every stage and side slot (bounded, even after
+            // an abort).
             int zero = 0;
             for (int s = 0; s < kStages && s < it; ++s) {
                 const int last = it - 1 - ((it - 1 - s) % kStages);
                 mbar_wait_bounded(full_bar(s), (last / kStages) & 1, &zero, args.dev_err, kWaitLimitNs);
+            }
+            for (int s = 0; s < S && s < it_side; ++s) {
+                const int last = it_side - 1 - ((it_side - 1 - s) % S);
+                mbar_wait_bounded(side_full_bar(s), (last / S) & 1, &zero, args.dev_err, kWaitLimitNs);
             }
         }
         __syncwarp();
@@ -369,50 +379,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         // the weight rows transposed inside each 16-row block, those four TMEM
         // columns are the four consecutive output columns 4*(t%4) + {0..3},
         // so one 16-byte shared load gives their scales (each used for four
-        // rows) and the stores are 4-wide.  Per group, y += s_a * (s_w * P_g)
-        // on (row, row + 8) pairs with f32x2 arithmetic (asymmetric first adds
-        // the exact integer zero-point terms to P_g).  Side values of the next
-        // group are prefetched one group ahead into registers and staged per
-        // warp in shared memory.
+        // rows) and the stores are 4-wide.  The thread's four row scales are
+        // one 16-byte load as well (rows are permuted in the side values).
+        // Per group, y += s_a * (s_w * P_g) on (row, row + 8) pairs with
+        // f32x2 arithmetic (asymmetric first adds the exact integer
+        // zero-point terms to P_g).
         // ------------------------------------------------------------------
+        constexpr int S = L::kSideSlots;
         const int quarter = warp & 3;
         const int slot = warp >> 2;
         const int trow = lane >> 2;          // row offset inside each 8-row band
         const int tq = 4 * (lane & 3);       // first of this thread's 4 output columns in a 16-column chunk
-        float *wbuf = reinterpret_cast<float *>(smem + L::kSide) + warp * (2 * NSIDE * kColsPerWarp);
-        const int64_t a_plane = args.m_pad * G;
-        const int64_t w_plane = args.n_pad * G;
-
-        // prefetch cursor: the (tile, group) whose side values are fetched next
-        int p_tile = blockIdx.x, p_g = 0;
-        const float *p_w = nullptr, *p_a = nullptr;
-        auto cursor_tile = [&]() {
-            int mt, nt;
-            tile_coords(p_tile, args, mt, nt);
-            p_w = args.w_side + static_cast<int64_t>(nt) * BN + slot * kColsPerWarp + 4 * (lane & 15);
-            p_a = args.a_side + static_cast<int64_t>(mt) * BM + quarter * 32 + trow;
-        };
-        float4 nxt_w[NSIDE];
-        float nxt_a[NSIDE][4];
-        auto fetch_advance = [&]() {
-            if (p_tile >= args.num_tiles) return;
-#pragma unroll
-            for (int sd = 0; sd < NSIDE; ++sd) {
-                nxt_w[sd] = ldg_f4(p_w + sd * w_plane);
-#pragma unroll
-                for (int k = 0; k < 4; ++k) nxt_a[sd][k] = __ldg(p_a + sd * a_plane + 8 * k);
-            }
-            if (++p_g == G) {
-                p_g = 0;
-                p_tile += gridDim.x;
-                if (p_tile < args.num_tiles) cursor_tile();
-            } else {
-                p_w += args.n_pad;
-                p_a += args.m_pad;
-            }
-        };
-        if (p_tile < args.num_tiles) cursor_tile();
-        fetch_advance();
 
         // acc[h][j]: output column 16*(j/4) + tq + j%4 of this warp's slice,
         // rows trow + 16h (.x) and trow + 16h + 8 (.y)
@@ -420,29 +397,35 @@ __global__ void __launch_bounds__(kThreads, 1)
         int it = 0;
         bool ok = true;
         for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
-            int mt, nt;
-            tile_coords(tile, args, mt, nt);
 #pragma unroll
             for (int h = 0; h < 2; ++h)
 #pragma unroll
                 for (int j = 0; j < 16; ++j) acc[h][j] = make_float2(0.f, 0.f);
             for (int g = 0; g < G; ++g, ++it) {
                 const int b = it & 1;
-                float *sb = wbuf + b * (NSIDE * kColsPerWarp);
-                float cur_a[NSIDE][4];
-#pragma unroll
-                for (int sd = 0; sd < NSIDE; ++sd) {
-                    if (lane < kColsPerWarp / 4)
-                        reinterpret_cast<float4 *>(sb + sd * kColsPerWarp)[lane] = nxt_w[sd];
-#pragma unroll
-                    for (int k = 0; k < 4; ++k) cur_a[sd][k] = nxt_a[sd][k];
+                const int ss = it % S;
+                if (!mbar_wait_bounded(side_full_bar(ss), (it / S) & 1, abort_flag, args.dev_err,
+                                       kWaitLimitNs)) {
+                    ok = false;
+                    break;
                 }
-                __syncwarp();
-                fetch_advance();
+                const uint32_t side_a = smem_base + L::kSide + ss * L::kSideSlotBytes + (quarter * 32 + 4 * trow) * 4;
+                const uint32_t side_w = smem_base + L::kSide + ss * L::kSideSlotBytes + L::kSideABytes +
+                                        (slot * kColsPerWarp + tq) * 4;
                 if (!mbar_wait_bounded(acc_full_bar(b), (it >> 1) & 1, abort_flag, args.dev_err,
                                        kWaitLimitNs)) {
                     ok = false;
                     break;
+                }
+                // cur_a[sd][k]: side value sd of row trow + 8k of the quarter
+                float cur_a[NSIDE][4];
+#pragma unroll
+                for (int sd = 0; sd < NSIDE; ++sd) {
+                    const float4 v = lds_f4(side_a + sd * BM * 4);
+                    cur_a[sd][0] = v.x;
+                    cur_a[sd][1] = v.y;
+                    cur_a[sd][2] = v.z;
+                    cur_a[sd][3] = v.w;
                 }
                 tc_fence_after();
                 const uint32_t tbase = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
@@ -452,12 +435,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                     uint32_t r[16];
                     tmem_ld_16x128b_x4_pair(tbase + 16 * chunk, tbase + (16u << 16) + 16 * chunk, r);
                     tmem_wait_ld(r);
-                    const float4 sw = *reinterpret_cast<const float4 *>(sb + 16 * chunk + tq);
+                    const float4 sw = lds_f4(side_w + 16 * chunk * 4);
                     const float swv[4] = {sw.x, sw.y, sw.z, sw.w};
                     float4 zw4 = make_float4(0.f, 0.f, 0.f, 0.f), gw4 = zw4;
                     if (MODE == QUARTZ_ASYMMETRIC) {
-                        zw4 = *reinterpret_cast<const float4 *>(sb + kColsPerWarp + 16 * chunk + tq);
-                        gw4 = *reinterpret_cast<const float4 *>(sb + 2 * kColsPerWarp + 16 * chunk + tq);
+                        zw4 = lds_f4(side_w + (BN + 16 * chunk) * 4);
+                        gw4 = lds_f4(side_w + (2 * BN + 16 * chunk) * 4);
                     }
                     const float zwv[4] = {zw4.x, zw4.y, zw4.z, zw4.w};
                     const float gwv[4] = {gw4.x, gw4.y, gw4.z, gw4.w};
@@ -467,6 +450,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                         for (int i = 0; i < 4; ++i) {
                             float2 p = make_float2(__uint_as_float(r[8 * h + 2 * i]), __uint_as_float(r[8 * h + 2 * i + 1]));
                             if (DUMP && g == args.partials_group) {
+                                int mt, nt;
+                                tile_coords(tile, args, mt, nt);
                                 const int64_t m = static_cast<int64_t>(mt) * BM + quarter * 32 + 16 * h + trow;
                                 const int64_t n = static_cast<int64_t>(nt) * BN + slot * kColsPerWarp + 16 * chunk + tq + i;
                                 if (n < args.N) {
@@ -488,9 +473,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(acc_empty_bar(b));
+                if (lane == 0) {
+                    mbar_arrive(acc_empty_bar(b));
+                    mbar_arrive(side_empty_bar(ss));
+                }
             }
             if (!ok) break;
+            int mt, nt;
+            tile_coords(tile, args, mt, nt);
             // ---- store: 4 rows x 4 chunks of 4 consecutive columns per thread ----
 #pragma unroll
             for (int h = 0; h < 2; ++h)
@@ -563,7 +553,7 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const __half *__restrict
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
             const int m = m0 + ty * 4 + i;
-            const float s_a = args.a_side[static_cast<int64_t>(g) * args.m_pad + m];
+            const float s_a = args.a_side[static_cast<int64_t>(g) * args.m_pad + perm32(m)];
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
                 const int n = n0 + tx * 4 + j;
@@ -571,8 +561,8 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const __half *__restrict
                 float P = static_cast<float>(p[i][j]);
                 if (args.partials && g == args.partials_group) args.partials[(int64_t)m * args.N + n] = p[i][j];
                 if (MODE == QUARTZ_ASYMMETRIC) {
-                    const float za = args.a_side[a_plane + (int64_t)g * args.m_pad + m];
-                    const float ua = args.a_side[2 * a_plane + (int64_t)g * args.m_pad + m];
+                    const float za = args.a_side[a_plane + (int64_t)g * args.m_pad + perm32(m)];
+                    const float ua = args.a_side[2 * a_plane + (int64_t)g * args.m_pad + perm32(m)];
                     const float zw = args.w_side[w_plane + (int64_t)g * args.n_pad + n];
                     const float gw = args.w_side[2 * w_plane + (int64_t)g * args.n_pad + n];
                     P = __fmaf_rn(zw, ua, P);
