@@ -2,30 +2,33 @@
 //
 // Pipeline of one quartz_linear call:
 //   1. expand: the packed 4-bit codes and per-subgroup FLAGs of both operands
-//      are decoded to v = sgn(c)(|c| << FLAG) and written as fp16 (exact: every
-//      decoded value has at most 3 significant bits and |v| <= 112), together
-//      with the group scales (and zero-point side values) transposed to
-//      [G][rows] fp32 for contiguous per-group access.  This pass is
-//      HBM-bound and touches each operand element once, instead of once per
-//      output tile that reads it.
+//      are decoded to v = sgn(c)(|c| << FLAG) and written as FP8 E4M3 (exact:
+//      every decoded value is |c| <= 7 times a power of two up to 2^4, i.e.
+//      at most 3 significant bits and |v| <= 112, inside E4M3's 4-bit
+//      significand and 448 range), together with the group scales (and
+//      zero-point side values) transposed to [G][rows] fp32 for contiguous
+//      per-group access.  This pass is HBM-bound and touches each operand
+//      element once, instead of once per output tile that reads it.
 //   2. GEMM: a persistent warp-specialised tcgen05 kernel.  One TMA warp
 //      streams 128x64 A and 256x64 W tiles (one 64-wide quantization group
-//      per stage, 128-byte swizzle) into a 4-stage shared-memory ring; one
-//      thread issues kind::f16 MMAs into a fresh fp32 TMEM accumulator for
-//      every group (double-buffered, 2 x 256 columns), so each accumulator
-//      holds exactly P_g = sum_{k in g} v_a v_w; eight epilogue warps read
-//      P_g with tcgen05.ld and fold it into the register-resident output as
+//      per stage, 64-byte swizzle) into an 8-stage shared-memory ring and
+//      each group's scales into a ring of its own; one thread issues
+//      kind::f8f6f4 MMAs into a fresh fp32 TMEM accumulator for every group
+//      (double-buffered, 2 x 256 columns), so each accumulator holds exactly
+//      P_g = sum_{k in g} v_a v_w; sixteen epilogue warps read P_g with
+//      tcgen05.ld and fold it into the register-resident output as
 //      y += s_a * (s_w * P_g) with packed f32x2 arithmetic.
 //
 // Exactness of P_g: the products v_a * v_w are integers of magnitude at most
 // 112^2 = 12544 and every partial sum over a group is an integer of
 // magnitude at most 64 * 12544 < 2^20, all exactly representable in the fp32
 // accumulator, so the tensor-core sum equals the integer sum.  (sm_103a has
-// no integer tcgen05 MMA kind; this is why the integer GEMM runs on the f16
-// pipe.)
+// no integer tcgen05 MMA kind; this is why the integer GEMM runs on the
+// floating-point pipe.)
 #include <cuda.h>
 #include <cuda_fp16.h>
 #include <cuda_bf16.h>
+#include <cuda_fp8.h>
 
 #include "ptx.cuh"
 #include "quartz_internal.h"
@@ -53,7 +56,7 @@ __global__ void __launch_bounds__(256) expand_kernel(const uint32_t *__restrict_
                                                      const uint8_t *__restrict__ flags,
                                                      int64_t n_chunks, int64_t chunks_per_row,
                                                      int64_t n_chunks_pad, int permute,
-                                                     uint4 *__restrict__ op)
+                                                     uint2 *__restrict__ op)
 {
     const int64_t c = static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x;
     if (c >= n_chunks_pad) return;
@@ -63,21 +66,20 @@ __global__ void __launch_bounds__(256) expand_kernel(const uint32_t *__restrict_
         dst = perm16(r) * chunks_per_row + (c - r * chunks_per_row);
     }
     if (c >= n_chunks) {  // padding rows up to a multiple of 16
-        op[dst] = make_uint4(0, 0, 0, 0);
+        op[dst] = make_uint2(0, 0);
         return;
     }
     const uint32_t word = codes[c];
     const int flag = flags[(c * 8) / GS];
     const int mul = 1 << flag;
-    uint32_t o[4];
+    uint32_t o[2] = {0u, 0u};
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const int c0 = static_cast<int>(word << (28 - 8 * i)) >> 28;
-        const int c1 = static_cast<int>(word << (24 - 8 * i)) >> 28;
-        const __half2 h = __floats2half2_rn(static_cast<float>(c0 * mul), static_cast<float>(c1 * mul));
-        o[i] = *reinterpret_cast<const uint32_t *>(&h);
+    for (int i = 0; i < 8; ++i) {
+        const int ci = static_cast<int>(word << (28 - 4 * i)) >> 28;
+        const uint32_t byte = __nv_cvt_float_to_fp8(static_cast<float>(ci * mul), __NV_SATFINITE, __NV_E4M3);
+        o[i >> 2] |= byte << (8 * (i & 3));
     }
-    op[dst] = make_uint4(o[0], o[1], o[2], o[3]);
+    op[dst] = make_uint2(o[0], o[1]);
 }
 
 // Position of activation row r in its group's side-value row: inside every
@@ -118,9 +120,9 @@ __global__ void side_kernel(const __half *__restrict__ scales, const int8_t *__r
 constexpr int BM = 128;
 constexpr int BN = 256;
 constexpr int BK = kGroupQ;
-constexpr int kStages = 4;
-constexpr int kABytes = BM * BK * 2;
-constexpr int kBBytes = BN * BK * 2;
+constexpr int kStages = 8;
+constexpr int kABytes = BM * BK;      // E4M3 operands: one byte per element
+constexpr int kBBytes = BN * BK;
 constexpr int kStageBytes = kABytes + kBBytes;
 // Warpgroups 0-3 dequantise (16 warps: four per 32-lane TMEM quarter, 64
 // columns each); warpgroup 4 holds the TMA producer, the MMA issuer and two
@@ -327,12 +329,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
       } else if (warp == kMmaWarp) {
         // ------------------------------------------------------------------
-        // MMA issuer: 4 x (M=128, N=256, K=16) kind::f16 MMAs per group into
+        // MMA issuer: 2 x (M=128, N=256, K=32) kind::f8f6f4 MMAs per group into
         // a fresh accumulator (first MMA overwrites), then two commits: one
         // frees the operand stage, one hands P_g to the epilogue.
         // ------------------------------------------------------------------
         if (lane == 0) {
-            constexpr uint32_t idesc = idesc_f16_f32(BM, BN);
+            constexpr uint32_t idesc = idesc_e4m3_f32(BM, BN);
             int it = 0;
             bool ok = true;
             for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
@@ -353,10 +355,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const uint32_t sa = smem_base + L::kOperands + s * kStageBytes;
                     const uint32_t d = tmem_base + static_cast<uint32_t>(b * BN);
 #pragma unroll
-                    for (int kk = 0; kk < BK / 16; ++kk) {
-                        const uint64_t adesc = sdesc_k_major_sw128(sa + kk * 32);
-                        const uint64_t bdesc = sdesc_k_major_sw128(sa + kABytes + kk * 32);
-                        mma_f16_ss(d, adesc, bdesc, idesc, kk > 0 ? 1u : 0u);
+                    for (int kk = 0; kk < BK / 32; ++kk) {
+                        const uint64_t adesc = sdesc_k_major_sw64(sa + kk * 32);
+                        const uint64_t bdesc = sdesc_k_major_sw64(sa + kABytes + kk * 32);
+                        mma_f8_ss(d, adesc, bdesc, idesc, kk > 0 ? 1u : 0u);
                     }
                     mma_commit(empty_bar(s));
                     mma_commit(acc_full_bar(b));
@@ -525,8 +527,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 //    64x64 output tile per 256-thread block, 4x4 outputs per thread.
 // ---------------------------------------------------------------------------
 template <int MODE, int OUT>
-__global__ void __launch_bounds__(256) gemm_simt_kernel(const __half *__restrict__ a_op,
-                                                        const __half *__restrict__ w_op,
+__global__ void __launch_bounds__(256) gemm_simt_kernel(const __nv_fp8_e4m3 *__restrict__ a_op,
+                                                        const __nv_fp8_e4m3 *__restrict__ w_op,
                                                         const GemmArgs args, int K)
 {
     __shared__ int16_t sa[64][kGroupQ + 2];
@@ -540,8 +542,8 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const __half *__restrict
         for (int i = threadIdx.x; i < 64 * kGroupQ; i += 256) {
             const int r = i / kGroupQ, k = i % kGroupQ;
             const int64_t kk = static_cast<int64_t>(g) * kGroupQ + k;
-            sa[r][k] = (m0 + r < args.M) ? static_cast<int16_t>(__half2float(a_op[(int64_t)(m0 + r) * K + kk])) : 0;
-            sw[r][k] = (n0 + r < args.N) ? static_cast<int16_t>(__half2float(w_op[perm16(n0 + r) * K + kk])) : 0;
+            sa[r][k] = (m0 + r < args.M) ? static_cast<int16_t>(static_cast<float>(a_op[(int64_t)(m0 + r) * K + kk])) : 0;
+            sw[r][k] = (n0 + r < args.N) ? static_cast<int16_t>(static_cast<float>(w_op[perm16(n0 + r) * K + kk])) : 0;
         }
         __syncthreads();
         int p[4][4] = {};
@@ -616,18 +618,18 @@ EncodeTiledFn encode_tiled_fn()
     return fn;
 }
 
-// K-major fp16 operand [rows, K] read in boxes of [box_rows, 64] with the
-// 128-byte swizzle; out-of-range rows read as zero.
+// K-major E4M3 operand [rows, K] (one byte per element) read in boxes of
+// [box_rows, 64] with the 64-byte swizzle; out-of-range rows read as zero.
 bool make_operand_map(CUtensorMap *m, const void *base, int64_t rows, int64_t K, int box_rows)
 {
     EncodeTiledFn fn = encode_tiled_fn();
     if (!fn) return false;
     const cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(rows)};
-    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(K) * 2};
+    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(K)};
     const cuuint32_t box[2] = {static_cast<cuuint32_t>(BK), static_cast<cuuint32_t>(box_rows)};
     const cuuint32_t estr[2] = {1, 1};
-    return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void *>(base), dims, strides, box, estr,
-              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void *>(base), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B,
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -669,8 +671,8 @@ template <int MODE, int OUT>
 cudaError_t launch_simt(const LinearWorkspace &ws, const GemmArgs &args, int K, cudaStream_t s)
 {
     dim3 grid(static_cast<unsigned>((args.N + 63) / 64), static_cast<unsigned>((args.M + 63) / 64));
-    gemm_simt_kernel<MODE, OUT><<<grid, 256, 0, s>>>(static_cast<const __half *>(ws.a_op),
-                                                     static_cast<const __half *>(ws.w_op), args, K);
+    gemm_simt_kernel<MODE, OUT><<<grid, 256, 0, s>>>(static_cast<const __nv_fp8_e4m3 *>(ws.a_op),
+                                                     static_cast<const __nv_fp8_e4m3 *>(ws.w_op), args, K);
     return cudaGetLastError();
 }
 
@@ -714,8 +716,8 @@ size_t linear_workspace_bytes(int64_t M, int64_t N, int64_t K, int mode)
 {
     const int nside = mode == QUARTZ_ASYMMETRIC ? 3 : 1;
     const int64_t G = K / kGroupQ;
-    size_t b = align256(static_cast<size_t>(M) * K * 2);
-    b += align256(static_cast<size_t>(round_up(N, 16)) * K * 2);
+    size_t b = align256(static_cast<size_t>(M) * K);
+    b += align256(static_cast<size_t>(round_up(N, 16)) * K);
     b += align256(static_cast<size_t>(nside) * G * round_up(M > 0 ? M : 1, BM) * 4);
     b += align256(static_cast<size_t>(nside) * G * round_up(N, BN) * 4);
     return b;
@@ -731,9 +733,9 @@ void linear_workspace_carve(void *base, int64_t M, int64_t N, int64_t K, int mod
     ws->m_pad = round_up(M > 0 ? M : 1, BM);
     ws->n_pad = round_up(N, BN);
     ws->a_op = p;
-    p += align256(static_cast<size_t>(M) * K * 2);
+    p += align256(static_cast<size_t>(M) * K);
     ws->w_op = p;
-    p += align256(static_cast<size_t>(round_up(N, 16)) * K * 2);
+    p += align256(static_cast<size_t>(round_up(N, 16)) * K);
     ws->a_side = reinterpret_cast<float *>(p);
     p += align256(static_cast<size_t>(nside) * G * ws->m_pad * 4);
     ws->w_side = reinterpret_cast<float *>(p);
@@ -749,7 +751,7 @@ cudaError_t launch_expand(const quartz_encoded_t *e, void *op, float *side, int6
     if (n_chunks_pad > 0) {
         const unsigned blocks = static_cast<unsigned>((n_chunks_pad + 255) / 256);
         const uint32_t *codes = reinterpret_cast<const uint32_t *>(e->codes);
-        uint4 *o = static_cast<uint4 *>(op);
+        uint2 *o = static_cast<uint2 *>(op);
         const int perm = is_a ? 0 : 1;
         switch (e->p.group_s) {
             case 8: expand_kernel<8><<<blocks, 256, 0, s>>>(codes, e->flags, n_chunks, cpr, n_chunks_pad, perm, o); break;

@@ -173,16 +173,36 @@ __device__ __forceinline__ void regs_decrease()
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
-// D[tmem] (+)= A[smem] * B[smem]^T, kind::f16 (fp16/bf16 inputs, fp32 accumulate).
-__device__ __forceinline__ void mma_f16_ss(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
-                                           uint32_t idesc, uint32_t accumulate)
+// Shared-memory matrix descriptor for a K-major tile with the 64-byte swizzle:
+// 64-byte rows, 8-row swizzle atoms 512 bytes apart (stride byte offset).
+__device__ __forceinline__ uint64_t sdesc_k_major_sw64(uint32_t addr)
+{
+    uint64_t d = 0;
+    d |= (uint64_t)((addr & 0x3FFFFu) >> 4);
+    d |= (uint64_t)1u << 16;
+    d |= (uint64_t)(512u >> 4) << 32;
+    d |= (uint64_t)1u << 46;
+    d |= (uint64_t)4u << 61;                          // swizzle: 64B
+    return d;
+}
+
+// D (TMEM, fp32) = A * B (+ D if `accumulate`), A and B FP8 from shared memory.
+__device__ __forceinline__ void mma_f8_ss(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                          uint32_t idesc, uint32_t accumulate)
 {
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
         "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
         "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
         : "memory");
+}
+
+// Instruction descriptor of kind::f8f6f4: E4M3 A and B (format 0, K-major),
+// fp32 D, shape M x N.
+__host__ __device__ constexpr uint32_t idesc_e4m3_f32(uint32_t M, uint32_t N)
+{
+    return (1u << 4) | (0u << 7) | (0u << 10) | ((N >> 3) << 17) | ((M >> 4) << 24);
 }
 
 // Arrive once on `bar` when every tcgen05 op issued so far by this thread is done.
@@ -191,46 +211,6 @@ __device__ __forceinline__ void mma_commit(uint32_t bar)
     asm volatile(
         "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
         : "memory");
-}
-
-// 32 lanes x 32 columns of 32-bit TMEM cells; thread t gets lane (base + t).
-__device__ __forceinline__ void tmem_ld_32x32b_x32(uint32_t taddr, uint32_t (&r)[32])
-{
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
-          "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
-          "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
-          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
-          "=r"(r[31])
-        : "r"(taddr)
-        : "memory");
-}
-
-// 32 lanes x 16 columns of 32-bit TMEM cells; thread t gets lane (base + t).
-__device__ __forceinline__ void tmem_ld_32x32b_x16(uint32_t taddr, uint32_t (&r)[16])
-{
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
-          "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-        : "r"(taddr)
-        : "memory");
-}
-
-__device__ __forceinline__ void tmem_wait_ld(uint32_t (&r)[16])
-{
-    asm volatile("tcgen05.wait::ld.sync.aligned;"
-                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]),
-                   "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]),
-                   "+r"(r[13]), "+r"(r[14]), "+r"(r[15])
-                 :
-                 : "memory");
 }
 
 // Two loads of 16 lanes x (4 x 128 bits) of TMEM, at t0 and t1.  For every
@@ -251,41 +231,14 @@ __device__ __forceinline__ void tmem_ld_16x128b_x4_pair(uint32_t t0, uint32_t t1
 
 // Wait for this thread's outstanding tcgen05.ld; the registers are passed as
 // read-write operands so that no use of them is scheduled before the wait.
-__device__ __forceinline__ void tmem_wait_ld(uint32_t (&r)[32])
+__device__ __forceinline__ void tmem_wait_ld(uint32_t (&r)[16])
 {
     asm volatile("tcgen05.wait::ld.sync.aligned;"
                  : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]),
                    "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]),
-                   "+r"(r[13]), "+r"(r[14]), "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]),
-                   "+r"(r[19]), "+r"(r[20]), "+r"(r[21]), "+r"(r[22]), "+r"(r[23]), "+r"(r[24]),
-                   "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]), "+r"(r[29]), "+r"(r[30]),
-                   "+r"(r[31])
+                   "+r"(r[13]), "+r"(r[14]), "+r"(r[15])
                  :
                  : "memory");
-}
-
-// Shared-memory matrix descriptor (tcgen05 format) for a K-major operand tile
-// stored with the 128-byte swizzle: rows of 128 bytes, 8-row atoms 1024 bytes
-// apart.  `addr` is the shared address of the (sub-)tile start.
-__device__ __forceinline__ uint64_t sdesc_k_major_sw128(uint32_t addr)
-{
-    uint64_t d = 0;
-    d |= (uint64_t)((addr & 0x3FFFFu) >> 4);        // start address >> 4      bits  0-13
-    d |= (uint64_t)1u << 16;                          // leading byte offset     bits 16-29 (unused)
-    d |= (uint64_t)(1024u >> 4) << 32;                // stride byte offset      bits 32-45
-    d |= (uint64_t)1u << 46;                          // descriptor version      bits 46-47
-    d |= (uint64_t)2u << 61;                          // swizzle: 128B           bits 61-63
-    return d;
-}
-
-// Instruction descriptor of kind::f16: fp16 A and B (K-major), fp32 D, shape M x N.
-__host__ __device__ constexpr uint32_t idesc_f16_f32(uint32_t M, uint32_t N)
-{
-    return (1u << 4)             // D format: f32
-           | (0u << 7)           // A format: f16
-           | (0u << 10)          // B format: f16
-           | ((N >> 3) << 17)    // N / 8
-           | ((M >> 4) << 24);   // M / 16
 }
 
 }  // namespace quartz

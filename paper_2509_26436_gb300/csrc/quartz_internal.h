@@ -27,8 +27,8 @@ cudaError_t launch_dequantize(const quartz_encoded_t *e, void *y, cudaStream_t s
 
 // Linear-layer workspace and launches (linear.cu).
 struct LinearWorkspace {
-    void *a_op;      // fp16 [M, K]  decoded activations, tensor-core input
-    void *w_op;      // fp16 [round_up(N, 16), K]  decoded weights, rows transposed 4x4 inside 16-row blocks
+    void *a_op;      // E4M3 [M, K]  decoded activations
+    void *w_op;      // E4M3 [round_up(N, 16), K]  decoded weights, rows transposed 4x4 inside 16-row blocks
     float *a_side;   // fp32 [nside][G][Mpad]  scale (and z, gsum when asymmetric)
     float *w_side;   // fp32 [nside][G][Npad]
     int64_t m_pad, n_pad;

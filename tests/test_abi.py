@@ -105,7 +105,8 @@ def test_linear_validation(lib):
     assert call(a, w, ws=None) == N.QUARTZ_ERR_WORKSPACE
     assert call(a, w, y=None) == N.QUARTZ_ERR_INVALID_ARG
     p = N.QuartzParams(64, 16, 0)
-    assert lib.quartz_linear_workspace_size(16, 24, 128, C.byref(p)) > 16 * 128 * 2 + 24 * 128 * 2
+    # at least both operands expanded to one byte per element
+    assert lib.quartz_linear_workspace_size(16, 24, 128, C.byref(p)) > 16 * 128 + 24 * 128
     assert lib.quartz_linear_workspace_size(16, 20, 128, C.byref(p)) == 0
     assert lib.quartz_selftest_timeout(10, None) == N.QUARTZ_ERR_INVALID_ARG
 

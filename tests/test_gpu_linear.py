@@ -180,3 +180,37 @@ def test_gemm_events_bracket_the_gemm_kernel(Q):
     t_gemm, t_call = g0.elapsed_time(g1), c0.elapsed_time(c1)
     assert 0 < t_gemm <= t_call
     assert Q.device_status() == 0
+
+
+def _lzs_extreme(rows, K, seed):
+    """Rows whose 16-wide subgroups alternate between the two ends of the LZS
+    range: even subgroups hold +-1.0 (the group maximum, q = +-127, FLAG 4,
+    decoded +-112) and odd subgroups hold q/127 with |q| <= 7 (FLAG 0,
+    decoded q).  One group partial then mixes products of 12544 with
+    products of 1, so any loss of low-order bits in the tensor-core sums
+    shows up as a wrong integer."""
+    rng = np.random.default_rng(seed)
+    x = np.where(rng.random((rows, K)) < 0.5, -1.0, 1.0)
+    small = rng.integers(-7, 8, size=(rows, K)) / 127.0
+    odd = (np.arange(K) // 16) % 2 == 1
+    x[:, odd] = small[:, odd]
+    return x.astype(np.float16)
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_group_partials_lzs_extremes_bit_exact(Q, seed):
+    M, N, K = 256, 272, 512
+    xa, xw = _lzs_extreme(M, K, 100 + seed), _lzs_extreme(N, K, 200 + seed)
+    ea, ew = O.encode(xa, 64, 16), O.encode(xw, 64, 16)
+    va, vw = O.decode_values(ea), O.decode_values(ew)
+    assert np.abs(va).max() == 112 and np.abs(vw).max() == 112
+    a = Q.quantize(torch.from_numpy(xa).cuda(), group_s=16)
+    w = Q.encode_weights(torch.from_numpy(xw).cuda(), group_s=16)
+    for g in range(K // 64):
+        y, part = Q.linear(a, w, out_dtype=torch.float32, partials_group=g)
+        assert Q.device_status() == 0
+        ref = O.group_partials(va[:, g * 64:(g + 1) * 64], vw[:, g * 64:(g + 1) * 64], 64)[0]
+        assert (np.abs(ref) > 2 ** 17).any() and (ref % 2 == 1).any()
+        assert np.array_equal(part.cpu().numpy().astype(np.int64), ref), f"group {g}"
+    ref, rabs = O.linear(ea, ew, with_abs=True)
+    _tol_check(y.cpu().numpy(), ref, rabs, K // 64, "float32")
