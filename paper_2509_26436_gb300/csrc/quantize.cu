@@ -1,13 +1,21 @@
 // QuaRTZ encoder (Section 3, Eq. 1 then Eq. 2) and dequantiser for sm_103a.
 //
 // The encoder is HBM-bound: per element it reads 2 bytes (fp16) and writes
-// half a byte of code, 1/G_s bytes of FLAG and 2/64 bytes of scale.  Each
-// thread owns one 16-byte chunk (8 consecutive elements along K) and eight
-// consecutive lanes own one 64-element quantization group, so a warp reads
-// 512 contiguous bytes, the group reductions are 3 xor-shuffles and the
-// code words of a warp form one contiguous 128-byte store.  Several chunks
-// per thread are loaded before any is processed to keep enough bytes in
-// flight to saturate HBM.
+// half a byte of code, 1/G_s bytes of FLAG and 2/64 bytes of scale.
+//
+// Symmetric mode (the default) keeps the per-element instruction count low
+// enough for HBM to be the limit: each thread owns 16 consecutive elements
+// (two 16-byte loads; four lanes form one 64-element group, so the group
+// maximum takes two xor-shuffles), the scale and FLAG come from the group and
+// subgroup maxima (max |q| = min(rne(max|x| * r), 127), since rounding and the
+// cap are monotonic), and the codes are formed four elements per 32-bit word:
+// rne(|x| r) is produced by the 1.5 * 2^23 rounding addend, which leaves the
+// integer in the low byte of the float, the bytes are gathered with byte
+// permutes, shifted right by FLAG in one 32-bit shift, and the sign applied
+// per byte in 4-bit two's complement.
+//
+// Asymmetric mode uses one thread per 8-element chunk (eight lanes per group)
+// with the same arithmetic written per element.
 #include <cuda_fp16.h>
 
 #include "quartz_internal.h"
@@ -26,6 +34,162 @@ __device__ __forceinline__ uint4 ldg_stream(const uint4 *p)
                  : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
                  : "l"(p));
     return v;
+}
+
+// ---------------------------------------------------------------------------
+// Symmetric encoder: 16 elements per thread
+// ---------------------------------------------------------------------------
+constexpr int kUnitsPerThread = 2;
+// Adding 1.5 * 2^23 to a float of magnitude below 2^22 rounds it to an
+// integer (round-to-nearest-even, the rounding of the addition) and leaves
+// that integer in the low mantissa bits: for 0 <= n < 256 the low byte of the
+// sum's bit pattern is n.
+constexpr float kRoundAddend = 12582912.0f;
+
+// a * b on float pairs, rounded to nearest even (PTX mul.rn.f32x2).
+__device__ __forceinline__ float2 mul2_rn(float2 a, float2 b)
+{
+    float2 d;
+    asm("{\n\t.reg .b64 a, b, d;\n\t"
+        "mov.b64 a, {%2, %3};\n\t"
+        "mov.b64 b, {%4, %5};\n\t"
+        "mul.rn.f32x2 d, a, b;\n\t"
+        "mov.b64 {%0, %1}, d;\n\t}"
+        : "=f"(d.x), "=f"(d.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return d;
+}
+
+__device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel)
+{
+    uint32_t d;
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(sel));
+    return d;
+}
+
+// Per byte: m (0..7) with the sign s (0x00 or 0xFF) applied in 4-bit two's
+// complement: m for s = 0, (16 - m) & 15 for s = 0xFF.
+__device__ __forceinline__ uint32_t signed_nibbles(uint32_t m, uint32_t s)
+{
+    return ((m ^ (s & 0x0F0F0F0Fu)) + (s & 0x01010101u)) & 0x0F0F0F0Fu;
+}
+
+// Eq. 2 codes of 8 elements given as four fp16 pairs `w` (the raw words) and
+// their sign-cleared copies `a`: q = rne(x r) (capped at +-127 when CAP), c =
+// sgn(q) (|q| >> flag), packed as 8 nibbles, element k in bits 4k..4k+3.
+template <bool CAP>
+__device__ __forceinline__ uint32_t lzs_word8(const uint32_t *w, const uint32_t *a, float r, int flag)
+{
+    uint32_t u[4][2];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const float2 f = __half22float2(*reinterpret_cast<const __half2 *>(&a[i]));
+        float2 t = mul2_rn(f, make_float2(r, r));
+        if (CAP) {
+            t.x = fminf(t.x, 127.0f);
+            t.y = fminf(t.y, 127.0f);
+        }
+        // Two scalar additions: a paired multiply followed by a paired add
+        // was observed to be fused into one multiply-add (parity tests
+        // failed on exact ties of x r), which rounds the unrounded product.
+        const float2 m = make_float2(__fadd_rn(t.x, kRoundAddend), __fadd_rn(t.y, kRoundAddend));
+        u[i][0] = __float_as_uint(m.x);
+        u[i][1] = __float_as_uint(m.y);
+    }
+    // byte k of ev / od: |q| of element 2k / 2k + 1
+    const uint32_t ev = prmt(prmt(u[0][0], u[1][0], 0x0040u), prmt(u[2][0], u[3][0], 0x0040u), 0x5410u);
+    const uint32_t od = prmt(prmt(u[0][1], u[1][1], 0x0040u), prmt(u[2][1], u[3][1], 0x0040u), 0x5410u);
+    // byte k of sev / sod: 0xFF when element 2k / 2k + 1 is negative (a
+    // selector nibble 8 + b replicates the sign bit of byte b)
+    const uint32_t sev = prmt(prmt(w[0], w[1], 0x00D9u), prmt(w[2], w[3], 0x00D9u), 0x5410u);
+    const uint32_t sod = prmt(prmt(w[0], w[1], 0x00FBu), prmt(w[2], w[3], 0x00FBu), 0x5410u);
+    const uint32_t keep = 0x01010101u * (0xFFu >> flag);
+    const uint32_t cev = signed_nibbles((ev >> flag) & keep, sev);
+    const uint32_t cod = signed_nibbles((od >> flag) & keep, sod);
+    return cev | (cod << 4);
+}
+
+__device__ __forceinline__ int lzs_flag_of(float amax_sub, float r)
+{
+    const int qmax = min(__float2int_rn(__fmul_rn(amax_sub, r)), 127);
+    return max(29 - __clz(qmax), 0);
+}
+
+template <int GS>
+__device__ __forceinline__ void encode_unit_sym(const uint4 lo, const uint4 hi, int64_t unit, bool valid,
+                                                int lane, uint2 *__restrict__ codes,
+                                                uint8_t *__restrict__ flags, __half *__restrict__ scales)
+{
+    const uint32_t w[8] = {lo.x, lo.y, lo.z, lo.w, hi.x, hi.y, hi.z, hi.w};
+    uint32_t a[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) a[i] = w[i] & 0x7FFF7FFFu;
+    // --- maxima of |x|: each 8-element half, the unit, the group ----------
+    __half2 m0 = __hmax2(__hmax2(*reinterpret_cast<const __half2 *>(&a[0]), *reinterpret_cast<const __half2 *>(&a[1])),
+                         __hmax2(*reinterpret_cast<const __half2 *>(&a[2]), *reinterpret_cast<const __half2 *>(&a[3])));
+    __half2 m1 = __hmax2(__hmax2(*reinterpret_cast<const __half2 *>(&a[4]), *reinterpret_cast<const __half2 *>(&a[5])),
+                         __hmax2(*reinterpret_cast<const __half2 *>(&a[6]), *reinterpret_cast<const __half2 *>(&a[7])));
+    const float2 f0 = __half22float2(m0), f1 = __half22float2(m1);
+    const float sub0 = fmaxf(f0.x, f0.y), sub1 = fmaxf(f1.x, f1.y);
+    const float unit_max = fmaxf(sub0, sub1);
+    const float pair_max = fmaxf(unit_max, __shfl_xor_sync(0xffffffffu, unit_max, 1));
+    const float amax = fmaxf(pair_max, __shfl_xor_sync(0xffffffffu, pair_max, 2));
+
+    // --- Eq. 1: scale and reciprocal (as the per-element path) ------------
+    const __half s16 = __float2half_rn(__fdiv_rn(amax, 127.0f));
+    const float s = __half2float(s16);
+    const float r = (s > 0.f) ? __frcp_rn(s) : 0.f;
+
+    // --- Eq. 2: FLAG of each subgroup from its maximum --------------------
+    int flag0, flag1;
+    if (GS == 8) {
+        flag0 = lzs_flag_of(sub0, r);
+        flag1 = lzs_flag_of(sub1, r);
+    } else {
+        const float m = GS == 16 ? unit_max : GS == 32 ? pair_max : amax;
+        flag0 = flag1 = lzs_flag_of(m, r);
+    }
+    uint32_t c0, c1;
+    if (__float2int_rn(__fmul_rn(amax, r)) > 127) {  // only when the fp16 scale rounded far down
+        c0 = lzs_word8<true>(w, a, r, flag0);
+        c1 = lzs_word8<true>(w + 4, a + 4, r, flag1);
+    } else {
+        c0 = lzs_word8<false>(w, a, r, flag0);
+        c1 = lzs_word8<false>(w + 4, a + 4, r, flag1);
+    }
+    if (!valid) return;
+    codes[unit] = make_uint2(c0, c1);
+    if (GS == 8) {
+        reinterpret_cast<uint16_t *>(flags)[unit] = static_cast<uint16_t>(flag0 | (flag1 << 8));
+    } else if (GS == 16) {
+        flags[unit] = static_cast<uint8_t>(flag0);
+    } else if ((lane & (GS / 16 - 1)) == 0) {
+        flags[unit / (GS / 16)] = static_cast<uint8_t>(flag0);
+    }
+    if ((lane & 3) == 0) scales[unit >> 2] = s16;
+}
+
+template <int GS>
+__global__ void __launch_bounds__(kThreads) quantize_sym_kernel(const uint4 *__restrict__ x, int64_t n_units,
+                                                                uint2 *__restrict__ codes,
+                                                                uint8_t *__restrict__ flags,
+                                                                __half *__restrict__ scales)
+{
+    const int lane = threadIdx.x & 31;
+    const int64_t base = static_cast<int64_t>(blockIdx.x) * (kThreads * kUnitsPerThread) + threadIdx.x;
+    uint4 raw[kUnitsPerThread][2];
+#pragma unroll
+    for (int j = 0; j < kUnitsPerThread; ++j) {
+        const int64_t u = base + j * kThreads;
+        const bool in = u < n_units;
+        raw[j][0] = in ? ldg_stream(x + 2 * u) : make_uint4(0, 0, 0, 0);
+        raw[j][1] = in ? ldg_stream(x + 2 * u + 1) : make_uint4(0, 0, 0, 0);
+    }
+#pragma unroll
+    for (int j = 0; j < kUnitsPerThread; ++j) {
+        const int64_t u = base + j * kThreads;
+        encode_unit_sym<GS>(raw[j][0], raw[j][1], u, u < n_units, lane, codes, flags, scales);
+    }
 }
 
 __device__ __forceinline__ void unpack8(const uint4 &raw, float (&x)[8])
@@ -181,13 +345,23 @@ __global__ void __launch_bounds__(kThreads) dequantize_kernel(
 template <int GS, int MODE>
 cudaError_t launch_q(const void *x, const quartz_encoded_t *e, cudaStream_t s)
 {
-    const int64_t n_chunks = e->rows * e->K / 8;
-    const int64_t per_block = kThreads * kChunksPerThread;
-    const int64_t blocks = (n_chunks + per_block - 1) / per_block;
-    quantize_kernel<GS, MODE><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(
-        static_cast<const uint4 *>(x), n_chunks, reinterpret_cast<uint32_t *>(e->codes), e->flags,
-        reinterpret_cast<__half *>(e->scales), e->zeros, e->gsum);
-    return cudaGetLastError();
+    if constexpr (MODE == QUARTZ_SYMMETRIC) {
+        const int64_t n_units = e->rows * e->K / 16;
+        const int64_t per_block = kThreads * kUnitsPerThread;
+        const int64_t blocks = (n_units + per_block - 1) / per_block;
+        quantize_sym_kernel<GS><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(
+            static_cast<const uint4 *>(x), n_units, reinterpret_cast<uint2 *>(e->codes), e->flags,
+            reinterpret_cast<__half *>(e->scales));
+        return cudaGetLastError();
+    } else {
+        const int64_t n_chunks = e->rows * e->K / 8;
+        const int64_t per_block = kThreads * kChunksPerThread;
+        const int64_t blocks = (n_chunks + per_block - 1) / per_block;
+        quantize_kernel<GS, MODE><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(
+            static_cast<const uint4 *>(x), n_chunks, reinterpret_cast<uint32_t *>(e->codes), e->flags,
+            reinterpret_cast<__half *>(e->scales), e->zeros, e->gsum);
+        return cudaGetLastError();
+    }
 }
 
 template <int MODE>

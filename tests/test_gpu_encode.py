@@ -70,8 +70,9 @@ def test_encode_all_int8_codes(Q, gs):
 
 
 def test_encode_edge_values(Q):
-    """All-zero groups, scale underflow, subnormal scales, fp16 extremes,
-    exact ties, all-equal and one-sided groups."""
+    """All-zero groups, scale underflow, subnormal scales (including ones
+    rounded so far down that |x| r exceeds 127), fp16 extremes, exact ties,
+    all-equal and one-sided groups."""
     rows = []
     rows.append(np.zeros(256))
     rows.append(np.full(256, 1e-7))
@@ -80,6 +81,11 @@ def test_encode_edge_values(Q):
                                 np.linspace(-65504, 65504, 128)]))
     t = np.zeros(256)
     t[:7] = np.array([127, 2.5, 3.5, -2.5, -0.5, 0.5, 1.5]) * 2.0 ** -10
+    rows.append(t)
+    t = np.zeros(256)  # subnormal scales rounded far down: |x| r exceeds 127 and is clamped
+    t[:64] = np.linspace(-189, 189, 64).round() * 2.0 ** -24
+    t[64:128] = np.arange(64) * 3 * 2.0 ** -24
+    t[128:192] = (np.arange(64) - 32) * 5 * 2.0 ** -24
     rows.append(t)
     rows.append(np.full(256, 0.5))
     rows.append(np.abs(np.random.default_rng(4).laplace(0, 1, 256)) + 1)
