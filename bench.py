@@ -48,14 +48,24 @@ def parse():
     return p.parse_args()
 
 
+FALLBACK_SM_MHZ = 2070.0
+# The GEMM's tensor-core work is FP8 E4M3 (kind::f8f6f4): its peak is the
+# measured bf16 peak times the nominal dense FP8 : BF16 ratio (4.5 : 2.25).
+FP8_OVER_BF16 = 2.0
+# FP32 pipe: 128 lanes per SM, one multiply or fused multiply-add per lane per
+# cycle (a paired f32x2 instruction occupies two lanes' worth).
+FP32_LANES_PER_SM = 128
+
+
 def peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
         with open(path) as f:
             d = json.load(f)
-        return float(d["hbm_gbs"]), float(d["bf16_tflops"]), "measured"
+        return (float(d["hbm_gbs"]), float(d["bf16_tflops"]), float(d.get("sm_max_mhz", FALLBACK_SM_MHZ)),
+                "measured")
     except (OSError, KeyError, ValueError):
-        return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS, "fallback"
+        return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS, FALLBACK_SM_MHZ, "fallback"
 
 
 def gemm_traffic():
@@ -236,7 +246,10 @@ def run_ours(args):
     if world > 1:
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=dev)
-    hbm_peak, tc_peak, peak_src = peaks()
+    hbm_peak, bf16_peak, sm_mhz, peak_src = peaks()
+    n_sm = torch.cuda.get_device_properties(dev).multi_processor_count
+    fp8_peak = bf16_peak * FP8_OVER_BF16                              # TFLOP/s
+    alu_peak = n_sm * FP32_LANES_PER_SM * sm_mhz * 1e6 / 1e12         # T fp32-pipe lane ops/s
     layers = select_layers(inputs.CONFIG4, args.layers)
 
     # ---- inputs (seeded, host) -> pinned host + device ---------------------
@@ -311,7 +324,14 @@ def run_ours(args):
                for i in range(nl)]
     quant_ms = [statistics.mean(r["q"][i][0].elapsed_time(r["q"][i][1]) for r in recs)
                 for i in range(nl)]
-    gemm_tflops = sum(l.ops for l in layers) / (sum(gemm_ms) / 1e3) / 1e12
+    t_gemm = sum(gemm_ms) / 1e3
+    gemm_tflops = sum(l.ops for l in layers) / t_gemm / 1e12
+    # dequant epilogue: one fp32 multiply and one fused multiply-add per
+    # output element and 64-wide group (y += s_a * (s_w * P_g))
+    epi_ops = sum(2 * l.M * l.N * (l.K // GROUP_Q) for l in layers)
+    gemm_alu = epi_ops / t_gemm / 1e12
+    t_floor_tensor = sum(l.ops for l in layers) / (fp8_peak * 1e12)
+    t_floor_alu = epi_ops / (alu_peak * 1e12)
     elems = sum(l.M * l.K for l in layers)
     enc_gbs = elems * encode_bytes_per_elem() / (sum(quant_ms) / 1e3) / 1e9
     launches_per_step = nl * (1 + 5)   # quantize; expand A, side A, expand W, side W, GEMM
@@ -368,11 +388,20 @@ def run_ours(args):
     out = {
         "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": t_step * 1e3, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "f16", "data": "synthetic",
+        "scaling": "weak", "vs_baseline": None, "dtype": "e4m3/f32", "data": "synthetic",
         "config": layer_config(layers),
-        "roofline": {"bound": "tensor", "achieved": gemm_tflops, "peak": tc_peak,
-                     "unit": "TFLOP/s", "frac": gemm_tflops / tc_peak, "traffic": gemm_traffic(),
-                     "kernel": "gemm_tcgen05_kernel", "peak_source": f"{peak_src} bf16 burst",
+        "roofline": {"bound": "alu" if t_floor_alu >= t_floor_tensor else "tensor",
+                     "achieved": gemm_alu, "peak": alu_peak, "unit": "Top/s",
+                     "frac": gemm_alu / alu_peak, "traffic": gemm_traffic(),
+                     "kernel": "gemm_tcgen05_kernel",
+                     "peak_source": f"derived: {n_sm} SMs x {FP32_LANES_PER_SM} fp32 lanes x "
+                                    f"{sm_mhz:.0f} MHz ({peak_src} max SM clock)",
+                     "work": "2 fp32 ops (multiply + fused multiply-add) per output per 64-wide group",
+                     "tensor": {"achieved": gemm_tflops, "unit": "TFLOP/s", "peak": fp8_peak,
+                                "frac": gemm_tflops / fp8_peak,
+                                "peak_source": f"{peak_src} bf16 burst {bf16_peak} x {FP8_OVER_BF16} "
+                                               "(nominal FP8 : BF16)"},
+                     "floors_ms": {"alu": t_floor_alu * 1e3, "tensor": t_floor_tensor * 1e3},
                      "per_layer_ms": gemm_ms},
         "encode": {"kernel": "quantize_kernel", "gbs": enc_gbs, "peak_gbs": hbm_peak,
                    "frac": enc_gbs / hbm_peak, "bytes_per_elem": encode_bytes_per_elem(),
