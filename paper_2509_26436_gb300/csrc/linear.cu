@@ -206,6 +206,24 @@ __device__ __forceinline__ void store_quad(void *y, int64_t off, float4 v)
     }
 }
 
+// One 16-column chunk of the epilogue: two 16x128b.x4 TMEM loads (lanes +0
+// and +16), then acc[h][i] += s_a[h] * (s_w[i] * P) on (row, row + 8) pairs,
+// all on explicit 64-bit register pairs.
+__device__ __forceinline__ void epi_chunk_sym(uint32_t t0, uint32_t t1, float4 sw, uint64_t sa0, uint64_t sa1,
+                                              uint64_t (&acc)[8])
+{
+    asm volatile("{\n\t.reg .b32 p<16>;\n\t.reg .b64 q<8>, t<8>, s<4>;\n\ttcgen05.ld.sync.aligned.16x128b.x4.b32 {p0,p1,p2,p3,p4,p5,p6,p7}, [%8];\n\ttcgen05.ld.sync.aligned.16x128b.x4.b32 {p8,p9,p10,p11,p12,p13,p14,p15}, [%9];\n\ttcgen05.wait::ld.sync.aligned;\n\tmov.b64 q0, {p0, p1};\n\tmov.b64 q1, {p2, p3};\n\tmov.b64 q2, {p4, p5};\n\tmov.b64 q3, {p6, p7};\n\tmov.b64 q4, {p8, p9};\n\tmov.b64 q5, {p10, p11};\n\tmov.b64 q6, {p12, p13};\n\tmov.b64 q7, {p14, p15};\n\tmov.b64 s0, {%10, %10};\n\tmov.b64 s1, {%11, %11};\n\tmov.b64 s2, {%12, %12};\n\tmov.b64 s3, {%13, %13};\n\tmul.rn.f32x2 t0, q0, s0;\n\tmul.rn.f32x2 t1, q1, s1;\n\tmul.rn.f32x2 t2, q2, s2;\n\tmul.rn.f32x2 t3, q3, s3;\n\tmul.rn.f32x2 t4, q4, s0;\n\tmul.rn.f32x2 t5, q5, s1;\n\tmul.rn.f32x2 t6, q6, s2;\n\tmul.rn.f32x2 t7, q7, s3;\n\tfma.rn.f32x2 %0, t0, %14, %0;\n\tfma.rn.f32x2 %1, t1, %14, %1;\n\tfma.rn.f32x2 %2, t2, %14, %2;\n\tfma.rn.f32x2 %3, t3, %14, %3;\n\tfma.rn.f32x2 %4, t4, %15, %4;\n\tfma.rn.f32x2 %5, t5, %15, %5;\n\tfma.rn.f32x2 %6, t6, %15, %6;\n\tfma.rn.f32x2 %7, t7, %15, %7;\n\t}"
+                 : "+l"(acc[0]), "+l"(acc[1]), "+l"(acc[2]), "+l"(acc[3]), "+l"(acc[4]), "+l"(acc[5]),
+                   "+l"(acc[6]), "+l"(acc[7])
+                 : "r"(t0), "r"(t1), "f"(sw.x), "f"(sw.y), "f"(sw.z), "f"(sw.w), "l"(sa0), "l"(sa1)
+                 : "memory");
+}
+
+__device__ __forceinline__ void lds_b64x2(uint32_t addr, uint64_t &a, uint64_t &b)
+{
+    asm volatile("ld.shared.v2.b64 {%0, %1}, [%2];" : "=l"(a), "=l"(b) : "r"(addr) : "memory");
+}
+
 template <int MODE, int OUT, bool DUMP>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tmap_a,
@@ -395,122 +413,203 @@ __global__ void __launch_bounds__(kThreads, 1)
 
         // acc[h][j]: output column 16*(j/4) + tq + j%4 of this warp's slice,
         // rows trow + 16h (.x) and trow + 16h + 8 (.y)
-        float2 acc[2][16];
-        int it = 0;
-        bool ok = true;
-        for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
+        if constexpr (MODE == QUARTZ_SYMMETRIC && !DUMP) {
+            // Symmetric fast path: each 16-column chunk (TMEM loads, wait and
+            // the scale arithmetic) is one PTX block on explicit 64-bit pairs.
+            // acc64[c][4h + i]: output column 16c + tq + i, rows trow + 16h (low) and + 8 (high)
+            uint64_t acc64[4][8];
+            int it = 0;
+            bool ok = true;
+            for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
 #pragma unroll
-            for (int h = 0; h < 2; ++h)
+                for (int c = 0; c < 4; ++c)
 #pragma unroll
-                for (int j = 0; j < 16; ++j) acc[h][j] = make_float2(0.f, 0.f);
-            for (int g = 0; g < G; ++g, ++it) {
-                const int b = it & 1;
-                const int ss = it % S;
-                if (!mbar_wait_bounded(side_full_bar(ss), (it / S) & 1, abort_flag, args.dev_err,
-                                       kWaitLimitNs)) {
-                    ok = false;
-                    break;
-                }
-                const uint32_t side_a = smem_base + L::kSide + ss * L::kSideSlotBytes + (quarter * 32 + 4 * trow) * 4;
-                const uint32_t side_w = smem_base + L::kSide + ss * L::kSideSlotBytes + L::kSideABytes +
-                                        (slot * kColsPerWarp + tq) * 4;
-                if (!mbar_wait_bounded(acc_full_bar(b), (it >> 1) & 1, abort_flag, args.dev_err,
-                                       kWaitLimitNs)) {
-                    ok = false;
-                    break;
-                }
-                // cur_a[sd][k]: side value sd of row trow + 8k of the quarter
-                float cur_a[NSIDE][4];
-#pragma unroll
-                for (int sd = 0; sd < NSIDE; ++sd) {
-                    const float4 v = lds_f4(side_a + sd * BM * 4);
-                    cur_a[sd][0] = v.x;
-                    cur_a[sd][1] = v.y;
-                    cur_a[sd][2] = v.z;
-                    cur_a[sd][3] = v.w;
-                }
-                tc_fence_after();
-                const uint32_t tbase = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
-                                       static_cast<uint32_t>(b * BN + slot * kColsPerWarp);
-#pragma unroll
-                for (int chunk = 0; chunk < 4; ++chunk) {    // 16-column chunks of the slice
-                    uint32_t r[16];
-                    tmem_ld_16x128b_x4_pair(tbase + 16 * chunk, tbase + (16u << 16) + 16 * chunk, r);
-                    tmem_wait_ld(r);
-                    const float4 sw = lds_f4(side_w + 16 * chunk * 4);
-                    const float swv[4] = {sw.x, sw.y, sw.z, sw.w};
-                    float4 zw4 = make_float4(0.f, 0.f, 0.f, 0.f), gw4 = zw4;
-                    if (MODE == QUARTZ_ASYMMETRIC) {
-                        zw4 = lds_f4(side_w + (BN + 16 * chunk) * 4);
-                        gw4 = lds_f4(side_w + (2 * BN + 16 * chunk) * 4);
+                    for (int j = 0; j < 8; ++j) acc64[c][j] = 0ull;
+                for (int g = 0; g < G; ++g, ++it) {
+                    const int b = it & 1;
+                    const int ss = it % S;
+                    if (!mbar_wait_bounded(side_full_bar(ss), (it / S) & 1, abort_flag, args.dev_err,
+                                           kWaitLimitNs)) {
+                        ok = false;
+                        break;
                     }
-                    const float zwv[4] = {zw4.x, zw4.y, zw4.z, zw4.w};
-                    const float gwv[4] = {gw4.x, gw4.y, gw4.z, gw4.w};
-#pragma unroll
-                    for (int h = 0; h < 2; ++h) {
-#pragma unroll
-                        for (int i = 0; i < 4; ++i) {
-                            float2 p = make_float2(__uint_as_float(r[8 * h + 2 * i]), __uint_as_float(r[8 * h + 2 * i + 1]));
-                            if (DUMP && g == args.partials_group) {
-                                int mt, nt;
-                                tile_coords(tile, args, mt, nt);
-                                const int64_t m = static_cast<int64_t>(mt) * BM + quarter * 32 + 16 * h + trow;
-                                const int64_t n = static_cast<int64_t>(nt) * BN + slot * kColsPerWarp + 16 * chunk + tq + i;
-                                if (n < args.N) {
-                                    if (m < args.M) args.partials[m * args.N + n] = __float2int_rn(p.x);
-                                    if (m + 8 < args.M) args.partials[(m + 8) * args.N + n] = __float2int_rn(p.y);
-                                }
-                            }
-                            if (MODE == QUARTZ_ASYMMETRIC) {
-                                const float2 ua = make_float2(cur_a[2][2 * h], cur_a[2][2 * h + 1]);
-                                const float2 nza = make_float2(-cur_a[1][2 * h], -cur_a[1][2 * h + 1]);
-                                p = __ffma2_rn(make_float2(zwv[i], zwv[i]), ua, p);
-                                p = __ffma2_rn(nza, make_float2(gwv[i], gwv[i]), p);
-                            }
-                            const float2 t = __fmul2_rn(p, make_float2(swv[i], swv[i]));
-                            acc[h][4 * chunk + i] = __ffma2_rn(t, make_float2(cur_a[0][2 * h], cur_a[0][2 * h + 1]),
-                                                               acc[h][4 * chunk + i]);
-                        }
+                    const uint32_t side_a = smem_base + L::kSide + ss * L::kSideSlotBytes + (quarter * 32 + 4 * trow) * 4;
+                    const uint32_t side_w = smem_base + L::kSide + ss * L::kSideSlotBytes + L::kSideABytes +
+                                            (slot * kColsPerWarp + tq) * 4;
+                    if (!mbar_wait_bounded(acc_full_bar(b), (it >> 1) & 1, abort_flag, args.dev_err,
+                                           kWaitLimitNs)) {
+                        ok = false;
+                        break;
                     }
-                }
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) {
-                    mbar_arrive(acc_empty_bar(b));
-                    mbar_arrive(side_empty_bar(ss));
-                }
-            }
-            if (!ok) break;
-            int mt, nt;
-            tile_coords(tile, args, mt, nt);
-            // ---- store: 4 rows x 4 chunks of 4 consecutive columns per thread ----
-#pragma unroll
-            for (int h = 0; h < 2; ++h)
-#pragma unroll
-                for (int e = 0; e < 2; ++e) {
-                    const int64_t m = static_cast<int64_t>(mt) * BM + quarter * 32 + 16 * h + 8 * e + trow;
-                    if (m >= args.M) continue;
+                    uint64_t sa0, sa1;
+                    lds_b64x2(side_a, sa0, sa1);
+                    tc_fence_after();
+                    const uint32_t tbase = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
+                                           static_cast<uint32_t>(b * BN + slot * kColsPerWarp);
 #pragma unroll
                     for (int chunk = 0; chunk < 4; ++chunk) {
-                        const int64_t n = static_cast<int64_t>(nt) * BN + slot * kColsPerWarp + 16 * chunk + tq;
-                        if (n >= args.N) continue;
-                        float4 v;
-                        v.x = e ? acc[h][4 * chunk + 0].y : acc[h][4 * chunk + 0].x;
-                        v.y = e ? acc[h][4 * chunk + 1].y : acc[h][4 * chunk + 1].x;
-                        v.z = e ? acc[h][4 * chunk + 2].y : acc[h][4 * chunk + 2].x;
-                        v.w = e ? acc[h][4 * chunk + 3].y : acc[h][4 * chunk + 3].x;
-                        if (args.bias) {
-                            const uint2 braw = __ldg(reinterpret_cast<const uint2 *>(args.bias + n));
-                            const float2 b0 = __half22float2(*reinterpret_cast<const __half2 *>(&braw.x));
-                            const float2 b1 = __half22float2(*reinterpret_cast<const __half2 *>(&braw.y));
-                            v.x = __fadd_rn(v.x, b0.x);
-                            v.y = __fadd_rn(v.y, b0.y);
-                            v.z = __fadd_rn(v.z, b1.x);
-                            v.w = __fadd_rn(v.w, b1.y);
-                        }
-                        store_quad<OUT>(args.y, m * args.N + n, v);
+                        const float4 sw = lds_f4(side_w + 16 * chunk * 4);
+                        epi_chunk_sym(tbase + 16 * chunk, tbase + (16u << 16) + 16 * chunk, sw, sa0, sa1, acc64[chunk]);
+                    }
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) {
+                        mbar_arrive(acc_empty_bar(b));
+                        mbar_arrive(side_empty_bar(ss));
                     }
                 }
+                if (!ok) break;
+                int mt, nt;
+                tile_coords(tile, args, mt, nt);
+#pragma unroll
+                for (int h = 0; h < 2; ++h)
+#pragma unroll
+                    for (int e = 0; e < 2; ++e) {
+                        const int64_t m = static_cast<int64_t>(mt) * BM + quarter * 32 + 16 * h + 8 * e + trow;
+                        if (m >= args.M) continue;
+#pragma unroll
+                        for (int chunk = 0; chunk < 4; ++chunk) {
+                            const int64_t n = static_cast<int64_t>(nt) * BN + slot * kColsPerWarp + 16 * chunk + tq;
+                            if (n >= args.N) continue;
+                            float4 v;
+                            float vv[4];
+#pragma unroll
+                            for (int i = 0; i < 4; ++i) {
+                                const uint64_t q = acc64[chunk][4 * h + i];
+                                vv[i] = __uint_as_float(static_cast<uint32_t>(e ? (q >> 32) : q));
+                            }
+                            v = make_float4(vv[0], vv[1], vv[2], vv[3]);
+                            if (args.bias) {
+                                const uint2 braw = __ldg(reinterpret_cast<const uint2 *>(args.bias + n));
+                                const float2 b0 = __half22float2(*reinterpret_cast<const __half2 *>(&braw.x));
+                                const float2 b1 = __half22float2(*reinterpret_cast<const __half2 *>(&braw.y));
+                                v.x = __fadd_rn(v.x, b0.x);
+                                v.y = __fadd_rn(v.y, b0.y);
+                                v.z = __fadd_rn(v.z, b1.x);
+                                v.w = __fadd_rn(v.w, b1.y);
+                            }
+                            store_quad<OUT>(args.y, m * args.N + n, v);
+                        }
+                    }
+            }
+        } else {
+            float2 acc[2][16];
+            int it = 0;
+            bool ok = true;
+            for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
+#pragma unroll
+                for (int h = 0; h < 2; ++h)
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) acc[h][j] = make_float2(0.f, 0.f);
+                for (int g = 0; g < G; ++g, ++it) {
+                    const int b = it & 1;
+                    const int ss = it % S;
+                    if (!mbar_wait_bounded(side_full_bar(ss), (it / S) & 1, abort_flag, args.dev_err,
+                                           kWaitLimitNs)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t side_a = smem_base + L::kSide + ss * L::kSideSlotBytes + (quarter * 32 + 4 * trow) * 4;
+                    const uint32_t side_w = smem_base + L::kSide + ss * L::kSideSlotBytes + L::kSideABytes +
+                                            (slot * kColsPerWarp + tq) * 4;
+                    if (!mbar_wait_bounded(acc_full_bar(b), (it >> 1) & 1, abort_flag, args.dev_err,
+                                           kWaitLimitNs)) {
+                        ok = false;
+                        break;
+                    }
+                    // cur_a[sd][k]: side value sd of row trow + 8k of the quarter
+                    float cur_a[NSIDE][4];
+#pragma unroll
+                    for (int sd = 0; sd < NSIDE; ++sd) {
+                        const float4 v = lds_f4(side_a + sd * BM * 4);
+                        cur_a[sd][0] = v.x;
+                        cur_a[sd][1] = v.y;
+                        cur_a[sd][2] = v.z;
+                        cur_a[sd][3] = v.w;
+                    }
+                    tc_fence_after();
+                    const uint32_t tbase = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
+                                           static_cast<uint32_t>(b * BN + slot * kColsPerWarp);
+#pragma unroll
+                    for (int chunk = 0; chunk < 4; ++chunk) {    // 16-column chunks of the slice
+                        uint32_t r[16];
+                        tmem_ld_16x128b_x4_pair(tbase + 16 * chunk, tbase + (16u << 16) + 16 * chunk, r);
+                        tmem_wait_ld(r);
+                        const float4 sw = lds_f4(side_w + 16 * chunk * 4);
+                        const float swv[4] = {sw.x, sw.y, sw.z, sw.w};
+                        float4 zw4 = make_float4(0.f, 0.f, 0.f, 0.f), gw4 = zw4;
+                        if (MODE == QUARTZ_ASYMMETRIC) {
+                            zw4 = lds_f4(side_w + (BN + 16 * chunk) * 4);
+                            gw4 = lds_f4(side_w + (2 * BN + 16 * chunk) * 4);
+                        }
+                        const float zwv[4] = {zw4.x, zw4.y, zw4.z, zw4.w};
+                        const float gwv[4] = {gw4.x, gw4.y, gw4.z, gw4.w};
+#pragma unroll
+                        for (int h = 0; h < 2; ++h) {
+#pragma unroll
+                            for (int i = 0; i < 4; ++i) {
+                                float2 p = make_float2(__uint_as_float(r[8 * h + 2 * i]), __uint_as_float(r[8 * h + 2 * i + 1]));
+                                if (DUMP && g == args.partials_group) {
+                                    int mt, nt;
+                                    tile_coords(tile, args, mt, nt);
+                                    const int64_t m = static_cast<int64_t>(mt) * BM + quarter * 32 + 16 * h + trow;
+                                    const int64_t n = static_cast<int64_t>(nt) * BN + slot * kColsPerWarp + 16 * chunk + tq + i;
+                                    if (n < args.N) {
+                                        if (m < args.M) args.partials[m * args.N + n] = __float2int_rn(p.x);
+                                        if (m + 8 < args.M) args.partials[(m + 8) * args.N + n] = __float2int_rn(p.y);
+                                    }
+                                }
+                                if (MODE == QUARTZ_ASYMMETRIC) {
+                                    const float2 ua = make_float2(cur_a[2][2 * h], cur_a[2][2 * h + 1]);
+                                    const float2 nza = make_float2(-cur_a[1][2 * h], -cur_a[1][2 * h + 1]);
+                                    p = __ffma2_rn(make_float2(zwv[i], zwv[i]), ua, p);
+                                    p = __ffma2_rn(nza, make_float2(gwv[i], gwv[i]), p);
+                                }
+                                const float2 t = __fmul2_rn(p, make_float2(swv[i], swv[i]));
+                                acc[h][4 * chunk + i] = __ffma2_rn(t, make_float2(cur_a[0][2 * h], cur_a[0][2 * h + 1]),
+                                                                   acc[h][4 * chunk + i]);
+                            }
+                        }
+                    }
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) {
+                        mbar_arrive(acc_empty_bar(b));
+                        mbar_arrive(side_empty_bar(ss));
+                    }
+                }
+                if (!ok) break;
+                int mt, nt;
+                tile_coords(tile, args, mt, nt);
+                // ---- store: 4 rows x 4 chunks of 4 consecutive columns per thread ----
+#pragma unroll
+                for (int h = 0; h < 2; ++h)
+#pragma unroll
+                    for (int e = 0; e < 2; ++e) {
+                        const int64_t m = static_cast<int64_t>(mt) * BM + quarter * 32 + 16 * h + 8 * e + trow;
+                        if (m >= args.M) continue;
+#pragma unroll
+                        for (int chunk = 0; chunk < 4; ++chunk) {
+                            const int64_t n = static_cast<int64_t>(nt) * BN + slot * kColsPerWarp + 16 * chunk + tq;
+                            if (n >= args.N) continue;
+                            float4 v;
+                            v.x = e ? acc[h][4 * chunk + 0].y : acc[h][4 * chunk + 0].x;
+                            v.y = e ? acc[h][4 * chunk + 1].y : acc[h][4 * chunk + 1].x;
+                            v.z = e ? acc[h][4 * chunk + 2].y : acc[h][4 * chunk + 2].x;
+                            v.w = e ? acc[h][4 * chunk + 3].y : acc[h][4 * chunk + 3].x;
+                            if (args.bias) {
+                                const uint2 braw = __ldg(reinterpret_cast<const uint2 *>(args.bias + n));
+                                const float2 b0 = __half22float2(*reinterpret_cast<const __half2 *>(&braw.x));
+                                const float2 b1 = __half22float2(*reinterpret_cast<const __half2 *>(&braw.y));
+                                v.x = __fadd_rn(v.x, b0.x);
+                                v.y = __fadd_rn(v.y, b0.y);
+                                v.z = __fadd_rn(v.z, b1.x);
+                                v.w = __fadd_rn(v.w, b1.y);
+                            }
+                            store_quad<OUT>(args.y, m * args.N + n, v);
+                        }
+                    }
+            }
         }
     }
 
