@@ -125,14 +125,17 @@ constexpr int kABytes = BM * BK;      // E4M3 operands: one byte per element
 constexpr int kBBytes = BN * BK;
 constexpr int kStageBytes = kABytes + kBBytes;
 // Warpgroups 0-3 dequantise (16 warps: four per 32-lane TMEM quarter, 64
-// columns each); warpgroup 4 holds the TMA producer, the MMA issuer and two
-// idle warps.  The dequant epilogue is the throughput-critical part (two fp32
-// operations per output element per group, as many cycles as the MMAs), so it
-// gets four warps per scheduler to hide FMA and shared-memory latency.
+// columns each); warpgroup 4 holds the operand TMA producer, the MMA issuer,
+// the scale copier and one idle warp.  The dequant epilogue is the
+// throughput-critical part (two fp32 operations per output element per
+// group), so it gets four warps per scheduler; the three control roles sit on
+// three different schedulers (warp w runs on scheduler w % 4) because each
+// slows the epilogue warps that share its scheduler.
 constexpr int kEpiWarps = 16;
 constexpr int kThreads = (kEpiWarps + 4) * 32;
 constexpr int kProducerWarp = kEpiWarps;
 constexpr int kMmaWarp = kEpiWarps + 1;
+constexpr int kSideWarp = kEpiWarps + 2;
 constexpr int kColsPerWarp = BN / 4;
 // Register split (setmaxnreg): 640 threads launch with 96 registers each;
 // warpgroup 4 drops to 32 so the epilogue warpgroups can hold 112
@@ -285,20 +288,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ------------------------------------------------------------------
         // TMA producer: one stage = one 64-wide group of A (128 rows) and W
         // (256 rows).  Rows past M or N are zero-filled by the tensor map.
-        // The group's side values (scales; asymmetric also zero-point terms)
-        // go by bulk copy into their own ring slot, which the epilogue frees.
         // ------------------------------------------------------------------
         if (lane == 0) {
-            constexpr int S = L::kSideSlots;
-            const int64_t a_plane = args.m_pad * G;
-            const int64_t w_plane = args.n_pad * G;
-            int it = 0;       // groups whose operand copies were issued
-            int it_side = 0;  // groups whose side-value copies were issued
+            int it = 0;  // groups whose operand copies were issued
             bool ok = true;
             for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
                 int mt, nt;
                 tile_coords(tile, args, mt, nt);
-                for (int g = 0; g < G; ++g) {
+                for (int g = 0; g < G; ++g, ++it) {
                     const int s = it % kStages;
                     if (it >= kStages &&
                         !mbar_wait_bounded(empty_bar(s), ((it / kStages) - 1) & 1, abort_flag,
@@ -310,37 +307,53 @@ __global__ void __launch_bounds__(kThreads, 1)
                     mbar_arrive_expect_tx(full_bar(s), kStageBytes);
                     tma_load_2d(sa, &tmap_a, g * BK, mt * BM, full_bar(s));
                     tma_load_2d(sa + kABytes, &tmap_w, g * BK, nt * BN, full_bar(s));
-                    ++it;
-
-                    const int ss = it_side % S;
-                    if (it_side >= S && !mbar_wait_bounded(side_empty_bar(ss), ((it_side / S) - 1) & 1,
-                                                           abort_flag, args.dev_err, kWaitLimitNs)) {
-                        ok = false;
-                        break;
-                    }
-                    const uint32_t sd_dst = smem_base + L::kSide + ss * L::kSideSlotBytes;
-                    mbar_arrive_expect_tx(side_full_bar(ss), L::kSideSlotBytes);
-                    const float *src_a = args.a_side + static_cast<int64_t>(g) * args.m_pad + static_cast<int64_t>(mt) * BM;
-                    const float *src_w = args.w_side + static_cast<int64_t>(g) * args.n_pad + static_cast<int64_t>(nt) * BN;
-#pragma unroll
-                    for (int sd = 0; sd < NSIDE; ++sd) {
-                        bulk_load(sd_dst + sd * BM * 4, src_a + sd * a_plane, BM * 4, side_full_bar(ss));
-                        bulk_load(sd_dst + L::kSideABytes + sd * BN * 4, src_w + sd * w_plane, BN * 4,
-                                  side_full_bar(ss));
-                    }
-                    ++it_side;
                 }
             }
             // Never leave the CTA with copies in flight: wait for the last
-            // load issued into every stage and side slot (bounded, even after
-            // an abort).
+            // load issued into every stage (bounded, even after an abort).
             int zero = 0;
             for (int s = 0; s < kStages && s < it; ++s) {
                 const int last = it - 1 - ((it - 1 - s) % kStages);
                 mbar_wait_bounded(full_bar(s), (last / kStages) & 1, &zero, args.dev_err, kWaitLimitNs);
             }
-            for (int s = 0; s < S && s < it_side; ++s) {
-                const int last = it_side - 1 - ((it_side - 1 - s) % S);
+        }
+        __syncwarp();
+      } else if (warp == kSideWarp) {
+        // ------------------------------------------------------------------
+        // Scale copier: each group's side values (scales; asymmetric also
+        // zero-point terms) go by bulk copy into a ring slot that the
+        // epilogue frees.
+        // ------------------------------------------------------------------
+        if (lane == 0) {
+            constexpr int S = L::kSideSlots;
+            const int64_t a_plane = args.m_pad * G;
+            const int64_t w_plane = args.n_pad * G;
+            int it = 0;  // groups whose side-value copies were issued
+            bool ok = true;
+            for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
+                int mt, nt;
+                tile_coords(tile, args, mt, nt);
+                for (int g = 0; g < G; ++g, ++it) {
+                    const int ss = it % S;
+                    if (it >= S && !mbar_wait_bounded(side_empty_bar(ss), ((it / S) - 1) & 1, abort_flag,
+                                                      args.dev_err, kWaitLimitNs)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t dst = smem_base + L::kSide + ss * L::kSideSlotBytes;
+                    mbar_arrive_expect_tx(side_full_bar(ss), L::kSideSlotBytes);
+                    const float *src_a = args.a_side + static_cast<int64_t>(g) * args.m_pad + static_cast<int64_t>(mt) * BM;
+                    const float *src_w = args.w_side + static_cast<int64_t>(g) * args.n_pad + static_cast<int64_t>(nt) * BN;
+#pragma unroll
+                    for (int sd = 0; sd < NSIDE; ++sd) {
+                        bulk_load(dst + sd * BM * 4, src_a + sd * a_plane, BM * 4, side_full_bar(ss));
+                        bulk_load(dst + L::kSideABytes + sd * BN * 4, src_w + sd * w_plane, BN * 4, side_full_bar(ss));
+                    }
+                }
+            }
+            int zero = 0;
+            for (int s = 0; s < S && s < it; ++s) {
+                const int last = it - 1 - ((it - 1 - s) % S);
                 mbar_wait_bounded(side_full_bar(s), (last / S) & 1, &zero, args.dev_err, kWaitLimitNs);
             }
         }
