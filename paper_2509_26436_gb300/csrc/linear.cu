@@ -209,19 +209,41 @@ __device__ __forceinline__ void store_quad(void *y, int64_t off, float4 v)
     }
 }
 
-// One 16-column chunk of the epilogue: two 16x128b.x4 TMEM loads (lanes +0
-// and +16), then acc[h][i] += s_a[h] * (s_w[i] * P) on (row, row + 8) pairs,
-// all on explicit 64-bit register pairs.
-__device__ __forceinline__ void epi_chunk_sym(uint32_t t0, uint32_t t1, float4 sw, uint64_t sa0, uint64_t sa1,
-                                              uint64_t (&acc)[8])
+// Half of one 16-column chunk: one 16x128b.x4 TMEM load (16 lanes), then
+// acc[i] += s_a * (s_w[i] * P_i) for the four pairs P_i = (row, row + 8) of
+// column i, on explicit 64-bit register pairs (q: the loaded pairs, s: the
+// column scale duplicated into both halves, t: s_w * P).
+__device__ __forceinline__ void epi_half_chunk_sym(uint32_t taddr, float4 sw, uint64_t sa, uint64_t *acc)
 {
-    asm volatile("{\n\t.reg .b32 p<16>;\n\t.reg .b64 q<8>, t<8>, s<4>;\n\ttcgen05.ld.sync.aligned.16x128b.x4.b32 {p0,p1,p2,p3,p4,p5,p6,p7}, [%8];\n\ttcgen05.ld.sync.aligned.16x128b.x4.b32 {p8,p9,p10,p11,p12,p13,p14,p15}, [%9];\n\ttcgen05.wait::ld.sync.aligned;\n\tmov.b64 q0, {p0, p1};\n\tmov.b64 q1, {p2, p3};\n\tmov.b64 q2, {p4, p5};\n\tmov.b64 q3, {p6, p7};\n\tmov.b64 q4, {p8, p9};\n\tmov.b64 q5, {p10, p11};\n\tmov.b64 q6, {p12, p13};\n\tmov.b64 q7, {p14, p15};\n\tmov.b64 s0, {%10, %10};\n\tmov.b64 s1, {%11, %11};\n\tmov.b64 s2, {%12, %12};\n\tmov.b64 s3, {%13, %13};\n\tmul.rn.f32x2 t0, q0, s0;\n\tmul.rn.f32x2 t1, q1, s1;\n\tmul.rn.f32x2 t2, q2, s2;\n\tmul.rn.f32x2 t3, q3, s3;\n\tmul.rn.f32x2 t4, q4, s0;\n\tmul.rn.f32x2 t5, q5, s1;\n\tmul.rn.f32x2 t6, q6, s2;\n\tmul.rn.f32x2 t7, q7, s3;\n\tfma.rn.f32x2 %0, t0, %14, %0;\n\tfma.rn.f32x2 %1, t1, %14, %1;\n\tfma.rn.f32x2 %2, t2, %14, %2;\n\tfma.rn.f32x2 %3, t3, %14, %3;\n\tfma.rn.f32x2 %4, t4, %15, %4;\n\tfma.rn.f32x2 %5, t5, %15, %5;\n\tfma.rn.f32x2 %6, t6, %15, %6;\n\tfma.rn.f32x2 %7, t7, %15, %7;\n\t}"
-                 : "+l"(acc[0]), "+l"(acc[1]), "+l"(acc[2]), "+l"(acc[3]), "+l"(acc[4]), "+l"(acc[5]),
-                   "+l"(acc[6]), "+l"(acc[7])
-                 : "r"(t0), "r"(t1), "f"(sw.x), "f"(sw.y), "f"(sw.z), "f"(sw.w), "l"(sa0), "l"(sa1)
-                 : "memory");
+    asm volatile(
+        "{\n\t"
+        ".reg .b32 p<8>;\n\t"
+        ".reg .b64 q<4>, t<4>, s<4>;\n\t"
+        "tcgen05.ld.sync.aligned.16x128b.x4.b32 {p0, p1, p2, p3, p4, p5, p6, p7}, [%4];\n\t"
+        "tcgen05.wait::ld.sync.aligned;\n\t"
+        "mov.b64 q0, {p0, p1};\n\t"
+        "mov.b64 q1, {p2, p3};\n\t"
+        "mov.b64 q2, {p4, p5};\n\t"
+        "mov.b64 q3, {p6, p7};\n\t"
+        "mov.b64 s0, {%5, %5};\n\t"
+        "mov.b64 s1, {%6, %6};\n\t"
+        "mov.b64 s2, {%7, %7};\n\t"
+        "mov.b64 s3, {%8, %8};\n\t"
+        "mul.rn.f32x2 t0, q0, s0;\n\t"
+        "fma.rn.f32x2 %0, t0, %9, %0;\n\t"
+        "mul.rn.f32x2 t1, q1, s1;\n\t"
+        "fma.rn.f32x2 %1, t1, %9, %1;\n\t"
+        "mul.rn.f32x2 t2, q2, s2;\n\t"
+        "fma.rn.f32x2 %2, t2, %9, %2;\n\t"
+        "mul.rn.f32x2 t3, q3, s3;\n\t"
+        "fma.rn.f32x2 %3, t3, %9, %3;\n\t"
+        "}"
+        : "+l"(acc[0]), "+l"(acc[1]), "+l"(acc[2]), "+l"(acc[3])
+        : "r"(taddr), "f"(sw.x), "f"(sw.y), "f"(sw.z), "f"(sw.w), "l"(sa)
+        : "memory");
 }
 
+// Two 64-bit words from shared memory (one 16-byte load).
 __device__ __forceinline__ void lds_b64x2(uint32_t addr, uint64_t &a, uint64_t &b)
 {
     asm volatile("ld.shared.v2.b64 {%0, %1}, [%2];" : "=l"(a), "=l"(b) : "r"(addr) : "memory");
@@ -427,8 +449,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         // acc[h][j]: output column 16*(j/4) + tq + j%4 of this warp's slice,
         // rows trow + 16h (.x) and trow + 16h + 8 (.y)
         if constexpr (MODE == QUARTZ_SYMMETRIC && !DUMP) {
-            // Symmetric fast path: each 16-column chunk (TMEM loads, wait and
-            // the scale arithmetic) is one PTX block on explicit 64-bit pairs.
+            // Symmetric fast path: each half chunk (16 lanes x 16 columns: TMEM
+            // load, wait and the scale arithmetic) is one PTX block on
+            // explicit 64-bit pairs, which keeps the kernel free of spills.
             // acc64[c][4h + i]: output column 16c + tq + i, rows trow + 16h (low) and + 8 (high)
             uint64_t acc64[4][8];
             int it = 0;
@@ -462,7 +485,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                     for (int chunk = 0; chunk < 4; ++chunk) {
                         const float4 sw = lds_f4(side_w + 16 * chunk * 4);
-                        epi_chunk_sym(tbase + 16 * chunk, tbase + (16u << 16) + 16 * chunk, sw, sa0, sa1, acc64[chunk]);
+                        epi_half_chunk_sym(tbase + 16 * chunk, sw, sa0, acc64[chunk]);
+                        epi_half_chunk_sym(tbase + (16u << 16) + 16 * chunk, sw, sa1, acc64[chunk] + 4);
                     }
                     tc_fence_before();
                     __syncwarp();
