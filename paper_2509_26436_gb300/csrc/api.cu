@@ -172,8 +172,7 @@ int32_t quartz_linear_ex(const quartz_encoded_t *a, const quartz_encoded_t *w,
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     LinearWorkspace ws;
     linear_workspace_carve(workspace, M, N, K, a->p.mode, &ws);
-    cudaError_t e = launch_expand(a, ws.a_op, ws.a_side, ws.m_pad, 1, s);
-    if (e == cudaSuccess) e = launch_expand(w, ws.w_op, ws.w_side, ws.n_pad, 0, s);
+    cudaError_t e = launch_prepare(a, w, ws, s);
     if (e != cudaSuccess) return QUARTZ_ERR_CUDA;
     if (o.gemm_event_begin && cudaEventRecord(static_cast<cudaEvent_t>(o.gemm_event_begin), s) != cudaSuccess)
         return QUARTZ_ERR_CUDA;

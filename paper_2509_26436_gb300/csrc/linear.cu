@@ -51,35 +51,45 @@ __host__ __device__ __forceinline__ int64_t perm16(int64_t r)
     return (r & ~int64_t(15)) | ((r & 3) << 2) | ((r >> 2) & 3);
 }
 
-template <int GS>
-__global__ void __launch_bounds__(256) expand_kernel(const uint32_t *__restrict__ codes,
-                                                     const uint8_t *__restrict__ flags,
-                                                     int64_t n_chunks, int64_t chunks_per_row,
-                                                     int64_t n_chunks_pad, int permute,
-                                                     uint2 *__restrict__ op)
+// Byte permute (PTX prmt, default mode: a selector nibble b < 8 copies byte b
+// of {hi:lo}, b + 8 replicates that byte's sign bit).
+__device__ __forceinline__ uint32_t prmt(uint32_t lo, uint32_t hi, uint32_t sel)
 {
-    const int64_t c = static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x;
-    if (c >= n_chunks_pad) return;
-    int64_t dst = c;
-    if (permute) {
-        const int64_t r = c / chunks_per_row;
-        dst = perm16(r) * chunks_per_row + (c - r * chunks_per_row);
-    }
-    if (c >= n_chunks) {  // padding rows up to a multiple of 16
-        op[dst] = make_uint2(0, 0);
-        return;
-    }
-    const uint32_t word = codes[c];
-    const int flag = flags[(c * 8) / GS];
-    const int mul = 1 << flag;
-    uint32_t o[2] = {0u, 0u};
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-        const int ci = static_cast<int>(word << (28 - 4 * i)) >> 28;
-        const uint32_t byte = __nv_cvt_float_to_fp8(static_cast<float>(ci * mul), __NV_SATFINITE, __NV_E4M3);
-        o[i >> 2] |= byte << (8 * (i & 3));
-    }
-    op[dst] = make_uint2(o[0], o[1]);
+    uint32_t d;
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(lo), "r"(hi), "r"(sel));
+    return d;
+}
+
+// Four table lookups at once: byte k of x (0..15) selects byte x_k of the
+// 16-byte table {t0, t1, t2, t3}.
+__device__ __forceinline__ uint32_t lut16(uint32_t x, uint32_t t0, uint32_t t1, uint32_t t2, uint32_t t3)
+{
+    const uint32_t y = x & 0x07070707u;
+    const uint32_t sel = prmt(y | (y >> 4), 0u, 0x0020u);  // nibble k = low 3 bits of byte k
+    const uint32_t lo = prmt(t0, t1, sel);
+    const uint32_t hi = prmt(t2, t3, sel);
+    const uint32_t use_hi = prmt(x << 4, 0u, 0xBA98u);      // 0xFF where bit 3 of byte k is set
+    return (hi & use_hi) | (lo & ~use_hi);
+}
+
+// Decode eight 4-bit codes (one 32-bit word, code k in bits 4k..4k+3) of one
+// subgroup with FLAG `flag` to E4M3 bytes of v = c * 2^flag, written to the
+// eight bytes of {lo, hi} in code order.  The E4M3 byte of a nonzero c is
+// sign | (7 + e + flag) << 3 | m for |c| = (1 + m/8) 2^e, so the table for
+// FLAG f is the FLAG-0 table with 8 f added to every nonzero entry (no carry
+// leaves a byte: the largest entry, 7 * 2^4 = 112, is 0x6E / 0xEE).
+__device__ __forceinline__ void e4m3_from_codes8(uint32_t word, int flag, uint32_t &lo, uint32_t &hi)
+{
+    const uint32_t add = (static_cast<uint32_t>(flag) << 3) * 0x01010101u;
+    // entries for codes 0..15 (two's complement -8..7; -8 never occurs)
+    const uint32_t t0 = 0x44403800u + (add & 0xFFFFFF00u);  //  0,  1,  2,  3
+    const uint32_t t1 = 0x4E4C4A48u + add;                  //  4,  5,  6,  7
+    const uint32_t t2 = 0xCACCCE00u + (add & 0xFFFFFF00u);  // -8, -7, -6, -5
+    const uint32_t t3 = 0xB8C0C4C8u + add;                  // -4, -3, -2, -1
+    const uint32_t ev = lut16(word & 0x0F0F0F0Fu, t0, t1, t2, t3);         // codes 0, 2, 4, 6
+    const uint32_t od = lut16((word >> 4) & 0x0F0F0F0Fu, t0, t1, t2, t3);  // codes 1, 3, 5, 7
+    lo = prmt(ev, od, 0x5140u);
+    hi = prmt(ev, od, 0x7362u);
 }
 
 // Position of activation row r in its group's side-value row: inside every
@@ -90,27 +100,101 @@ __host__ __device__ __forceinline__ int64_t perm32(int64_t r)
     return (r & ~int64_t(31)) | ((r & 7) << 2) | ((r >> 3) & 3);
 }
 
-// side[0][g][.] = s[r, g]; asymmetric adds side[1] = z and side[2] =
-// (is_a ? 64 z - gsum : gsum), so that the epilogue's integer correction is
-// P + z_w * (64 z_a - A_g) - z_a * W_g.  Rows in [rows, rows_pad) are 0.
-// Weight rows are stored in natural order, activation rows at perm32(r).
-__global__ void side_kernel(const __half *__restrict__ scales, const int8_t *__restrict__ zeros,
-                            const int32_t *__restrict__ gsum, int64_t rows, int64_t rows_pad,
-                            int G, int nside, int is_a, float *__restrict__ side)
+// One launch prepares both GEMM operands (jobs selected by block index):
+//   expand A, expand W: 16 codes per thread (8 bytes in, 16 E4M3 bytes out);
+//     the weight operand is row-permuted (perm16) and zero-padded to a
+//     multiple of 16 rows;
+//   side A, side W: side[0][g][.] = s[r, g]; asymmetric adds side[1] = z and
+//     side[2] = (is_a ? 64 z - gsum : gsum), so that the epilogue's integer
+//     correction is P + z_w * (64 z_a - A_g) - z_a * W_g.  Rows in
+//     [rows, rows_pad) are 0; weight rows are stored in natural order,
+//     activation rows at perm32(r).  One thread per row and 8 groups: its
+//     reads stay in L1 lines, consecutive threads write consecutive rows.
+struct ExpandJob {
+    const uint2 *codes;          // [rows, K/16] units of 16 codes
+    const uint8_t *flags;        // [rows, K/G_s]
+    uint4 *out;                  // [rows_out, K/16] units of 16 E4M3 values
+    int64_t units, units_pad, units_per_row;
+    int permute;
+};
+struct SideJob {
+    const __half *scales;
+    const int8_t *zeros;
+    const int32_t *gsum;
+    float *side;
+    int64_t rows, rows_pad;
+    int is_a;
+};
+struct PrepArgs {
+    ExpandJob ex_a, ex_w;
+    SideJob sd_a, sd_w;
+    int64_t block_end[4];        // cumulative block counts: expand A, expand W, side A, side W
+    int G, nside;
+};
+constexpr int kPrepThreads = 256;
+constexpr int kSideGroupsPerThread = 8;
+
+template <int GS>
+__device__ __forceinline__ void run_expand(const ExpandJob &j, int64_t u)
 {
-    const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
-    const int64_t total = rows_pad * G;
-    if (i >= total) return;
-    const int64_t g = i / rows_pad;
-    const int64_t r = i - g * rows_pad;
-    const int64_t o = g * rows_pad + (is_a ? perm32(r) : r);
-    const bool in = r < rows;
-    side[o] = in ? __half2float(scales[r * G + g]) : 0.f;
-    if (nside > 1) {
-        const float z = in ? static_cast<float>(zeros[r * G + g]) : 0.f;
-        const float gs = in ? static_cast<float>(gsum[r * G + g]) : 0.f;
-        side[total + o] = z;
-        side[2 * total + o] = is_a ? (static_cast<float>(kGroupQ) * z - gs) : gs;
+    if (u >= j.units_pad) return;
+    int64_t dst = u;
+    if (j.permute) {
+        const int64_t r = u / j.units_per_row;
+        dst = perm16(r) * j.units_per_row + (u - r * j.units_per_row);
+    }
+    if (u >= j.units) {  // padding rows
+        j.out[dst] = make_uint4(0, 0, 0, 0);
+        return;
+    }
+    const uint2 c = j.codes[u];
+    int f0, f1;
+    if (GS == 8) {
+        const uint32_t ff = reinterpret_cast<const uint16_t *>(j.flags)[u];
+        f0 = static_cast<int>(ff & 0xFFu);
+        f1 = static_cast<int>(ff >> 8);
+    } else {
+        f0 = f1 = j.flags[(u * 16) / GS];
+    }
+    uint4 o;
+    e4m3_from_codes8(c.x, f0, o.x, o.y);
+    e4m3_from_codes8(c.y, f1, o.z, o.w);
+    j.out[dst] = o;
+}
+
+__device__ __forceinline__ void run_side(const SideJob &j, int64_t t, int G, int nside)
+{
+    const int64_t r = t % j.rows_pad;
+    const int g0 = static_cast<int>(t / j.rows_pad) * kSideGroupsPerThread;
+    if (g0 >= G) return;
+    const int g1 = min(g0 + kSideGroupsPerThread, G);
+    const int64_t total = j.rows_pad * G;
+    const int64_t o = j.is_a ? perm32(r) : r;
+    const bool in = r < j.rows;
+    for (int g = g0; g < g1; ++g) {
+        const int64_t i = static_cast<int64_t>(g) * j.rows_pad + o;
+        j.side[i] = in ? __half2float(j.scales[r * G + g]) : 0.f;
+        if (nside > 1) {
+            const float z = in ? static_cast<float>(j.zeros[r * G + g]) : 0.f;
+            const float gs = in ? static_cast<float>(j.gsum[r * G + g]) : 0.f;
+            j.side[total + i] = z;
+            j.side[2 * total + i] = j.is_a ? (static_cast<float>(kGroupQ) * z - gs) : gs;
+        }
+    }
+}
+
+template <int GS>
+__global__ void __launch_bounds__(kPrepThreads) prep_kernel(const __grid_constant__ PrepArgs args)
+{
+    const int64_t bid = blockIdx.x;
+    if (bid < args.block_end[0]) {
+        run_expand<GS>(args.ex_a, bid * kPrepThreads + threadIdx.x);
+    } else if (bid < args.block_end[1]) {
+        run_expand<GS>(args.ex_w, (bid - args.block_end[0]) * kPrepThreads + threadIdx.x);
+    } else if (bid < args.block_end[2]) {
+        run_side(args.sd_a, (bid - args.block_end[1]) * kPrepThreads + threadIdx.x, args.G, args.nside);
+    } else {
+        run_side(args.sd_w, (bid - args.block_end[2]) * kPrepThreads + threadIdx.x, args.G, args.nside);
     }
 }
 
@@ -877,33 +961,37 @@ void linear_workspace_carve(void *base, int64_t M, int64_t N, int64_t K, int mod
     ws->w_side = reinterpret_cast<float *>(p);
 }
 
-cudaError_t launch_expand(const quartz_encoded_t *e, void *op, float *side, int64_t rows_pad,
-                          int is_a, cudaStream_t s)
+cudaError_t launch_prepare(const quartz_encoded_t *a, const quartz_encoded_t *w, const LinearWorkspace &ws,
+                           cudaStream_t s)
 {
-    const int64_t cpr = e->K / 8;
-    const int64_t n_chunks = e->rows * cpr;
+    const int64_t K = a->K;
+    const int64_t upr = K / 16;
+    PrepArgs p{};
+    p.G = static_cast<int>(K / kGroupQ);
+    p.nside = ws.nside;
+    p.ex_a = {reinterpret_cast<const uint2 *>(a->codes), a->flags, static_cast<uint4 *>(ws.a_op),
+              a->rows * upr, a->rows * upr, upr, 0};
     // the weight operand is row-permuted and padded to a multiple of 16 rows
-    const int64_t n_chunks_pad = is_a ? n_chunks : round_up(e->rows, 16) * cpr;
-    if (n_chunks_pad > 0) {
-        const unsigned blocks = static_cast<unsigned>((n_chunks_pad + 255) / 256);
-        const uint32_t *codes = reinterpret_cast<const uint32_t *>(e->codes);
-        uint2 *o = static_cast<uint2 *>(op);
-        const int perm = is_a ? 0 : 1;
-        switch (e->p.group_s) {
-            case 8: expand_kernel<8><<<blocks, 256, 0, s>>>(codes, e->flags, n_chunks, cpr, n_chunks_pad, perm, o); break;
-            case 16: expand_kernel<16><<<blocks, 256, 0, s>>>(codes, e->flags, n_chunks, cpr, n_chunks_pad, perm, o); break;
-            case 32: expand_kernel<32><<<blocks, 256, 0, s>>>(codes, e->flags, n_chunks, cpr, n_chunks_pad, perm, o); break;
-            default: expand_kernel<64><<<blocks, 256, 0, s>>>(codes, e->flags, n_chunks, cpr, n_chunks_pad, perm, o); break;
-        }
-        cudaError_t err = cudaGetLastError();
-        if (err != cudaSuccess) return err;
+    p.ex_w = {reinterpret_cast<const uint2 *>(w->codes), w->flags, static_cast<uint4 *>(ws.w_op),
+              w->rows * upr, round_up(w->rows, 16) * upr, upr, 1};
+    p.sd_a = {reinterpret_cast<const __half *>(a->scales), a->zeros, a->gsum, ws.a_side, a->rows, ws.m_pad, 1};
+    p.sd_w = {reinterpret_cast<const __half *>(w->scales), w->zeros, w->gsum, ws.w_side, w->rows, ws.n_pad, 0};
+    const int64_t side_chunks = (p.G + kSideGroupsPerThread - 1) / kSideGroupsPerThread;
+    const int64_t threads[4] = {p.ex_a.units_pad, p.ex_w.units_pad, ws.m_pad * side_chunks,
+                                ws.n_pad * side_chunks};
+    int64_t acc = 0;
+    for (int i = 0; i < 4; ++i) {
+        acc += (threads[i] + kPrepThreads - 1) / kPrepThreads;
+        p.block_end[i] = acc;
     }
-    const int G = static_cast<int>(e->K / kGroupQ);
-    const int nside = e->p.mode == QUARTZ_ASYMMETRIC ? 3 : 1;
-    const int64_t total = rows_pad * G;
-    side_kernel<<<static_cast<unsigned>((total + 255) / 256), 256, 0, s>>>(
-        reinterpret_cast<const __half *>(e->scales), e->zeros, e->gsum, e->rows, rows_pad, G,
-        nside, is_a, side);
+    if (acc == 0) return cudaSuccess;
+    const unsigned blocks = static_cast<unsigned>(acc);
+    switch (a->p.group_s) {
+        case 8: prep_kernel<8><<<blocks, kPrepThreads, 0, s>>>(p); break;
+        case 16: prep_kernel<16><<<blocks, kPrepThreads, 0, s>>>(p); break;
+        case 32: prep_kernel<32><<<blocks, kPrepThreads, 0, s>>>(p); break;
+        default: prep_kernel<64><<<blocks, kPrepThreads, 0, s>>>(p); break;
+    }
     return cudaGetLastError();
 }
 

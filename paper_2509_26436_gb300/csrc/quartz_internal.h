@@ -37,8 +37,10 @@ struct LinearWorkspace {
 size_t linear_workspace_bytes(int64_t M, int64_t N, int64_t K, int mode);
 void linear_workspace_carve(void *base, int64_t M, int64_t N, int64_t K, int mode,
                             LinearWorkspace *ws);
-cudaError_t launch_expand(const quartz_encoded_t *e, void *op, float *side, int64_t rows_pad,
-                          int is_a, cudaStream_t s);
+// Expands both operands to E4M3 and transposes their scales into the
+// workspace (one launch).
+cudaError_t launch_prepare(const quartz_encoded_t *a, const quartz_encoded_t *w, const LinearWorkspace &ws,
+                           cudaStream_t s);
 cudaError_t launch_gemm_tcgen05(const LinearWorkspace &ws, int64_t M, int64_t N, int64_t K,
                                 int mode, const void *bias, void *y, int y_type,
                                 int32_t *partials, int partials_group, int *dev_err,

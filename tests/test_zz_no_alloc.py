@@ -57,7 +57,8 @@ def test_noalloc_matches_workspace_entry_point(Q):
 
 def test_noalloc_rejects_oversized_problem(Q):
     lib = Q._native.load()
-    # a workspace of about 2 x 8192 x 4096 x 2 bytes, far above the scratch array
+    # a workspace of more than 2 x 8192 x 4096 bytes (both operands expanded to one
+    # byte per element), far above the 32 MiB scratch array
     p = Q._native.QuartzParams(64, 16, 0)
     a = Q._native.QuartzEncoded(0x1000, 0x1000, 0x1000, 0, 0, 8192, 4096, p)
     w = Q._native.QuartzEncoded(0x1000, 0x1000, 0x1000, 0, 0, 8192, 4096, p)
