@@ -334,7 +334,7 @@ def run_ours(args):
     t_floor_alu = epi_ops / (alu_peak * 1e12)
     elems = sum(l.M * l.K for l in layers)
     enc_gbs = elems * encode_bytes_per_elem() / (sum(quant_ms) / 1e3) / 1e9
-    launches_per_step = nl * (1 + 5)   # quantize; expand A, side A, expand W, side W, GEMM
+    launches_per_step = nl * 3   # quantize; prepare (both operands); GEMM
 
     # ---- end to end through the public API with host buffers ---------------
     # Each (step, layer) unit copies its activations from pinned host memory,
