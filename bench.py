@@ -44,6 +44,7 @@ def parse():
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
     p.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline leg")
+    p.add_argument("--no-fused", action="store_true", help="skip the fused activation-path leg")
     p.add_argument("--layers", default="", help="comma-separated subset of layer names (profiling)")
     return p.parse_args()
 
@@ -336,6 +337,35 @@ def run_ours(args):
     enc_gbs = elems * encode_bytes_per_elem() / (sum(quant_ms) / 1e3) / 1e9
     launches_per_step = nl * 3   # quantize; prepare (both operands); GEMM
 
+    # ---- fused activation path (quartz_linear_f16: encode into the operand) -
+    fused = None
+    if not args.no_fused:
+        def fused_step():
+            for i in range(nl):
+                Q.linear_f16(x_dev[i], enc_w[i], out=y_dev[i], workspace=workspace)
+
+        for _ in range(args.warmup):
+            fused_step()
+        torch.cuda.synchronize()
+        barrier()
+        f0, f1 = ev(), ev()
+        f0.record(stream)
+        for _ in range(args.steps):
+            fused_step()
+        f1.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        assert Q.device_status() == 0
+        tf = f0.elapsed_time(f1) / 1e3 / args.steps
+        if world > 1:
+            import torch.distributed as dist
+            t = torch.tensor([tf], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            tf = float(t.item())
+        fused = {"value": world * ops_step / tf / 1e12, "unit": "TOPS", "ms_per_step": tf * 1e3,
+                 "path": "quartz_linear_f16 per layer (activations encoded straight into the GEMM "
+                         "operand; bit-identical to quantize + linear)"}
+
     # ---- end to end through the public API with host buffers ---------------
     # Each (step, layer) unit copies its activations from pinned host memory,
     # encodes them, runs the linear layer and copies the fp16 output back to
@@ -436,6 +466,7 @@ def run_ours(args):
                    "per_layer_ms": quant_ms, "peak_source": peak_src},
         "clocks": clocks,
         "gpu_launches": launches_per_step * args.steps,
+        "fused": fused,
         "e2e": e2e,
         "cpu_baseline": cpu,
     }

@@ -165,6 +165,24 @@ int32_t quartz_linear_ex(const quartz_encoded_t *a, const quartz_encoded_t *w,
                          const void *bias_f16, void *y, int32_t y_type, void *workspace,
                          size_t workspace_bytes, const quartz_linear_opts_t *opts, void *stream);
 
+/* Fused activation path: the W4A4 linear layer straight from fp16
+ * activations, encoding them on the fly (the "on-the-fly activation
+ * compression" of Appendix C).  One pass over x does Eq. 1 and Eq. 2 and
+ * writes the tensor-core operand directly, instead of writing the encoded
+ * activations and reading them back; results are bit-identical to
+ * quartz_quantize followed by quartz_linear with the same parameters.
+ *   x_f16      fp16 [M, K] device, 16-byte aligned
+ *   w          encoded weights [N, K]; its params (group_s, mode) are used
+ *              for the activations; SYMMETRIC mode only (else
+ *              QUARTZ_ERR_UNSUPPORTED)
+ *   bias_f16, y, y_type, workspace, workspace_bytes: as quartz_linear
+ *              (quartz_linear_workspace_size(M, N, K, &w->p) bytes)
+ *   a_out      NULL, or an encoded [M, K] tensor with w's params that also
+ *              receives the activations' encoding (codes, FLAGs, scales) */
+int32_t quartz_linear_f16(const void *x_f16, int64_t M, const quartz_encoded_t *w, const void *bias_f16,
+                          void *y, int32_t y_type, const quartz_encoded_t *a_out, void *workspace,
+                          size_t workspace_bytes, void *stream);
+
 /* Scratch-free variant of quartz_linear, for callers that cannot allocate
  * device memory (for example a plugin inside a host framework that owns all
  * device memory through its own pool and forbids side allocations, or code on

@@ -169,6 +169,33 @@ def linear(a: Encoded, w: Encoded, bias=None, out_dtype=None, out=None, workspac
     return y if part is None else (y, part)
 
 
+def linear_f16(x, w: Encoded, bias=None, out_dtype=None, out=None, workspace=None,
+               a_out: Encoded | None = None, stream=None):
+    """Fused activation path: y = linear(quantize(x), w) from fp16 x [M, K]
+    in one pass over x (the activations are encoded straight into the GEMM
+    operand; symmetric mode).  `a_out` optionally receives the encoding."""
+    torch = _torch()
+    _check_f16(x, "x")
+    out_dtype = out_dtype or torch.float16
+    M, K = x.shape
+    Nn = w.rows
+    y = out if out is not None else torch.empty((M, Nn), dtype=out_dtype, device=x.device)
+    y_type = _OUT[str(y.dtype).replace("torch.", "")]
+    if workspace is None:
+        workspace = torch.empty(max(linear_workspace_size(M, Nn, K, w.params), 16),
+                                dtype=torch.uint8, device=x.device)
+    if bias is not None and not (bias.dtype == torch.float16 and bias.is_cuda and bias.numel() == Nn):
+        raise ValueError("bias must be a float16 CUDA tensor of N elements")
+    wc = w.c()
+    ac = a_out.c() if a_out is not None else None
+    rc = N.load().quartz_linear_f16(
+        x.data_ptr(), M, C.byref(wc), None if bias is None else bias.data_ptr(), y.data_ptr(), y_type,
+        None if ac is None else C.byref(ac), workspace.data_ptr(),
+        workspace.numel() * workspace.element_size(), _stream(stream))
+    N.check(rc, "quartz_linear_f16")
+    return y
+
+
 def device_status(stream=None) -> int:
     """Synchronise the stream; return (and clear) the library's device status."""
     return int(N.load().quartz_device_status(_stream(stream)))

@@ -64,6 +64,8 @@ SIGNATURES = {
                                 _P, _SZ, C.POINTER(QuartzLinearOpts), _P]),
     "quartz_linear_noalloc": (_I32, [C.POINTER(QuartzEncoded), C.POINTER(QuartzEncoded), _P, _P,
                                      _I32, _P]),
+    "quartz_linear_f16": (_I32, [_P, _I64, C.POINTER(QuartzEncoded), _P, _P, _I32,
+                                 C.POINTER(QuartzEncoded), _P, _SZ, _P]),
     "quartz_device_status": (_I32, [_P]),
     "quartz_selftest_timeout": (_I32, [_I64, _P]),
 }

@@ -193,6 +193,46 @@ int32_t quartz_linear(const quartz_encoded_t *a, const quartz_encoded_t *w, cons
     return quartz_linear_ex(a, w, bias_f16, y, y_type, workspace, workspace_bytes, nullptr, stream);
 }
 
+int32_t quartz_linear_f16(const void *x_f16, int64_t M, const quartz_encoded_t *w, const void *bias_f16,
+                          void *y, int32_t y_type, const quartz_encoded_t *a_out, void *workspace,
+                          size_t workspace_bytes, void *stream)
+{
+    int32_t rc = check_encoded(w);
+    if (rc) return rc;
+    if (w->p.mode != QUARTZ_SYMMETRIC) return QUARTZ_ERR_UNSUPPORTED;
+    const int64_t N = w->rows, K = w->K;
+    rc = check_shape(M, K, &w->p);
+    if (rc) return rc;
+    if (N <= 0 || N % 8 != 0 || N > (int64_t(1) << 24)) return QUARTZ_ERR_INVALID_ARG;
+    if (y_type != QUARTZ_OUT_F16 && y_type != QUARTZ_OUT_BF16 && y_type != QUARTZ_OUT_F32)
+        return QUARTZ_ERR_INVALID_ARG;
+    if (a_out) {
+        rc = check_encoded(a_out);
+        if (rc) return rc;
+        if (a_out->rows != M || a_out->K != K || a_out->p.group_q != w->p.group_q ||
+            a_out->p.group_s != w->p.group_s || a_out->p.mode != w->p.mode)
+            return QUARTZ_ERR_INVALID_ARG;
+    }
+    if (M * N >= (int64_t(1) << 40)) return QUARTZ_ERR_UNSUPPORTED;
+    if (M == 0) return QUARTZ_OK;
+    if (!x_f16 || !y) return QUARTZ_ERR_INVALID_ARG;
+    if (!aligned16(x_f16) || !aligned16(y) || (bias_f16 && !aligned16(bias_f16))) return QUARTZ_ERR_ALIGNMENT;
+    const size_t need = linear_workspace_bytes(M, N, K, w->p.mode);
+    if (!workspace || workspace_bytes < need) return QUARTZ_ERR_WORKSPACE;
+    if (!aligned16(workspace)) return QUARTZ_ERR_ALIGNMENT;
+    int *dev_err = device_error_word();
+    if (!dev_err) return QUARTZ_ERR_CUDA;
+
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    LinearWorkspace ws;
+    linear_workspace_carve(workspace, M, N, K, w->p.mode, &ws);
+    cudaError_t e = launch_encode_operand(x_f16, M, K, &w->p, ws, a_out, s);
+    if (e == cudaSuccess) e = launch_prepare(nullptr, w, ws, s);
+    if (e == cudaSuccess)
+        e = launch_gemm_tcgen05(ws, M, N, K, w->p.mode, bias_f16, y, y_type, nullptr, 0, dev_err, s);
+    return map_cuda(e);
+}
+
 int32_t quartz_device_status(void *stream)
 {
     cudaStream_t s = static_cast<cudaStream_t>(stream);

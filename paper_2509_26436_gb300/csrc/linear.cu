@@ -30,6 +30,7 @@
 #include <cuda_bf16.h>
 #include <cuda_fp8.h>
 
+#include "lzs_e4m3.cuh"
 #include "ptx.cuh"
 #include "quartz_internal.h"
 
@@ -49,55 +50,6 @@ constexpr int kGroupQ = 64;
 __host__ __device__ __forceinline__ int64_t perm16(int64_t r)
 {
     return (r & ~int64_t(15)) | ((r & 3) << 2) | ((r >> 2) & 3);
-}
-
-// Byte permute (PTX prmt, default mode: a selector nibble b < 8 copies byte b
-// of {hi:lo}, b + 8 replicates that byte's sign bit).
-__device__ __forceinline__ uint32_t prmt(uint32_t lo, uint32_t hi, uint32_t sel)
-{
-    uint32_t d;
-    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(lo), "r"(hi), "r"(sel));
-    return d;
-}
-
-// Four table lookups at once: byte k of x (0..15) selects byte x_k of the
-// 16-byte table {t0, t1, t2, t3}.
-__device__ __forceinline__ uint32_t lut16(uint32_t x, uint32_t t0, uint32_t t1, uint32_t t2, uint32_t t3)
-{
-    const uint32_t y = x & 0x07070707u;
-    const uint32_t sel = prmt(y | (y >> 4), 0u, 0x0020u);  // nibble k = low 3 bits of byte k
-    const uint32_t lo = prmt(t0, t1, sel);
-    const uint32_t hi = prmt(t2, t3, sel);
-    const uint32_t use_hi = prmt(x << 4, 0u, 0xBA98u);      // 0xFF where bit 3 of byte k is set
-    return (hi & use_hi) | (lo & ~use_hi);
-}
-
-// Decode eight 4-bit codes (one 32-bit word, code k in bits 4k..4k+3) of one
-// subgroup with FLAG `flag` to E4M3 bytes of v = c * 2^flag, written to the
-// eight bytes of {lo, hi} in code order.  The E4M3 byte of a nonzero c is
-// sign | (7 + e + flag) << 3 | m for |c| = (1 + m/8) 2^e, so the table for
-// FLAG f is the FLAG-0 table with 8 f added to every nonzero entry (no carry
-// leaves a byte: the largest entry, 7 * 2^4 = 112, is 0x6E / 0xEE).
-__device__ __forceinline__ void e4m3_from_codes8(uint32_t word, int flag, uint32_t &lo, uint32_t &hi)
-{
-    const uint32_t add = (static_cast<uint32_t>(flag) << 3) * 0x01010101u;
-    // entries for codes 0..15 (two's complement -8..7; -8 never occurs)
-    const uint32_t t0 = 0x44403800u + (add & 0xFFFFFF00u);  //  0,  1,  2,  3
-    const uint32_t t1 = 0x4E4C4A48u + add;                  //  4,  5,  6,  7
-    const uint32_t t2 = 0xCACCCE00u + (add & 0xFFFFFF00u);  // -8, -7, -6, -5
-    const uint32_t t3 = 0xB8C0C4C8u + add;                  // -4, -3, -2, -1
-    const uint32_t ev = lut16(word & 0x0F0F0F0Fu, t0, t1, t2, t3);         // codes 0, 2, 4, 6
-    const uint32_t od = lut16((word >> 4) & 0x0F0F0F0Fu, t0, t1, t2, t3);  // codes 1, 3, 5, 7
-    lo = prmt(ev, od, 0x5140u);
-    hi = prmt(ev, od, 0x7362u);
-}
-
-// Position of activation row r in its group's side-value row: inside every
-// block of 32 rows, row 8a + b sits at 4b + a, so that the four rows
-// b + {0, 8, 16, 24} one epilogue thread scales are one 16-byte vector.
-__host__ __device__ __forceinline__ int64_t perm32(int64_t r)
-{
-    return (r & ~int64_t(31)) | ((r & 7) << 2) | ((r >> 3) & 3);
 }
 
 // One launch prepares both GEMM operands (jobs selected by block index):
@@ -964,20 +916,22 @@ void linear_workspace_carve(void *base, int64_t M, int64_t N, int64_t K, int mod
 cudaError_t launch_prepare(const quartz_encoded_t *a, const quartz_encoded_t *w, const LinearWorkspace &ws,
                            cudaStream_t s)
 {
-    const int64_t K = a->K;
+    const int64_t K = w->K;
     const int64_t upr = K / 16;
     PrepArgs p{};
     p.G = static_cast<int>(K / kGroupQ);
     p.nside = ws.nside;
-    p.ex_a = {reinterpret_cast<const uint2 *>(a->codes), a->flags, static_cast<uint4 *>(ws.a_op),
-              a->rows * upr, a->rows * upr, upr, 0};
+    if (a)
+        p.ex_a = {reinterpret_cast<const uint2 *>(a->codes), a->flags, static_cast<uint4 *>(ws.a_op),
+                  a->rows * upr, a->rows * upr, upr, 0};
     // the weight operand is row-permuted and padded to a multiple of 16 rows
     p.ex_w = {reinterpret_cast<const uint2 *>(w->codes), w->flags, static_cast<uint4 *>(ws.w_op),
               w->rows * upr, round_up(w->rows, 16) * upr, upr, 1};
-    p.sd_a = {reinterpret_cast<const __half *>(a->scales), a->zeros, a->gsum, ws.a_side, a->rows, ws.m_pad, 1};
+    if (a)
+        p.sd_a = {reinterpret_cast<const __half *>(a->scales), a->zeros, a->gsum, ws.a_side, a->rows, ws.m_pad, 1};
     p.sd_w = {reinterpret_cast<const __half *>(w->scales), w->zeros, w->gsum, ws.w_side, w->rows, ws.n_pad, 0};
     const int64_t side_chunks = (p.G + kSideGroupsPerThread - 1) / kSideGroupsPerThread;
-    const int64_t threads[4] = {p.ex_a.units_pad, p.ex_w.units_pad, ws.m_pad * side_chunks,
+    const int64_t threads[4] = {p.ex_a.units_pad, p.ex_w.units_pad, a ? ws.m_pad * side_chunks : 0,
                                 ws.n_pad * side_chunks};
     int64_t acc = 0;
     for (int i = 0; i < 4; ++i) {
@@ -986,7 +940,7 @@ cudaError_t launch_prepare(const quartz_encoded_t *a, const quartz_encoded_t *w,
     }
     if (acc == 0) return cudaSuccess;
     const unsigned blocks = static_cast<unsigned>(acc);
-    switch (a->p.group_s) {
+    switch (w->p.group_s) {
         case 8: prep_kernel<8><<<blocks, kPrepThreads, 0, s>>>(p); break;
         case 16: prep_kernel<16><<<blocks, kPrepThreads, 0, s>>>(p); break;
         case 32: prep_kernel<32><<<blocks, kPrepThreads, 0, s>>>(p); break;

@@ -18,6 +18,7 @@
 // with the same arithmetic written per element.
 #include <cuda_fp16.h>
 
+#include "lzs_e4m3.cuh"
 #include "quartz_internal.h"
 
 namespace quartz {
@@ -115,10 +116,17 @@ __device__ __forceinline__ int lzs_flag_of(float amax_sub, float r)
     return max(29 - __clz(qmax), 0);
 }
 
+// Eq. 1 + Eq. 2 on the 16 elements of one unit (lo, hi: eight fp16 pairs):
+// the group scale and, per 8-element half, the FLAG and the eight codes.  All
+// 32 lanes must call it together (group and subgroup maxima are shuffles).
+struct UnitCodes {
+    uint32_t c0, c1;   // codes of elements 0-7 and 8-15 (element k in bits 4k..4k+3)
+    int flag0, flag1;  // their FLAGs (equal unless G_s = 8)
+    __half s16;        // the group's fp16 scale
+};
+
 template <int GS>
-__device__ __forceinline__ void encode_unit_sym(const uint4 lo, const uint4 hi, int64_t unit, bool valid,
-                                                int lane, uint2 *__restrict__ codes,
-                                                uint8_t *__restrict__ flags, __half *__restrict__ scales)
+__device__ __forceinline__ UnitCodes encode_unit_sym(const uint4 lo, const uint4 hi)
 {
     const uint32_t w[8] = {lo.x, lo.y, lo.z, lo.w, hi.x, hi.y, hi.z, hi.w};
     uint32_t a[8];
@@ -136,37 +144,44 @@ __device__ __forceinline__ void encode_unit_sym(const uint4 lo, const uint4 hi, 
     const float amax = fmaxf(pair_max, __shfl_xor_sync(0xffffffffu, pair_max, 2));
 
     // --- Eq. 1: scale and reciprocal (as the per-element path) ------------
-    const __half s16 = __float2half_rn(__fdiv_rn(amax, 127.0f));
-    const float s = __half2float(s16);
+    UnitCodes u;
+    u.s16 = __float2half_rn(__fdiv_rn(amax, 127.0f));
+    const float s = __half2float(u.s16);
     const float r = (s > 0.f) ? __frcp_rn(s) : 0.f;
 
     // --- Eq. 2: FLAG of each subgroup from its maximum --------------------
-    int flag0, flag1;
     if (GS == 8) {
-        flag0 = lzs_flag_of(sub0, r);
-        flag1 = lzs_flag_of(sub1, r);
+        u.flag0 = lzs_flag_of(sub0, r);
+        u.flag1 = lzs_flag_of(sub1, r);
     } else {
         const float m = GS == 16 ? unit_max : GS == 32 ? pair_max : amax;
-        flag0 = flag1 = lzs_flag_of(m, r);
+        u.flag0 = u.flag1 = lzs_flag_of(m, r);
     }
-    uint32_t c0, c1;
     if (__float2int_rn(__fmul_rn(amax, r)) > 127) {  // only when the fp16 scale rounded far down
-        c0 = lzs_word8<true>(w, a, r, flag0);
-        c1 = lzs_word8<true>(w + 4, a + 4, r, flag1);
+        u.c0 = lzs_word8<true>(w, a, r, u.flag0);
+        u.c1 = lzs_word8<true>(w + 4, a + 4, r, u.flag1);
     } else {
-        c0 = lzs_word8<false>(w, a, r, flag0);
-        c1 = lzs_word8<false>(w + 4, a + 4, r, flag1);
+        u.c0 = lzs_word8<false>(w, a, r, u.flag0);
+        u.c1 = lzs_word8<false>(w + 4, a + 4, r, u.flag1);
     }
-    if (!valid) return;
-    codes[unit] = make_uint2(c0, c1);
+    return u;
+}
+
+// Store one unit's encoding: codes, FLAG byte(s), and the scale once per group.
+template <int GS>
+__device__ __forceinline__ void store_unit_sym(const UnitCodes &u, int64_t unit, int lane,
+                                               uint2 *__restrict__ codes, uint8_t *__restrict__ flags,
+                                               __half *__restrict__ scales)
+{
+    codes[unit] = make_uint2(u.c0, u.c1);
     if (GS == 8) {
-        reinterpret_cast<uint16_t *>(flags)[unit] = static_cast<uint16_t>(flag0 | (flag1 << 8));
+        reinterpret_cast<uint16_t *>(flags)[unit] = static_cast<uint16_t>(u.flag0 | (u.flag1 << 8));
     } else if (GS == 16) {
-        flags[unit] = static_cast<uint8_t>(flag0);
+        flags[unit] = static_cast<uint8_t>(u.flag0);
     } else if ((lane & (GS / 16 - 1)) == 0) {
-        flags[unit / (GS / 16)] = static_cast<uint8_t>(flag0);
+        flags[unit / (GS / 16)] = static_cast<uint8_t>(u.flag0);
     }
-    if ((lane & 3) == 0) scales[unit >> 2] = s16;
+    if ((lane & 3) == 0) scales[unit >> 2] = u.s16;
 }
 
 template <int GS>
@@ -188,7 +203,48 @@ __global__ void __launch_bounds__(kThreads) quantize_sym_kernel(const uint4 *__r
 #pragma unroll
     for (int j = 0; j < kUnitsPerThread; ++j) {
         const int64_t u = base + j * kThreads;
-        encode_unit_sym<GS>(raw[j][0], raw[j][1], u, u < n_units, lane, codes, flags, scales);
+        const UnitCodes c = encode_unit_sym<GS>(raw[j][0], raw[j][1]);
+        if (u < n_units) store_unit_sym<GS>(c, u, lane, codes, flags, scales);
+    }
+}
+
+// Fused activation path of the linear layer: the same encoding, decoded at
+// once to the GEMM's E4M3 operand (16 bytes per unit, row-major) and its
+// scale side values (fp32, [G][m_pad], rows at perm32(r)); units of the
+// padding rows [M, m_pad) write zero scales.  When `codes` is not NULL the
+// encoded tensor is stored as well.
+template <int GS>
+__global__ void __launch_bounds__(kThreads) encode_operand_kernel(
+    const uint4 *__restrict__ x, int64_t n_units, int64_t n_units_pad, int64_t units_per_row, int64_t m_pad,
+    uint4 *__restrict__ a_op, float *__restrict__ a_side, uint2 *__restrict__ codes,
+    uint8_t *__restrict__ flags, __half *__restrict__ scales)
+{
+    const int lane = threadIdx.x & 31;
+    const int64_t base = static_cast<int64_t>(blockIdx.x) * (kThreads * kUnitsPerThread) + threadIdx.x;
+    uint4 raw[kUnitsPerThread][2];
+#pragma unroll
+    for (int j = 0; j < kUnitsPerThread; ++j) {
+        const int64_t u = base + j * kThreads;
+        const bool in = u < n_units;
+        raw[j][0] = in ? ldg_stream(x + 2 * u) : make_uint4(0, 0, 0, 0);
+        raw[j][1] = in ? ldg_stream(x + 2 * u + 1) : make_uint4(0, 0, 0, 0);
+    }
+#pragma unroll
+    for (int j = 0; j < kUnitsPerThread; ++j) {
+        const int64_t u = base + j * kThreads;
+        const UnitCodes c = encode_unit_sym<GS>(raw[j][0], raw[j][1]);
+        if (u >= n_units_pad) continue;
+        const int64_t row = u / units_per_row;
+        if ((lane & 3) == 0) {
+            const int64_t g = (u - row * units_per_row) >> 2;
+            a_side[g * m_pad + perm32(row)] = u < n_units ? __half2float(c.s16) : 0.f;
+        }
+        if (u >= n_units) continue;
+        uint4 o;
+        e4m3_from_codes8(c.c0, c.flag0, o.x, o.y);
+        e4m3_from_codes8(c.c1, c.flag1, o.z, o.w);
+        a_op[u] = o;
+        if (codes) store_unit_sym<GS>(c, u, lane, codes, flags, scales);
     }
 }
 
@@ -383,6 +439,28 @@ cudaError_t launch_quantize(const void *x, const quartz_encoded_t *out, cudaStre
     if (out->rows == 0) return cudaSuccess;
     return out->p.mode == QUARTZ_SYMMETRIC ? launch_q_mode<QUARTZ_SYMMETRIC>(x, out, s)
                                            : launch_q_mode<QUARTZ_ASYMMETRIC>(x, out, s);
+}
+
+cudaError_t launch_encode_operand(const void *x, int64_t M, int64_t K, const quartz_params_t *p,
+                                  const LinearWorkspace &ws, const quartz_encoded_t *enc, cudaStream_t s)
+{
+    const int64_t upr = K / 16;
+    const int64_t n_units = M * upr;
+    const int64_t n_units_pad = ws.m_pad * upr;
+    const int64_t per_block = kThreads * kUnitsPerThread;
+    const unsigned blocks = static_cast<unsigned>((n_units_pad + per_block - 1) / per_block);
+    const uint4 *xv = static_cast<const uint4 *>(x);
+    uint4 *op = static_cast<uint4 *>(ws.a_op);
+    uint2 *codes = enc ? reinterpret_cast<uint2 *>(enc->codes) : nullptr;
+    uint8_t *flags = enc ? enc->flags : nullptr;
+    __half *scales = enc ? reinterpret_cast<__half *>(enc->scales) : nullptr;
+    switch (p->group_s) {
+        case 8: encode_operand_kernel<8><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales); break;
+        case 16: encode_operand_kernel<16><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales); break;
+        case 32: encode_operand_kernel<32><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales); break;
+        default: encode_operand_kernel<64><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales); break;
+    }
+    return cudaGetLastError();
 }
 
 cudaError_t launch_dequantize(const quartz_encoded_t *e, void *y, cudaStream_t s)

@@ -25,6 +25,14 @@ int *device_error_word();
 cudaError_t launch_quantize(const void *x, const quartz_encoded_t *out, cudaStream_t s);
 cudaError_t launch_dequantize(const quartz_encoded_t *e, void *y, cudaStream_t s);
 
+// Position of activation row r in its group's side-value row: inside every
+// block of 32 rows, row 8a + b sits at 4b + a, so that the four rows
+// b + {0, 8, 16, 24} one epilogue thread scales are one 16-byte vector.
+__host__ __device__ __forceinline__ int64_t perm32(int64_t r)
+{
+    return (r & ~int64_t(31)) | ((r & 7) << 2) | ((r >> 3) & 3);
+}
+
 // Linear-layer workspace and launches (linear.cu).
 struct LinearWorkspace {
     void *a_op;      // E4M3 [M, K]  decoded activations
@@ -37,10 +45,16 @@ struct LinearWorkspace {
 size_t linear_workspace_bytes(int64_t M, int64_t N, int64_t K, int mode);
 void linear_workspace_carve(void *base, int64_t M, int64_t N, int64_t K, int mode,
                             LinearWorkspace *ws);
-// Expands both operands to E4M3 and transposes their scales into the
-// workspace (one launch).
+// Expands the operands to E4M3 and transposes their scales into the
+// workspace (one launch).  `a` may be NULL: then only the weight operand is
+// prepared (the fused encoder below has written the activation side).
 cudaError_t launch_prepare(const quartz_encoded_t *a, const quartz_encoded_t *w, const LinearWorkspace &ws,
                            cudaStream_t s);
+// Fused activation path (quantize.cu, symmetric mode): Eq. 1 + Eq. 2 on fp16
+// x [M, K] written straight into the workspace as E4M3 operand and scale
+// side values; `enc` (may be NULL) also receives the encoded tensor.
+cudaError_t launch_encode_operand(const void *x, int64_t M, int64_t K, const quartz_params_t *p,
+                                  const LinearWorkspace &ws, const quartz_encoded_t *enc, cudaStream_t s);
 cudaError_t launch_gemm_tcgen05(const LinearWorkspace &ws, int64_t M, int64_t N, int64_t K,
                                 int mode, const void *bias, void *y, int y_type,
                                 int32_t *partials, int partials_group, int *dev_err,

@@ -111,6 +111,28 @@ def test_linear_validation(lib):
     assert lib.quartz_selftest_timeout(10, None) == N.QUARTZ_ERR_INVALID_ARG
 
 
+def test_linear_f16_validation(lib):
+    """Host checks of the fused activation path: nothing is launched on error."""
+    L = lib.quartz_linear_f16
+    w = _enc(24, 128)
+    ok = dict(x=0x1000, M=16, bias=None, y=0x2000, t=0, aout=None, ws=0x3000, wsb=1 << 30)
+
+    def call(w, **kw):
+        d = dict(ok, **kw)
+        return L(d["x"], d["M"], C.byref(w), d["bias"], d["y"], d["t"], d["aout"], d["ws"], d["wsb"], None)
+
+    assert call(_enc(24, 128, mode=1)) == N.QUARTZ_ERR_UNSUPPORTED      # asymmetric not fused
+    assert call(_enc(20, 128)) == N.QUARTZ_ERR_INVALID_ARG             # N % 8 != 0
+    assert call(w, M=-1) == N.QUARTZ_ERR_INVALID_ARG
+    assert call(w, t=3) == N.QUARTZ_ERR_INVALID_ARG
+    assert call(w, x=0x1008) == N.QUARTZ_ERR_ALIGNMENT
+    assert call(w, x=None) == N.QUARTZ_ERR_INVALID_ARG
+    assert call(w, wsb=16) == N.QUARTZ_ERR_WORKSPACE
+    assert call(w, aout=C.byref(_enc(8, 128))) == N.QUARTZ_ERR_INVALID_ARG       # rows != M
+    assert call(w, aout=C.byref(_enc(16, 128, gs=32))) == N.QUARTZ_ERR_INVALID_ARG
+    assert call(w, M=0, x=None, y=None) == N.QUARTZ_OK                   # empty: no-op
+
+
 def test_missing_library_fails_loudly(tmp_path):
     saved = N._lib
     try:

@@ -214,3 +214,40 @@ def test_group_partials_lzs_extremes_bit_exact(Q, seed):
         assert np.array_equal(part.cpu().numpy().astype(np.int64), ref), f"group {g}"
     ref, rabs = O.linear(ea, ew, with_abs=True)
     _tol_check(y.cpu().numpy(), ref, rabs, K // 64, "float32")
+
+
+@pytest.mark.parametrize("gs", [8, 16, 32, 64])
+@pytest.mark.parametrize("M,N,K", [(200, 264, 640), (1, 8, 64), (300, 1024, 1216)])
+def test_linear_f16_fused_is_bit_identical(Q, gs, M, N, K):
+    """quartz_linear_f16 (encode on the fly into the GEMM operand) gives the
+    same bits as quartz_quantize + quartz_linear, and its optional encoded
+    output equals quartz_quantize's."""
+    x16 = inputs.mixture_activations(M, K, seed=M + 3 * N + gs)
+    w16 = inputs.gaussian_weights(N, K, seed=N + gs)
+    x = torch.from_numpy(x16).cuda()
+    w = Q.encode_weights(torch.from_numpy(w16).cuda(), group_s=gs)
+    bias = torch.from_numpy(inputs.gaussian_weights(1, N, seed=5)[0]).cuda()
+    a = Q.quantize(x, group_s=gs)
+    for dt in (torch.float16, torch.float32):
+        ref = Q.linear(a, w, bias, out_dtype=dt)
+        a_out = Q.empty_encoded(M, K, Q.Params(64, gs, O.SYMMETRIC), x.device)
+        y = Q.linear_f16(x, w, bias, out_dtype=dt, a_out=a_out)
+        assert Q.device_status() == 0
+        assert torch.equal(y, ref)
+        assert torch.equal(a_out.codes, a.codes) and torch.equal(a_out.flags, a.flags)
+        assert torch.equal(a_out.scales.view(torch.int16), a.scales.view(torch.int16))
+    # and against the oracle directly (same tolerance as the other linear tests)
+    ref, rabs = O.linear(O.encode(x16, 64, gs), O.encode(w16, 64, gs), bias.cpu().numpy(), with_abs=True)
+    y = Q.linear_f16(x, w, bias, out_dtype=torch.float32)
+    _tol_check(y.cpu().numpy(), ref, rabs, K // 64, "float32")
+
+
+def test_linear_f16_flux_layer_matches_two_call_path(Q):
+    """Full-size FLUX fc1 activations, fused path vs quantize + linear."""
+    layer = [l for l in inputs.CONFIG4 if l.name == "flux_fc1"][0]
+    x = torch.from_numpy(layer.activations()).cuda()
+    w = Q.encode_weights(torch.from_numpy(layer.weights()).cuda(), group_s=16)
+    ref = Q.linear(Q.quantize(x, group_s=16), w)
+    y = Q.linear_f16(x, w)
+    assert Q.device_status() == 0
+    assert torch.equal(y, ref)
