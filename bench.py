@@ -45,6 +45,8 @@ def parse():
     p.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
     p.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline leg")
     p.add_argument("--no-fused", action="store_true", help="skip the fused activation-path leg")
+    p.add_argument("--compare-algos", action="store_true",
+                   help="also time the three GEMM algorithms (tcgen05, simt, shift) on each layer")
     p.add_argument("--layers", default="", help="comma-separated subset of layer names (profiling)")
     return p.parse_args()
 
@@ -366,6 +368,24 @@ def run_ours(args):
                  "path": "quartz_linear_f16 per layer (activations encoded straight into the GEMM "
                          "operand; bit-identical to quantize + linear)"}
 
+    # ---- GEMM algorithms side by side (optional) ----------------------------
+    algos = None
+    if args.compare_algos:
+        algos = {}
+        for name, algo in (("tcgen05", Q.ALGO_TCGEN05), ("simt", Q.ALGO_SIMT), ("shift", Q.ALGO_SHIFT)):
+            per = []
+            for i in range(nl):
+                Q.quantize(x_dev[i], out=enc_a[i], group_s=GROUP_S)
+                Q.linear(enc_a[i], enc_w[i], out=y_dev[i], workspace=workspace, algo=algo)
+                evs = [(ev(), ev()) for _ in range(3)]
+                for e in evs:
+                    Q.linear(enc_a[i], enc_w[i], out=y_dev[i], workspace=workspace, algo=algo, gemm_events=e)
+                torch.cuda.synchronize()
+                ms = statistics.median(e[0].elapsed_time(e[1]) for e in evs)
+                per.append({"layer": layers[i].name, "ms": ms, "TOPS": layers[i].ops / ms / 1e9})
+            algos[name] = per
+        assert Q.device_status() == 0
+
     # ---- end to end through the public API with host buffers ---------------
     # Each (step, layer) unit copies its activations from pinned host memory,
     # encodes them, runs the linear layer and copies the fp16 output back to
@@ -467,6 +487,7 @@ def run_ours(args):
         "clocks": clocks,
         "gpu_launches": launches_per_step * args.steps,
         "fused": fused,
+        "gemm_algos": algos,
         "e2e": e2e,
         "cpu_baseline": cpu,
     }

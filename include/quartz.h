@@ -56,9 +56,13 @@ typedef enum { QUARTZ_SYMMETRIC = 0, QUARTZ_ASYMMETRIC = 1 } quartz_mode_t;
 typedef enum { QUARTZ_OUT_F16 = 0, QUARTZ_OUT_BF16 = 1, QUARTZ_OUT_F32 = 2 } quartz_out_t;
 
 /* GEMM implementations behind quartz_linear_ex.  TCGEN05 is the product
- * path (tcgen05 tensor cores, TMEM accumulators); SIMT is a plain CUDA-core
- * kernel with the same arithmetic, kept as a second on-device path. */
-typedef enum { QUARTZ_ALGO_TCGEN05 = 0, QUARTZ_ALGO_SIMT = 1 } quartz_algo_t;
+ * path (tcgen05 tensor cores, TMEM accumulators, operands decoded first);
+ * SIMT is a plain CUDA-core kernel with the same arithmetic, kept as a second
+ * on-device path; SHIFT is the paper's own schedule (Section 4.4): integer
+ * dot products of the packed 4-bit codes per subgroup, each shifted by the
+ * two operands' FLAGs, with no decoded operand (CUDA cores, dp4a).  All three
+ * give the same exact group partials P_g. */
+typedef enum { QUARTZ_ALGO_TCGEN05 = 0, QUARTZ_ALGO_SIMT = 1, QUARTZ_ALGO_SHIFT = 2 } quartz_algo_t;
 
 typedef struct {
     int32_t group_q; /* min-max quantization group along K; 64 (Appendix C) */

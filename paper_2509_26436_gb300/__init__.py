@@ -18,7 +18,7 @@ import ctypes as C
 from dataclasses import dataclass
 
 from . import _native as N
-from ._native import (ALGO_SIMT, ALGO_TCGEN05, ASYMMETRIC, OUT_BF16, OUT_F16, OUT_F32,  # noqa: F401
+from ._native import (ALGO_SHIFT, ALGO_SIMT, ALGO_TCGEN05, ASYMMETRIC, OUT_BF16, OUT_F16, OUT_F32,  # noqa: F401
                       SYMMETRIC, QuartzError)
 
 __all__ = ["Params", "Encoded", "quantize", "encode_weights", "dequantize", "linear",

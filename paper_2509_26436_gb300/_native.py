@@ -28,6 +28,7 @@ OUT_F32 = 2
 
 ALGO_TCGEN05 = 0
 ALGO_SIMT = 1
+ALGO_SHIFT = 2
 
 # every symbol the header declares, with (restype, argtypes)
 _P = C.c_void_p

@@ -155,7 +155,8 @@ int32_t quartz_linear_ex(const quartz_encoded_t *a, const quartz_encoded_t *w,
     if (N <= 0 || N % 8 != 0 || N > (int64_t(1) << 24)) return QUARTZ_ERR_INVALID_ARG;
     if (y_type != QUARTZ_OUT_F16 && y_type != QUARTZ_OUT_BF16 && y_type != QUARTZ_OUT_F32)
         return QUARTZ_ERR_INVALID_ARG;
-    if (algo != QUARTZ_ALGO_TCGEN05 && algo != QUARTZ_ALGO_SIMT) return QUARTZ_ERR_INVALID_ARG;
+    if (algo != QUARTZ_ALGO_TCGEN05 && algo != QUARTZ_ALGO_SIMT && algo != QUARTZ_ALGO_SHIFT)
+        return QUARTZ_ERR_INVALID_ARG;
     if (partials && (partials_group < 0 || partials_group >= K / a->p.group_q))
         return QUARTZ_ERR_INVALID_ARG;
     if (M * N >= (int64_t(1) << 40)) return QUARTZ_ERR_UNSUPPORTED;
@@ -172,12 +173,14 @@ int32_t quartz_linear_ex(const quartz_encoded_t *a, const quartz_encoded_t *w,
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     LinearWorkspace ws;
     linear_workspace_carve(workspace, M, N, K, a->p.mode, &ws);
-    cudaError_t e = launch_prepare(a, w, ws, s);
+    cudaError_t e = launch_prepare(a, w, ws, s, algo != QUARTZ_ALGO_SHIFT);
     if (e != cudaSuccess) return QUARTZ_ERR_CUDA;
     if (o.gemm_event_begin && cudaEventRecord(static_cast<cudaEvent_t>(o.gemm_event_begin), s) != cudaSuccess)
         return QUARTZ_ERR_CUDA;
     if (algo == QUARTZ_ALGO_SIMT)
         e = launch_gemm_simt(ws, M, N, K, a->p.mode, bias_f16, y, y_type, partials, partials_group, s);
+    else if (algo == QUARTZ_ALGO_SHIFT)
+        e = launch_gemm_shift(ws, a, w, bias_f16, y, y_type, partials, partials_group, s);
     else
         e = launch_gemm_tcgen05(ws, M, N, K, a->p.mode, bias_f16, y, y_type, partials,
                                 partials_group, dev_err, s);

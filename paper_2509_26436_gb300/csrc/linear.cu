@@ -766,6 +766,111 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const __nv_fp8_e4m3 *__r
 }
 
 // ---------------------------------------------------------------------------
+// 4. Accumulator-shift GEMM (the paper's own schedule, Section 4.4): works on
+//    the packed 4-bit codes and FLAGs directly, with no decoded operand.  Per
+//    subgroup j of G_s elements it forms the integer dot product of the codes
+//    and shifts it by the two FLAGs: P_g = sum_j (sum_{k in j} c_a c_w)
+//    << (F_a[j] + F_w[j]), which equals sum_k v_a v_w exactly.  The dot
+//    products run on dp4a over the codes placed in the high nibble of each
+//    byte (int8 value 16c, so a dot product is 256 x the code dot product).
+//    The dequant arithmetic is the SIMT kernel's.  64x64 output tile per
+//    256-thread block, 4x4 outputs per thread.
+// ---------------------------------------------------------------------------
+template <int GS, int MODE, int OUT>
+__global__ void __launch_bounds__(256) gemm_shift_kernel(const uint32_t *__restrict__ a_codes,
+                                                         const uint8_t *__restrict__ a_flags,
+                                                         const uint32_t *__restrict__ w_codes,
+                                                         const uint8_t *__restrict__ w_flags,
+                                                         const GemmArgs args, int K)
+{
+    constexpr int kSub = kGroupQ / GS;            // subgroups per group
+    constexpr int kWordsPerSub = GS / 4;          // int8x4 words per subgroup
+    __shared__ uint32_t sa[64][2 * kGroupQ / 8 + 1];
+    __shared__ uint32_t sw[64][2 * kGroupQ / 8 + 1];
+    __shared__ uint8_t fa[64][kSub];
+    __shared__ uint8_t fw[64][kSub];
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+    const int m0 = blockIdx.y * 64, n0 = blockIdx.x * 64;
+    const int64_t words_per_row = K / 8, flags_per_row = K / GS;
+    float y[4][4] = {};
+    const int64_t a_plane = args.m_pad * args.G;
+    const int64_t w_plane = args.n_pad * args.G;
+    for (int g = 0; g < args.G; ++g) {
+        for (int i = threadIdx.x; i < 64 * (kGroupQ / 8); i += 256) {
+            const int r = i / (kGroupQ / 8), wi = i % (kGroupQ / 8);
+            const int64_t col = static_cast<int64_t>(g) * (kGroupQ / 8) + wi;
+            const uint32_t ca = (m0 + r < args.M) ? a_codes[(m0 + r) * words_per_row + col] : 0u;
+            const uint32_t cw = (n0 + r < args.N) ? w_codes[(n0 + r) * words_per_row + col] : 0u;
+            sa[r][2 * wi] = (ca << 4) & 0xF0F0F0F0u;  // even codes, as 16c
+            sa[r][2 * wi + 1] = ca & 0xF0F0F0F0u;     // odd codes, as 16c
+            sw[r][2 * wi] = (cw << 4) & 0xF0F0F0F0u;
+            sw[r][2 * wi + 1] = cw & 0xF0F0F0F0u;
+        }
+        for (int i = threadIdx.x; i < 64 * kSub; i += 256) {
+            const int r = i / kSub, j = i % kSub;
+            const int64_t col = static_cast<int64_t>(g) * kSub + j;
+            fa[r][j] = (m0 + r < args.M) ? a_flags[(m0 + r) * flags_per_row + col] : 0;
+            fw[r][j] = (n0 + r < args.N) ? w_flags[(n0 + r) * flags_per_row + col] : 0;
+        }
+        __syncthreads();
+        int p[4][4] = {};
+#pragma unroll
+        for (int j = 0; j < kSub; ++j) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                for (int jj = 0; jj < 4; ++jj) {
+                    int dot = 0;
+#pragma unroll
+                    for (int q = 0; q < kWordsPerSub; ++q)
+                        dot = __dp4a(static_cast<int>(sa[ty * 4 + i][j * kWordsPerSub + q]),
+                                     static_cast<int>(sw[tx * 4 + jj][j * kWordsPerSub + q]), dot);
+                    p[i][jj] += (dot >> 8) * (1 << (fa[ty * 4 + i][j] + fw[tx * 4 + jj][j]));
+                }
+        }
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int m = m0 + ty * 4 + i;
+            if (m >= args.M) continue;
+            const float s_a = args.a_side[static_cast<int64_t>(g) * args.m_pad + perm32(m)];
+#pragma unroll
+            for (int jj = 0; jj < 4; ++jj) {
+                const int n = n0 + tx * 4 + jj;
+                if (n >= args.N) continue;
+                float P = static_cast<float>(p[i][jj]);
+                if (args.partials && g == args.partials_group) args.partials[(int64_t)m * args.N + n] = p[i][jj];
+                if (MODE == QUARTZ_ASYMMETRIC) {
+                    const float za = args.a_side[a_plane + (int64_t)g * args.m_pad + perm32(m)];
+                    const float ua = args.a_side[2 * a_plane + (int64_t)g * args.m_pad + perm32(m)];
+                    const float zw = args.w_side[w_plane + (int64_t)g * args.n_pad + n];
+                    const float gw = args.w_side[2 * w_plane + (int64_t)g * args.n_pad + n];
+                    P = __fmaf_rn(zw, ua, P);
+                    P = __fmaf_rn(-za, gw, P);
+                }
+                const float t = __fmul_rn(P, args.w_side[static_cast<int64_t>(g) * args.n_pad + n]);
+                y[i][jj] = __fmaf_rn(t, s_a, y[i][jj]);
+            }
+        }
+        __syncthreads();
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int m = m0 + ty * 4 + i;
+#pragma unroll
+        for (int jj = 0; jj < 4; ++jj) {
+            const int n = n0 + tx * 4 + jj;
+            if (m >= args.M || n >= args.N) continue;
+            float v = y[i][jj];
+            if (args.bias) v = __fadd_rn(v, __half2float(args.bias[n]));
+            const int64_t off = (int64_t)m * args.N + n;
+            if (OUT == QUARTZ_OUT_F16) static_cast<__half *>(args.y)[off] = __float2half_rn(v);
+            else if (OUT == QUARTZ_OUT_BF16) static_cast<__nv_bfloat16 *>(args.y)[off] = __float2bfloat16_rn(v);
+            else static_cast<float *>(args.y)[off] = v;
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
 int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
@@ -914,7 +1019,7 @@ void linear_workspace_carve(void *base, int64_t M, int64_t N, int64_t K, int mod
 }
 
 cudaError_t launch_prepare(const quartz_encoded_t *a, const quartz_encoded_t *w, const LinearWorkspace &ws,
-                           cudaStream_t s)
+                           cudaStream_t s, bool expand)
 {
     const int64_t K = w->K;
     const int64_t upr = K / 16;
@@ -931,8 +1036,8 @@ cudaError_t launch_prepare(const quartz_encoded_t *a, const quartz_encoded_t *w,
         p.sd_a = {reinterpret_cast<const __half *>(a->scales), a->zeros, a->gsum, ws.a_side, a->rows, ws.m_pad, 1};
     p.sd_w = {reinterpret_cast<const __half *>(w->scales), w->zeros, w->gsum, ws.w_side, w->rows, ws.n_pad, 0};
     const int64_t side_chunks = (p.G + kSideGroupsPerThread - 1) / kSideGroupsPerThread;
-    const int64_t threads[4] = {p.ex_a.units_pad, p.ex_w.units_pad, a ? ws.m_pad * side_chunks : 0,
-                                ws.n_pad * side_chunks};
+    const int64_t threads[4] = {expand ? p.ex_a.units_pad : 0, expand ? p.ex_w.units_pad : 0,
+                                a ? ws.m_pad * side_chunks : 0, ws.n_pad * side_chunks};
     int64_t acc = 0;
     for (int i = 0; i < 4; ++i) {
         acc += (threads[i] + kPrepThreads - 1) / kPrepThreads;
@@ -972,6 +1077,53 @@ cudaError_t launch_gemm_simt(const LinearWorkspace &ws, int64_t M, int64_t N, in
     return mode == QUARTZ_ASYMMETRIC
                ? launch_simt_out<QUARTZ_ASYMMETRIC>(ws, args, static_cast<int>(K), y_type, s)
                : launch_simt_out<QUARTZ_SYMMETRIC>(ws, args, static_cast<int>(K), y_type, s);
+}
+
+namespace {
+template <int GS, int MODE, int OUT>
+cudaError_t launch_shift(const quartz_encoded_t *a, const quartz_encoded_t *w, const GemmArgs &args,
+                         cudaStream_t s)
+{
+    dim3 grid(static_cast<unsigned>((args.N + 63) / 64), static_cast<unsigned>((args.M + 63) / 64));
+    gemm_shift_kernel<GS, MODE, OUT><<<grid, 256, 0, s>>>(
+        reinterpret_cast<const uint32_t *>(a->codes), a->flags, reinterpret_cast<const uint32_t *>(w->codes),
+        w->flags, args, static_cast<int>(a->K));
+    return cudaGetLastError();
+}
+
+template <int GS, int MODE>
+cudaError_t launch_shift_out(const quartz_encoded_t *a, const quartz_encoded_t *w, const GemmArgs &args,
+                             int y_type, cudaStream_t s)
+{
+    switch (y_type) {
+        case QUARTZ_OUT_F16: return launch_shift<GS, MODE, QUARTZ_OUT_F16>(a, w, args, s);
+        case QUARTZ_OUT_BF16: return launch_shift<GS, MODE, QUARTZ_OUT_BF16>(a, w, args, s);
+        default: return launch_shift<GS, MODE, QUARTZ_OUT_F32>(a, w, args, s);
+    }
+}
+
+template <int GS>
+cudaError_t launch_shift_mode(const quartz_encoded_t *a, const quartz_encoded_t *w, const GemmArgs &args,
+                              int y_type, cudaStream_t s)
+{
+    return a->p.mode == QUARTZ_ASYMMETRIC ? launch_shift_out<GS, QUARTZ_ASYMMETRIC>(a, w, args, y_type, s)
+                                          : launch_shift_out<GS, QUARTZ_SYMMETRIC>(a, w, args, y_type, s);
+}
+}  // namespace
+
+cudaError_t launch_gemm_shift(const LinearWorkspace &ws, const quartz_encoded_t *a, const quartz_encoded_t *w,
+                              const void *bias, void *y, int y_type, int32_t *partials, int partials_group,
+                              cudaStream_t s)
+{
+    const int64_t M = a->rows, N = w->rows, K = a->K;
+    if (M == 0) return cudaSuccess;
+    const GemmArgs args = make_args(ws, M, N, K, bias, y, y_type, partials, partials_group, nullptr);
+    switch (a->p.group_s) {
+        case 8: return launch_shift_mode<8>(a, w, args, y_type, s);
+        case 16: return launch_shift_mode<16>(a, w, args, y_type, s);
+        case 32: return launch_shift_mode<32>(a, w, args, y_type, s);
+        default: return launch_shift_mode<64>(a, w, args, y_type, s);
+    }
 }
 
 // ---------------------------------------------------------------------------

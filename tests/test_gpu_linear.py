@@ -51,28 +51,29 @@ def _run(Q, xa, xw, gs, mode, bias=None, out_dtype="float16", algo=None, partial
     return r
 
 
-@pytest.mark.parametrize("algo", ["tcgen05", "simt"])
+ALGOS = {"tcgen05": 0, "simt": 1, "shift": 2}
+
+
+@pytest.mark.parametrize("algo", list(ALGOS))
 @pytest.mark.parametrize("out_dtype", ["float16", "bfloat16", "float32"])
 def test_linear_single_layer(Q, algo, out_dtype):
     """256 tokens x 1152 -> 1152, G_s = 16, symmetric, with bias."""
     layer = inputs.CONFIG0[0]
     xa, xw = layer.activations(), layer.weights()
     bias = inputs.gaussian_weights(1, layer.N, seed=3)[0]
-    alg = Q.ALGO_TCGEN05 if algo == "tcgen05" else Q.ALGO_SIMT
-    y = _run(Q, xa, xw, 16, O.SYMMETRIC, bias, out_dtype, alg)
+    y = _run(Q, xa, xw, 16, O.SYMMETRIC, bias, out_dtype, ALGOS[algo])
     a, w = O.encode(xa, 64, 16), O.encode(xw, 64, 16)
     ref, rabs = O.linear(a, w, bias, with_abs=True)
     _tol_check(y.float().cpu().numpy(), ref, rabs, layer.K // 64, out_dtype)
 
 
-@pytest.mark.parametrize("algo", ["tcgen05", "simt"])
+@pytest.mark.parametrize("algo", list(ALGOS))
 @pytest.mark.parametrize("group", [0, 9, 17])
 def test_group_partials_bit_exact(Q, algo, group):
     """The integer MMA result of one group equals the oracle's int64 sum."""
     layer = inputs.CONFIG0[0]
     xa, xw = layer.activations(), layer.weights()
-    alg = Q.ALGO_TCGEN05 if algo == "tcgen05" else Q.ALGO_SIMT
-    _, part = _run(Q, xa, xw, 16, O.SYMMETRIC, algo=alg, partials_group=group)
+    _, part = _run(Q, xa, xw, 16, O.SYMMETRIC, algo=ALGOS[algo], partials_group=group)
     va = O.decode_values(O.encode(xa, 64, 16))[:, group * 64:(group + 1) * 64]
     vw = O.decode_values(O.encode(xw, 64, 16))[:, group * 64:(group + 1) * 64]
     ref = O.group_partials(va, vw, 64)[0]
@@ -251,3 +252,38 @@ def test_linear_f16_flux_layer_matches_two_call_path(Q):
     y = Q.linear_f16(x, w)
     assert Q.device_status() == 0
     assert torch.equal(y, ref)
+
+
+@pytest.mark.parametrize("mode", [O.SYMMETRIC, O.ASYMMETRIC])
+@pytest.mark.parametrize("gs", [8, 16, 32, 64])
+@pytest.mark.parametrize("M,N,K", [(1, 8, 64), (200, 264, 640), (129, 520, 1216)])
+def test_shift_schedule_matches_decode_before_mma(Q, mode, gs, M, N, K):
+    """The paper's accumulator-shift schedule (integer code dot products per
+    subgroup, shifted by both FLAGs) gives the same exact group partials as
+    decode-before-MMA on the tensor cores, and outputs within tolerance."""
+    xa = inputs.mixture_activations(M, K, seed=7 * M + K + gs)
+    xw = inputs.gaussian_weights(N, K, seed=N + K + gs)
+    g = (K // 64) // 2
+    y_s, p_s = _run(Q, xa, xw, gs, mode, None, "float32", Q.ALGO_SHIFT, partials_group=g)
+    y_t, p_t = _run(Q, xa, xw, gs, mode, None, "float32", Q.ALGO_TCGEN05, partials_group=g)
+    assert torch.equal(p_s, p_t)
+    a, w = O.encode(xa, 64, gs, mode), O.encode(xw, 64, gs, mode)
+    ref, rabs = O.linear(a, w, with_abs=True)
+    _tol_check(y_s.cpu().numpy(), ref, rabs, K // 64, "float32")
+    va = O.decode_values(a)[:, g * 64:(g + 1) * 64]
+    vw = O.decode_values(w)[:, g * 64:(g + 1) * 64]
+    assert np.array_equal(p_s.cpu().numpy().astype(np.int64), O.group_partials(va, vw, 64)[0])
+
+
+@pytest.mark.parametrize("seed", [0, 1])
+def test_shift_schedule_lzs_extremes(Q, seed):
+    """Groups mixing decoded +-112 and +-1..7 through the shift schedule."""
+    M, N, K = 128, 136, 256
+    xa, xw = _lzs_extreme(M, K, 300 + seed), _lzs_extreme(N, K, 400 + seed)
+    va, vw = O.decode_values(O.encode(xa, 64, 16)), O.decode_values(O.encode(xw, 64, 16))
+    a = Q.quantize(torch.from_numpy(xa).cuda(), group_s=16)
+    w = Q.encode_weights(torch.from_numpy(xw).cuda(), group_s=16)
+    for g in range(K // 64):
+        _, part = Q.linear(a, w, out_dtype=torch.float32, partials_group=g, algo=Q.ALGO_SHIFT)
+        ref = O.group_partials(va[:, g * 64:(g + 1) * 64], vw[:, g * 64:(g + 1) * 64], 64)[0]
+        assert np.array_equal(part.cpu().numpy().astype(np.int64), ref), f"group {g}"
