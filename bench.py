@@ -71,21 +71,30 @@ def peaks():
         return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS, FALLBACK_SM_MHZ, "fallback"
 
 
+def gemm_source_hash():
+    """sha256 (first 16 hex) of the tcgen05 GEMM's source: its section of
+    csrc/linear.cu (from the "2. tcgen05 GEMM" banner to the "3. SIMT GEMM"
+    banner) plus csrc/ptx.cuh."""
+    import hashlib
+    csrc = os.path.join(ROOT, "paper_2509_26436_gb300", "csrc")
+    with open(os.path.join(csrc, "linear.cu")) as fh:
+        src = fh.read()
+    section = src[src.index("// 2. tcgen05 GEMM"):src.index("// 3. SIMT GEMM")]
+    h = hashlib.sha256(section.encode())
+    with open(os.path.join(csrc, "ptx.cuh"), "rb") as fh:
+        h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
 def gemm_traffic():
     """DRAM bytes per GEMM launch from the committed ncu summary, if it was
     taken on the GEMM source as it is now (else None)."""
-    import hashlib
-    csrc = os.path.join(ROOT, "paper_2509_26436_gb300", "csrc")
-    h = hashlib.sha256()
-    for f in ("linear.cu", "ptx.cuh"):
-        with open(os.path.join(csrc, f), "rb") as fh:
-            h.update(fh.read())
     try:
         with open(os.path.join(ROOT, "profiles", "gemm_tcgen05_flux_block.md")) as fh:
             kv = dict(line.split(": ", 1) for line in fh if line.startswith(("gemm_source_sha16", "dram_bytes")))
     except OSError:
         return None
-    if kv.get("gemm_source_sha16", "").strip() != h.hexdigest()[:16]:
+    if kv.get("gemm_source_sha16", "").strip() != gemm_source_hash():
         return None
     return float(kv["dram_bytes_per_launch"])
 
