@@ -65,6 +65,8 @@ def _load():
             lib.oracle_unpack_nibbles.argtypes = [P, i64, P]
             lib.oracle_unpack_nibbles.restype = None
             lib.oracle_encode.argtypes = [P, i64, i64, i32, i32, i32, P, P, P, P, P]
+            lib.oracle_quantize_static.argtypes = [P, i64, C.c_uint16, P]
+            lib.oracle_encode_static.argtypes = [P, i64, i64, C.c_uint16, i32, i32, P, P, P]
             lib.oracle_decode_codes.argtypes = [P, P, i64, i64, i32, P]
             lib.oracle_dequantize.argtypes = [P, P, P, P, i64, i64, i32, i32, P]
             lib.oracle_group_partials.argtypes = [P, P, i64, i64, i64, i32, P, i64, P]
@@ -192,6 +194,28 @@ def encode(x16: np.ndarray, group_q: int = 64, group_s: int = 16, mode: int = SY
     _check(_load().oracle_encode(_ptr(xb), R, K, group_q, group_s, mode, _ptr(codes),
                                  _ptr(flags), _ptr(scales), _ptr(zeros), _ptr(gsum)))
     return Encoded(codes, flags, scales.view(np.float16), zeros, gsum, group_q, group_s, mode)
+
+
+def quantize_static(x16: np.ndarray, s16) -> np.ndarray:
+    """Static per-tensor Eq. 1 with a given fp16 scale: q int8, same shape."""
+    xb = _as_u16(x16)
+    q = np.empty(xb.shape, np.int8)
+    _check(_load().oracle_quantize_static(_ptr(xb), xb.size, int(np.float16(s16).view(np.uint16)), _ptr(q)))
+    return q
+
+
+def encode_static(x16: np.ndarray, s16, group_q: int = 64, group_s: int = 16) -> Encoded:
+    """Encoder with a static (calibrated) scale for every group (symmetric)."""
+    xb = _as_u16(x16)
+    R, K = xb.shape
+    G = K // group_q
+    codes = np.empty((R, K // 2), np.uint8)
+    flags = np.empty((R, K // group_s), np.uint8)
+    scales = np.empty((R, G), np.uint16)
+    _check(_load().oracle_encode_static(_ptr(xb), R, K, int(np.float16(s16).view(np.uint16)), group_q,
+                                        group_s, _ptr(codes), _ptr(flags), _ptr(scales)))
+    return Encoded(codes, flags, scales.view(np.float16), np.zeros((R, G), np.int8),
+                   np.zeros((R, G), np.int32), group_q, group_s, SYMMETRIC)
 
 
 def decode_values(e: Encoded) -> np.ndarray:

@@ -164,6 +164,31 @@ int oracle_quantize(const uint16_t *x, int64_t rows, int64_t K, int group_q, int
 }
 
 /* ---------------------------------------------------------------------------
+ * Static per-tensor quantization (Appendix C: the latent-diffusion setting
+ * quantizes activations statically per tensor).  The scale s (fp16 bits) is
+ * calibrated beforehand and given; every element is quantized with it as in
+ * Eq. 1 (symmetric, z = 0): x_hat = clamp(round(x / s), -127, 127), x / s
+ * evaluated as x * r with r = RN(1/s) (R3); s = 0 gives all-zero codes (R5).
+ * Values beyond 127 s saturate.  Output q [n].
+ * ------------------------------------------------------------------------- */
+int oracle_quantize_static(const uint16_t *x, int64_t n, uint16_t s16, int8_t *q)
+{
+    float s = oracle_half_to_float(s16);
+    if (n < 0 || !(s >= 0.0f) || s > 65504.0f) return ORACLE_ERR_ARG;
+    if (s == 0.0f) {
+        for (int64_t i = 0; i < n; ++i) q[i] = 0;
+        return ORACLE_OK;
+    }
+    float r = 1.0f / s;
+    for (int64_t i = 0; i < n; ++i) {
+        float t = oracle_half_to_float(x[i]) * r;
+        t = clamp_float(t, -1024.0f, 1024.0f);
+        q[i] = (int8_t)clamp_int(rne_int(t), -127, 127);
+    }
+    return ORACLE_OK;
+}
+
+/* ---------------------------------------------------------------------------
  * Stage 2: Leading Zero Suppression (Section 3, Eq. 2).
  * Each int8 code is viewed as sign + 7-bit magnitude; per subgroup of G_s
  * codes the magnitudes are OR-ed into m, FLAG = max(29 - clz(m), 0), and
@@ -276,6 +301,27 @@ int oracle_encode(const uint16_t *x, int64_t rows, int64_t K, int gq, int gs, in
                 gsum[row * G + g] = s;
             }
         }
+    }
+    return ORACLE_OK;
+}
+
+/* Encoder with a static scale: Eq. 1 with the given scale (above), then
+ * Eq. 2 as oracle_encode; scales [rows, K/gq] all receive s16 (symmetric). */
+int oracle_encode_static(const uint16_t *x, int64_t rows, int64_t K, uint16_t s16, int gq, int gs,
+                         uint8_t *codes, uint8_t *flags, uint16_t *scales)
+{
+    if (gs <= 0 || gq % gs != 0 || K % gq != 0 || K % 2 != 0) return ORACLE_ERR_ARG;
+    int8_t q[65536];
+    int8_t c[65536];
+    if (K > 65536) return ORACLE_ERR_ARG;
+    int64_t G = K / gq;
+    for (int64_t row = 0; row < rows; ++row) {
+        int rc = oracle_quantize_static(x + row * K, K, s16, q);
+        if (rc) return rc;
+        rc = oracle_lzs_encode(q, K, gs, flags + row * (K / gs), c);
+        if (rc) return rc;
+        oracle_pack_nibbles(c, K, codes + row * (K / 2));
+        for (int64_t g = 0; g < G; ++g) scales[row * G + g] = s16;
     }
     return ORACLE_OK;
 }

@@ -451,3 +451,41 @@ def test_quantize_ties_and_zero_point_golden():
     assert int(z[0, 0]) == int(g["asym_zero"][0])
     assert list(q[0, :len(t)]) == [int(v) for v in g["asym_q"]]
     assert (q[0, len(t):] == int(g["asym_zero"][0])).all()
+
+
+# --- static per-tensor quantization (Appendix C, latent-diffusion setting) ---
+
+def test_static_scale_equals_own_per_tensor_scale():
+    """With the tensor's own per-tensor scale, static encoding equals dynamic
+    encoding of the whole tensor as one quantization group (flattened to a
+    single row): the dynamic route computes the scale from the data, the
+    static route is handed it."""
+    x = inputs.mixture_activations(8, 512, seed=91)
+    s16 = np.float16(np.float32(np.abs(x.astype(np.float32)).max()) / np.float32(127))
+    for gs in (8, 16, 32, 64):
+        st = O.encode_static(x, s16, 512, gs)
+        dyn = O.encode(x.reshape(1, -1), x.size, gs)
+        assert np.array_equal(st.codes.reshape(-1), dyn.codes.reshape(-1))
+        assert np.array_equal(st.flags.reshape(-1), dyn.flags.reshape(-1))
+        assert np.all(st.scales.view(np.uint16) == dyn.scales.view(np.uint16)[0, 0])
+
+
+def test_static_scale_saturates_and_rounds():
+    """Closed form: q = clamp(round-half-even(x * r), -127, 127), r = RN(1/s),
+    checked on values chosen exactly in units of s = 2^-4 (r exact)."""
+    s16 = np.float16(2.0 ** -4)
+    units = np.array([0, 1, -1, 2.5, -2.5, 3.5, 126.5, 127, 127.5, 200, -200, -300, 1000, -1e4])
+    x = (units * 2.0 ** -4).astype(np.float16)
+    q = O.quantize_static(x.reshape(1, -1), s16).ravel()
+    expect = np.clip(np.round(units), -127, 127)      # numpy rounds half to even
+    assert np.array_equal(q, expect.astype(np.int8))
+    assert np.array_equal(O.quantize_static(x.reshape(1, -1), np.float16(0)).ravel(), np.zeros_like(q))
+
+
+def test_static_scale_codes_follow_lzs_of_saturated_values():
+    """Every saturated element becomes code +-7 with FLAG 4 (decoded +-112)."""
+    x = np.full((1, 64), 50.0, np.float16)
+    x[0, 1::2] = -50.0
+    e = O.encode_static(x, np.float16(0.01), 64, 16)
+    v = O.decode_values(e)
+    assert np.all(np.abs(v) == 112) and np.all(e.flags == 4)
