@@ -65,7 +65,9 @@ typedef enum { QUARTZ_OUT_F16 = 0, QUARTZ_OUT_BF16 = 1, QUARTZ_OUT_F32 = 2 } qua
 typedef enum { QUARTZ_ALGO_TCGEN05 = 0, QUARTZ_ALGO_SIMT = 1, QUARTZ_ALGO_SHIFT = 2 } quartz_algo_t;
 
 typedef struct {
-    int32_t group_q; /* min-max quantization group along K; 64 (Appendix C) */
+    int32_t group_q; /* min-max quantization group along K: 64 (Appendix C), or K
+                      * (one scale per row: per-token activations / per-channel
+                      * weights; SYMMETRIC only) */
     int32_t group_s; /* LZS subgroup G_s along K: 8, 16, 32 or 64 (Section 3, Table 1) */
     int32_t mode;    /* quartz_mode_t */
 } quartz_params_t;
@@ -113,6 +115,15 @@ int32_t quartz_encoded_sizes(int64_t rows, int64_t K, const quartz_params_t *p, 
  * Requirements: rows >= 0, K > 0, K % 64 == 0, group_q == 64, group_s in
  * {8,16,32,64}.  rows == 0 is a no-op. */
 int32_t quartz_quantize(const void *x_f16, const quartz_encoded_t *out, void *stream);
+
+/* Static per-tensor quantization (Appendix C: the latent-diffusion models
+ * quantize activations with one static, calibrated scale per tensor): Eq. 1
+ * with the given fp16 scale `scale_f16` (bits; finite, >= 0) for every
+ * element instead of a scale computed from the data, then Eq. 2.  Elements
+ * beyond 127 * scale saturate to +-127 before LZS.  SYMMETRIC mode; any
+ * group_q; every stored scale of `out` is `scale_f16`.  A zero scale gives
+ * all-zero codes. */
+int32_t quartz_quantize_static(const void *x_f16, uint16_t scale_f16, const quartz_encoded_t *out, void *stream);
 
 /* The same encoder applied to nn.Linear weights [N, K] (one quantization
  * row per output channel, groups along K).  Weights are encoded once,

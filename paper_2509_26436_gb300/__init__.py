@@ -93,20 +93,37 @@ def _check_f16(x, name):
 
 
 def quantize(x, group_s: int = 16, mode: int = SYMMETRIC, out: Encoded | None = None,
-             stream=None, _entry="quartz_quantize") -> Encoded:
-    """Eq. 1 + Eq. 2 on fp16 activations [M, K] (K % 64 == 0)."""
+             stream=None, _entry="quartz_quantize", group_q: int = 64) -> Encoded:
+    """Eq. 1 + Eq. 2 on fp16 activations [M, K] (K % 64 == 0); group_q = 64
+    or K (one scale per row)."""
     _check_f16(x, "x")
     rows, K = x.shape
-    e = out if out is not None else empty_encoded(rows, K, Params(64, group_s, mode), x.device)
+    e = out if out is not None else empty_encoded(rows, K, Params(group_q, group_s, mode), x.device)
     ec = e.c()
     N.check(getattr(N.load(), _entry)(x.data_ptr(), C.byref(ec), _stream(stream)), _entry)
     return e
 
 
 def encode_weights(w, group_s: int = 16, mode: int = SYMMETRIC, out: Encoded | None = None,
-                   stream=None) -> Encoded:
-    """The same encoder applied to nn.Linear weights [N, K], run offline."""
-    return quantize(w, group_s, mode, out, stream, _entry="quartz_encode_weights")
+                   stream=None, group_q: int = 64) -> Encoded:
+    """The same encoder applied to nn.Linear weights [N, K], run offline
+    (group_q = K gives per-output-channel scales)."""
+    return quantize(w, group_s, mode, out, stream, _entry="quartz_encode_weights", group_q=group_q)
+
+
+def quantize_static(x, scale, group_s: int = 16, group_q: int = 64, out: Encoded | None = None,
+                    stream=None) -> Encoded:
+    """Static per-tensor quantization: Eq. 1 with the given calibrated fp16
+    scale for every element (symmetric), then Eq. 2."""
+    import numpy as np
+    _check_f16(x, "x")
+    rows, K = x.shape
+    e = out if out is not None else empty_encoded(rows, K, Params(group_q, group_s, SYMMETRIC), x.device)
+    ec = e.c()
+    bits = int(np.float16(scale).view(np.uint16))
+    N.check(N.load().quartz_quantize_static(x.data_ptr(), bits, C.byref(ec), _stream(stream)),
+            "quartz_quantize_static")
+    return e
 
 
 def dequantize(e: Encoded, stream=None):

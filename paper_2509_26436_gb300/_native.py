@@ -56,6 +56,7 @@ SIGNATURES = {
     "quartz_version": (_I32, []),
     "quartz_encoded_sizes": (_I32, [_I64, _I64, C.POINTER(QuartzParams), C.POINTER(_SZ)]),
     "quartz_quantize": (_I32, [_P, C.POINTER(QuartzEncoded), _P]),
+    "quartz_quantize_static": (_I32, [_P, C.c_uint16, C.POINTER(QuartzEncoded), _P]),
     "quartz_encode_weights": (_I32, [_P, C.POINTER(QuartzEncoded), _P]),
     "quartz_dequantize": (_I32, [C.POINTER(QuartzEncoded), _P, _P]),
     "quartz_linear_workspace_size": (_SZ, [_I64, _I64, _I64, C.POINTER(QuartzParams)]),

@@ -22,7 +22,7 @@ int32_t check_params(const quartz_params_t *p)
     if (p->group_s != 8 && p->group_s != 16 && p->group_s != 32 && p->group_s != 64)
         return QUARTZ_ERR_INVALID_ARG;
     if (p->group_q <= 0 || p->group_q % p->group_s != 0) return QUARTZ_ERR_INVALID_ARG;
-    if (p->group_q != 64) return QUARTZ_ERR_UNSUPPORTED;
+    if (p->group_q % 64 != 0) return QUARTZ_ERR_UNSUPPORTED;
     return QUARTZ_OK;
 }
 
@@ -32,6 +32,9 @@ int32_t check_shape(int64_t rows, int64_t K, const quartz_params_t *p)
     if (rc) return rc;
     if (rows < 0 || K <= 0 || K % p->group_q != 0) return QUARTZ_ERR_INVALID_ARG;
     if (rows > (int64_t(1) << 31) || K > (int64_t(1) << 24)) return QUARTZ_ERR_UNSUPPORTED;
+    // groups of 64 along K (Appendix C), or one group per row (per-token /
+    // per-channel scales, symmetric)
+    if (p->group_q != 64 && (p->group_q != K || p->mode != QUARTZ_SYMMETRIC)) return QUARTZ_ERR_UNSUPPORTED;
     return QUARTZ_OK;
 }
 
@@ -113,6 +116,21 @@ int32_t quartz_quantize(const void *x_f16, const quartz_encoded_t *out, void *st
     return map_cuda(launch_quantize(x_f16, out, static_cast<cudaStream_t>(stream)));
 }
 
+int32_t quartz_quantize_static(const void *x_f16, uint16_t scale_f16, const quartz_encoded_t *out, void *stream)
+{
+    int32_t rc = check_encoded(out);
+    if (rc) return rc;
+    if (out->p.mode != QUARTZ_SYMMETRIC) return QUARTZ_ERR_UNSUPPORTED;
+    // a finite, non-negative fp16 scale
+    if ((scale_f16 & 0x8000u) && scale_f16 != 0x8000u) return QUARTZ_ERR_INVALID_ARG;
+    if ((scale_f16 & 0x7C00u) == 0x7C00u) return QUARTZ_ERR_INVALID_ARG;
+    if (out->rows == 0) return QUARTZ_OK;
+    if (!x_f16) return QUARTZ_ERR_INVALID_ARG;
+    if (!aligned16(x_f16)) return QUARTZ_ERR_ALIGNMENT;
+    return map_cuda(launch_quantize_static(x_f16, out, static_cast<uint16_t>(scale_f16 & 0x7FFFu),
+                                           static_cast<cudaStream_t>(stream)));
+}
+
 int32_t quartz_encode_weights(const void *w_f16, const quartz_encoded_t *out, void *stream)
 {
     return quartz_quantize(w_f16, out, stream);
@@ -151,6 +169,7 @@ int32_t quartz_linear_ex(const quartz_encoded_t *a, const quartz_encoded_t *w,
     if (a->K != w->K || a->p.group_q != w->p.group_q || a->p.group_s != w->p.group_s ||
         a->p.mode != w->p.mode)
         return QUARTZ_ERR_INVALID_ARG;
+    if (a->p.group_q != 64) return QUARTZ_ERR_UNSUPPORTED;
     const int64_t M = a->rows, N = w->rows, K = a->K;
     if (N <= 0 || N % 8 != 0 || N > (int64_t(1) << 24)) return QUARTZ_ERR_INVALID_ARG;
     if (y_type != QUARTZ_OUT_F16 && y_type != QUARTZ_OUT_BF16 && y_type != QUARTZ_OUT_F32)
@@ -202,7 +221,7 @@ int32_t quartz_linear_f16(const void *x_f16, int64_t M, const quartz_encoded_t *
 {
     int32_t rc = check_encoded(w);
     if (rc) return rc;
-    if (w->p.mode != QUARTZ_SYMMETRIC) return QUARTZ_ERR_UNSUPPORTED;
+    if (w->p.mode != QUARTZ_SYMMETRIC || w->p.group_q != 64) return QUARTZ_ERR_UNSUPPORTED;
     const int64_t N = w->rows, K = w->K;
     rc = check_shape(M, K, &w->p);
     if (rc) return rc;

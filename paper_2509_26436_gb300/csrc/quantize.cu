@@ -167,6 +167,45 @@ __device__ __forceinline__ UnitCodes encode_unit_sym(const uint4 lo, const uint4
     return u;
 }
 
+// The same encoding with a scale fixed beforehand (one per row, or a static
+// calibrated one): FLAGs from the subgroup maxima (shuffles over 2 or 4
+// lanes for G_s = 32, 64; all 32 lanes call it together) and codes capped at
+// +-127 when an element of this thread exceeds the scale's range.
+template <int GS>
+__device__ __forceinline__ UnitCodes encode_unit_sym_scaled(const uint4 lo, const uint4 hi, __half s16, float r)
+{
+    const uint32_t w[8] = {lo.x, lo.y, lo.z, lo.w, hi.x, hi.y, hi.z, hi.w};
+    uint32_t a[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) a[i] = w[i] & 0x7FFF7FFFu;
+    __half2 m0 = __hmax2(__hmax2(*reinterpret_cast<const __half2 *>(&a[0]), *reinterpret_cast<const __half2 *>(&a[1])),
+                         __hmax2(*reinterpret_cast<const __half2 *>(&a[2]), *reinterpret_cast<const __half2 *>(&a[3])));
+    __half2 m1 = __hmax2(__hmax2(*reinterpret_cast<const __half2 *>(&a[4]), *reinterpret_cast<const __half2 *>(&a[5])),
+                         __hmax2(*reinterpret_cast<const __half2 *>(&a[6]), *reinterpret_cast<const __half2 *>(&a[7])));
+    const float2 f0 = __half22float2(m0), f1 = __half22float2(m1);
+    const float sub0 = fmaxf(f0.x, f0.y), sub1 = fmaxf(f1.x, f1.y);
+    const float unit_max = fmaxf(sub0, sub1);
+    UnitCodes u;
+    u.s16 = s16;
+    if (GS == 8) {
+        u.flag0 = lzs_flag_of(sub0, r);
+        u.flag1 = lzs_flag_of(sub1, r);
+    } else {
+        float m = unit_max;
+        if (GS >= 32) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 1));
+        if (GS >= 64) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 2));
+        u.flag0 = u.flag1 = lzs_flag_of(m, r);
+    }
+    if (__float2int_rn(fminf(__fmul_rn(unit_max, r), 1024.0f)) > 127) {
+        u.c0 = lzs_word8<true>(w, a, r, u.flag0);
+        u.c1 = lzs_word8<true>(w + 4, a + 4, r, u.flag1);
+    } else {
+        u.c0 = lzs_word8<false>(w, a, r, u.flag0);
+        u.c1 = lzs_word8<false>(w + 4, a + 4, r, u.flag1);
+    }
+    return u;
+}
+
 // Store one unit's encoding: codes, FLAG byte(s), and the scale once per group.
 template <int GS>
 __device__ __forceinline__ void store_unit_sym(const UnitCodes &u, int64_t unit, int lane,
@@ -205,6 +244,72 @@ __global__ void __launch_bounds__(kThreads) quantize_sym_kernel(const uint4 *__r
         const int64_t u = base + j * kThreads;
         const UnitCodes c = encode_unit_sym<GS>(raw[j][0], raw[j][1]);
         if (u < n_units) store_unit_sym<GS>(c, u, lane, codes, flags, scales);
+    }
+}
+
+// One block per row, for scales that are not per 64-group: either the row's
+// own scale (group_q = K, per-token / per-channel: a first pass over the row
+// finds max |x|), or a static calibrated scale `static_s16` given by the
+// caller (any group_q; every group's stored scale is that value).  A second
+// pass encodes the row with it.
+template <int GS>
+__global__ void __launch_bounds__(kThreads) quantize_row_sym_kernel(const uint4 *__restrict__ x, int64_t K,
+                                                                    int group_q, int use_static,
+                                                                    unsigned short static_s16,
+                                                                    uint2 *__restrict__ codes,
+                                                                    uint8_t *__restrict__ flags,
+                                                                    __half *__restrict__ scales)
+{
+    __shared__ float warp_max[kThreads / 32];
+    const int lane = threadIdx.x & 31;
+    const int64_t row = blockIdx.x;
+    const int64_t U = K / 16;                       // units per row (a multiple of 4)
+    const int64_t rounds = (U + kThreads - 1) / kThreads;
+    const uint4 *xr = x + row * U * 2;
+    __half s16;
+    if (use_static) {
+        s16 = __ushort_as_half(static_s16);
+    } else {
+        float m = 0.f;
+        for (int64_t it = 0; it < rounds; ++it) {
+            const int64_t j = it * kThreads + threadIdx.x;
+            if (j >= U) break;
+            const uint4 lo = ldg_stream(xr + 2 * j), hi = ldg_stream(xr + 2 * j + 1);
+            const uint32_t w[8] = {lo.x, lo.y, lo.z, lo.w, hi.x, hi.y, hi.z, hi.w};
+            __half2 h = __habs2(*reinterpret_cast<const __half2 *>(&w[0]));
+#pragma unroll
+            for (int i = 1; i < 8; ++i) h = __hmax2(h, __habs2(*reinterpret_cast<const __half2 *>(&w[i])));
+            const float2 f = __half22float2(h);
+            m = fmaxf(m, fmaxf(f.x, f.y));
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+        if (lane == 0) warp_max[threadIdx.x >> 5] = m;
+        __syncthreads();
+        m = 0.f;
+#pragma unroll
+        for (int i = 0; i < kThreads / 32; ++i) m = fmaxf(m, warp_max[i]);
+        s16 = __float2half_rn(__fdiv_rn(m, 127.0f));
+    }
+    const float s = __half2float(s16);
+    const float r = (s > 0.f) ? __frcp_rn(s) : 0.f;
+    for (int64_t it = 0; it < rounds; ++it) {   // the same trip count in every lane (shuffles)
+        const int64_t j = it * kThreads + threadIdx.x;
+        const bool in = j < U;
+        const uint4 lo = in ? ldg_stream(xr + 2 * j) : make_uint4(0, 0, 0, 0);
+        const uint4 hi = in ? ldg_stream(xr + 2 * j + 1) : make_uint4(0, 0, 0, 0);
+        const UnitCodes c = encode_unit_sym_scaled<GS>(lo, hi, s16, r);
+        if (!in) continue;
+        const int64_t u = row * U + j;
+        codes[u] = make_uint2(c.c0, c.c1);
+        if (GS == 8) {
+            reinterpret_cast<uint16_t *>(flags)[u] = static_cast<uint16_t>(c.flag0 | (c.flag1 << 8));
+        } else if (GS == 16) {
+            flags[u] = static_cast<uint8_t>(c.flag0);
+        } else if ((lane & (GS / 16 - 1)) == 0) {
+            flags[u / (GS / 16)] = static_cast<uint8_t>(c.flag0);
+        }
+        if ((j * 16) % group_q == 0) scales[(u * 16) / group_q] = s16;
     }
 }
 
@@ -375,14 +480,14 @@ __global__ void __launch_bounds__(kThreads) quantize_kernel(const uint4 *__restr
 // x_hat = s * (v - z), v = sgn(c) (|c| << FLAG); one thread per 8 elements.
 __global__ void __launch_bounds__(kThreads) dequantize_kernel(
     const uint32_t *__restrict__ codes, const uint8_t *__restrict__ flags,
-    const __half *__restrict__ scales, const int8_t *__restrict__ zeros, int group_s,
+    const __half *__restrict__ scales, const int8_t *__restrict__ zeros, int group_s, int group_q,
     int64_t n_chunks, uint4 *__restrict__ out)
 {
     const int64_t c = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x;
     if (c >= n_chunks) return;
     const uint32_t word = codes[c];
     const int flag = flags[(c * 8) / group_s];
-    const int64_t g = c >> 3;
+    const int64_t g = (c * 8) / group_q;
     const float s = __half2float(scales[g]);
     const int z = zeros ? zeros[g] : 0;
     uint32_t o[4];
@@ -431,12 +536,40 @@ cudaError_t launch_q_mode(const void *x, const quartz_encoded_t *e, cudaStream_t
     }
 }
 
+template <int GS>
+cudaError_t launch_row(const void *x, const quartz_encoded_t *e, int use_static, unsigned short s16,
+                       cudaStream_t s)
+{
+    quantize_row_sym_kernel<GS><<<static_cast<unsigned>(e->rows), kThreads, 0, s>>>(
+        static_cast<const uint4 *>(x), e->K, e->p.group_q, use_static, s16, reinterpret_cast<uint2 *>(e->codes),
+        e->flags, reinterpret_cast<__half *>(e->scales));
+    return cudaGetLastError();
+}
+
+cudaError_t launch_quantize_row(const void *x, const quartz_encoded_t *e, int use_static, unsigned short s16,
+                                cudaStream_t s)
+{
+    switch (e->p.group_s) {
+        case 8: return launch_row<8>(x, e, use_static, s16, s);
+        case 16: return launch_row<16>(x, e, use_static, s16, s);
+        case 32: return launch_row<32>(x, e, use_static, s16, s);
+        default: return launch_row<64>(x, e, use_static, s16, s);
+    }
+}
+
 }  // namespace
+
+cudaError_t launch_quantize_static(const void *x, const quartz_encoded_t *out, uint16_t s16, cudaStream_t s)
+{
+    if (out->rows == 0) return cudaSuccess;
+    return launch_quantize_row(x, out, 1, s16, s);
+}
 
 cudaError_t launch_quantize(const void *x, const quartz_encoded_t *out, cudaStream_t s)
 {
     static_assert(kGroupQ == 64, "one quantization group is 8 lanes x 8 elements");
     if (out->rows == 0) return cudaSuccess;
+    if (out->p.group_q != kGroupQ) return launch_quantize_row(x, out, 0, 0, s);  // group_q == K
     return out->p.mode == QUARTZ_SYMMETRIC ? launch_q_mode<QUARTZ_SYMMETRIC>(x, out, s)
                                            : launch_q_mode<QUARTZ_ASYMMETRIC>(x, out, s);
 }
@@ -471,7 +604,7 @@ cudaError_t launch_dequantize(const quartz_encoded_t *e, void *y, cudaStream_t s
     dequantize_kernel<<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(
         reinterpret_cast<const uint32_t *>(e->codes), e->flags,
         reinterpret_cast<const __half *>(e->scales),
-        e->p.mode == QUARTZ_ASYMMETRIC ? e->zeros : nullptr, e->p.group_s, n_chunks,
+        e->p.mode == QUARTZ_ASYMMETRIC ? e->zeros : nullptr, e->p.group_s, e->p.group_q, n_chunks,
         static_cast<uint4 *>(y));
     return cudaGetLastError();
 }

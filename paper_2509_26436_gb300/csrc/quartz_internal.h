@@ -24,6 +24,8 @@ int *device_error_word();
 // Encoder / decoder launches (quantize.cu).  Arguments are pre-validated.
 cudaError_t launch_quantize(const void *x, const quartz_encoded_t *out, cudaStream_t s);
 cudaError_t launch_dequantize(const quartz_encoded_t *e, void *y, cudaStream_t s);
+// Symmetric encoding with a static (calibrated) fp16 scale `s16` for every group.
+cudaError_t launch_quantize_static(const void *x, const quartz_encoded_t *out, uint16_t s16, cudaStream_t s);
 
 // Position of activation row r in its group's side-value row: inside every
 // block of 32 rows, row 8a + b sits at 4b + a, so that the four rows

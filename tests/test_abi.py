@@ -66,8 +66,12 @@ def test_host_validation_rejects_before_launch(lib):
     assert q(0x1000, C.byref(e), None) == N.QUARTZ_ERR_INVALID_ARG
     e = _enc(4, 128, gs=12)                            # G_s not in {8,16,32,64}
     assert q(0x1000, C.byref(e), None) == N.QUARTZ_ERR_INVALID_ARG
-    e = N.QuartzEncoded(0x1000, 0x1000, 0x1000, 0, 0, 4, 128, N.QuartzParams(128, 16, 0))
-    assert q(0x1000, C.byref(e), None) == N.QUARTZ_ERR_UNSUPPORTED   # group_q != 64
+    e = N.QuartzEncoded(0x1000, 0x1000, 0x1000, 0, 0, 4, 256, N.QuartzParams(128, 16, 0))
+    assert q(0x1000, C.byref(e), None) == N.QUARTZ_ERR_UNSUPPORTED   # group_q neither 64 nor K
+    e = N.QuartzEncoded(0x1000, 0x1000, 0x1000, 0, 0, 4, 192, N.QuartzParams(96, 16, 0))
+    assert q(0x1000, C.byref(e), None) == N.QUARTZ_ERR_UNSUPPORTED   # group_q not a multiple of 64
+    e = N.QuartzEncoded(0x1000, 0x1000, 0x1000, 0x1000, 0x1000, 4, 256, N.QuartzParams(256, 16, 1))
+    assert q(0x1000, C.byref(e), None) == N.QUARTZ_ERR_UNSUPPORTED   # per-row scales are symmetric only
     e = _enc(4, 128, mode=7)
     assert q(0x1000, C.byref(e), None) == N.QUARTZ_ERR_INVALID_ARG
     e = _enc(4, 128)
@@ -80,6 +84,17 @@ def test_host_validation_rejects_before_launch(lib):
     e = _enc(-1, 128)
     assert q(0x1000, C.byref(e), None) == N.QUARTZ_ERR_INVALID_ARG
     assert lib.quartz_dequantize(C.byref(_enc(4, 128)), None, None) == N.QUARTZ_ERR_INVALID_ARG
+
+
+def test_quantize_static_validation(lib):
+    qs = lib.quartz_quantize_static
+    e = _enc(4, 128)
+    assert qs(0x1000, 0x7C00, C.byref(e), None) == N.QUARTZ_ERR_INVALID_ARG   # +inf scale
+    assert qs(0x1000, 0xBC00, C.byref(e), None) == N.QUARTZ_ERR_INVALID_ARG   # -1.0
+    assert qs(0x1000, 0x7E00, C.byref(e), None) == N.QUARTZ_ERR_INVALID_ARG   # NaN
+    assert qs(0x1001, 0x3C00, C.byref(e), None) == N.QUARTZ_ERR_ALIGNMENT
+    assert qs(0x1000, 0x3C00, C.byref(_enc(4, 128, mode=1)), None) == N.QUARTZ_ERR_UNSUPPORTED
+    assert qs(None, 0x3C00, C.byref(_enc(0, 128)), None) == N.QUARTZ_OK         # empty
 
 
 def test_linear_validation(lib):

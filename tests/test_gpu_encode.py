@@ -135,3 +135,32 @@ def test_weights_encoder_is_the_same_arithmetic(Q):
     torch.cuda.synchronize()
     _assert_encoded_equal(e, O.encode(w, 64, 16, O.SYMMETRIC), O.SYMMETRIC)
     assert Q.device_status() == 0
+
+
+@pytest.mark.parametrize("gs", [8, 16, 32, 64])
+@pytest.mark.parametrize("shape", [(1, 64), (37, 1152), (5, 12288), (300, 3072)])
+def test_encode_per_row_scale_bit_exact(Q, gs, shape):
+    """group_q = K: one scale per row (per-token activations / per-channel
+    weights), bit-exact against the oracle."""
+    rows, K = shape
+    x = inputs.mixture_activations(rows, K, seed=2000 + rows + gs)
+    e = Q.quantize(torch.from_numpy(x).cuda(), group_s=gs, group_q=K)
+    torch.cuda.synchronize()
+    ref = O.encode(x, K, gs)
+    _assert_encoded_equal(e, ref, O.SYMMETRIC)
+    xh = Q.dequantize(e)
+    assert torch.equal(xh.cpu(), torch.from_numpy(O.dequantize(ref).astype(np.float16)))
+
+
+@pytest.mark.parametrize("gs", [8, 16, 32, 64])
+@pytest.mark.parametrize("group_q", [64, "K"])
+def test_encode_static_scale_bit_exact(Q, gs, group_q):
+    """Static per-tensor scale (calibrated elsewhere): bit-exact against the
+    oracle, including saturation of values beyond 127 * scale."""
+    rows, K = 40, 1152
+    gq = K if group_q == "K" else 64
+    x = inputs.mixture_activations(rows, K, seed=3000 + gs)
+    for scale in (np.float16(0.06), np.float16(0.004), np.float16(2.0 ** -20), np.float16(0)):
+        e = Q.quantize_static(torch.from_numpy(x).cuda(), scale, group_s=gs, group_q=gq)
+        torch.cuda.synchronize()
+        _assert_encoded_equal(e, O.encode_static(x, scale, gq, gs), O.SYMMETRIC)
