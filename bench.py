@@ -45,6 +45,9 @@ def parse():
     p.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
     p.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline leg")
     p.add_argument("--no-fused", action="store_true", help="skip the fused activation-path leg")
+    p.add_argument("--scales", choices=["group64", "per-row"], default="group64",
+                   help="group64: 64-wide groups along K (Appendix C, the default workload); "
+                        "per-row: one scale per token row and per output channel (group_q = K)")
     p.add_argument("--compare-algos", action="store_true",
                    help="also time the three GEMM algorithms (tcgen05, simt, shift) on each layer")
     p.add_argument("--layers", default="", help="comma-separated subset of layer names (profiling)")
@@ -104,9 +107,10 @@ def dist_env():
             int(os.environ.get("LOCAL_RANK", 0)))
 
 
-def layer_config(layers):
+def layer_config(layers, per_row=False):
     return {"workload": "flux1_schnell_mmdit_block_linears", "tokens": layers[0].M,
-            "layers": [f"{l.name}:{l.K}->{l.N}" for l in layers], "group_q": GROUP_Q,
+            "layers": [f"{l.name}:{l.K}->{l.N}" for l in layers],
+            "group_q": "K (per-token x per-channel)" if per_row else GROUP_Q,
             "group_s": GROUP_S, "mode": "symmetric", "out": "f16",
             "inputs": "seeded synthetic Laplace(0,0.05), 0.1% channels x50; weights N(0,0.02)",
             "l2": "activations per step 0.8 GB > 129 MB L2, no flush"}
@@ -122,10 +126,10 @@ def select_layers(all_layers, names):
     return sel
 
 
-def encode_bytes_per_elem(gs=GROUP_S):
+def encode_bytes_per_elem(gs=GROUP_S, gq=GROUP_Q):
     """Algorithmic HBM bytes of the encoder per element: fp16 in, 4-bit code,
-    one FLAG byte per G_s, one fp16 scale per 64 (symmetric)."""
-    return 2.0 + 0.5 + 1.0 / gs + 2.0 / GROUP_Q
+    one FLAG byte per G_s, one fp16 scale per group_q (symmetric)."""
+    return 2.0 + 0.5 + 1.0 / gs + 2.0 / gq
 
 
 # --------------------------------------------------------------------------
@@ -184,7 +188,7 @@ class ClockSampler:
 # --------------------------------------------------------------------------
 # CPU oracle baseline (a bounded sample of the same workload)
 # --------------------------------------------------------------------------
-def oracle_sample(layers, rows_per_layer, xs=None, ws=None, cols_per_layer=None):
+def oracle_sample(layers, rows_per_layer, xs=None, ws=None, cols_per_layer=None, per_row=False):
     """Time the oracle on `rows_per_layer` token rows of every layer (and the
     first `cols_per_layer` output channels, or all): encode (Eq. 1 + Eq. 2)
     of those rows plus the W4A4 linear for them.  Weights are encoded before
@@ -197,14 +201,14 @@ def oracle_sample(layers, rows_per_layer, xs=None, ws=None, cols_per_layer=None)
         w = ws[i] if ws is not None else l.weights()
         if cols_per_layer is not None:
             w = np.ascontiguousarray(w[:cols_per_layer])
-        enc_w.append(O.encode(w, GROUP_Q, GROUP_S))
+        enc_w.append(O.encode(w, l.K if per_row else GROUP_Q, GROUP_S))
         x = xs[i] if xs is not None else l.activations()
         sel = np.linspace(0, l.M - 1, rows_per_layer).astype(np.int64)
         xa_s.append(np.ascontiguousarray(x[sel]))
     t0 = time.perf_counter()
     ops = 0
     for l, x, ew in zip(layers, xa_s, enc_w):
-        ea = O.encode(x, GROUP_Q, GROUP_S)
+        ea = O.encode(x, l.K if per_row else GROUP_Q, GROUP_S)
         O.linear(ea, ew)
         ops += 2 * x.shape[0] * ew.rows * l.K
     return time.perf_counter() - t0, ops
@@ -269,8 +273,10 @@ def run_ours(args):
     ws = [l.weights() for l in layers]
     x_host = [torch.from_numpy(x).pin_memory() for x in xs]
     x_dev = [h.to(dev) for h in x_host]
-    enc_w = [Q.encode_weights(torch.from_numpy(w).to(dev), group_s=GROUP_S) for w in ws]
-    enc_a = [Q.empty_encoded(l.M, l.K, Q.Params(GROUP_Q, GROUP_S), dev) for l in layers]
+    per_row = args.scales == "per-row"
+    gq = [l.K if per_row else GROUP_Q for l in layers]
+    enc_w = [Q.encode_weights(torch.from_numpy(w).to(dev), group_s=GROUP_S, group_q=g) for w, g in zip(ws, gq)]
+    enc_a = [Q.empty_encoded(l.M, l.K, Q.Params(g, GROUP_S), dev) for l, g in zip(layers, gq)]
     y_dev = [torch.empty((l.M, l.N), dtype=torch.float16, device=dev) for l in layers]
     ws_bytes = max(Q.linear_workspace_size(l.M, l.N, l.K) for l in layers)
     workspace = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
@@ -285,7 +291,7 @@ def run_ours(args):
         for i in range(nl):
             if rec is not None:
                 rec["q"][i][0].record(stream)
-            Q.quantize(x_dev[i], out=enc_a[i], group_s=GROUP_S)
+            Q.quantize(x_dev[i], out=enc_a[i], group_s=GROUP_S, group_q=gq[i])
             if rec is not None:
                 rec["q"][i][1].record(stream)
             Q.linear(enc_a[i], enc_w[i], out=y_dev[i], workspace=workspace,
@@ -339,18 +345,40 @@ def run_ours(args):
     t_gemm = sum(gemm_ms) / 1e3
     gemm_tflops = sum(l.ops for l in layers) / t_gemm / 1e12
     # dequant epilogue: one fp32 multiply and one fused multiply-add per
-    # output element and 64-wide group (y += s_a * (s_w * P_g))
-    epi_ops = sum(2 * l.M * l.N * (l.K // GROUP_Q) for l in layers)
+    # output element and 64-wide group (y += s_a * (s_w * P_g)); with per-row
+    # scales one float add and one integer add per output and 256 of K
+    if per_row:
+        epi_ops = sum(2 * l.M * l.N * -(-l.K // 256) for l in layers)
+    else:
+        epi_ops = sum(2 * l.M * l.N * (l.K // GROUP_Q) for l in layers)
     gemm_alu = epi_ops / t_gemm / 1e12
     t_floor_tensor = sum(l.ops for l in layers) / (fp8_peak * 1e12)
     t_floor_alu = epi_ops / (alu_peak * 1e12)
     elems = sum(l.M * l.K for l in layers)
-    enc_gbs = elems * encode_bytes_per_elem() / (sum(quant_ms) / 1e3) / 1e9
+    enc_bytes = sum(l.M * l.K * encode_bytes_per_elem(GROUP_S, g) for l, g in zip(layers, gq))
+    enc_gbs = enc_bytes / (sum(quant_ms) / 1e3) / 1e9
     launches_per_step = nl * 3   # quantize; prepare (both operands); GEMM
+
+    alu_view = {"achieved": gemm_alu, "unit": "Top/s", "peak": alu_peak, "frac": gemm_alu / alu_peak,
+                "peak_source": f"derived: {n_sm} SMs x {FP32_LANES_PER_SM} fp32 lanes x "
+                               f"{sm_mhz:.0f} MHz ({peak_src} max SM clock)",
+                "work": ("1 fp32 add + 1 int32 add per output per 256 of K" if per_row else
+                         "2 fp32 ops (multiply + fused multiply-add) per output per 64-wide group")}
+    tensor_view = {"achieved": gemm_tflops, "unit": "TFLOP/s", "peak": fp8_peak, "frac": gemm_tflops / fp8_peak,
+                   "peak_source": f"{peak_src} bf16 burst {bf16_peak} x {FP8_OVER_BF16} (nominal FP8 : BF16)",
+                   "work": "2 M N K FP8 MMA flops"}
+    bound = "alu" if t_floor_alu >= t_floor_tensor else "tensor"
+    main, other = (alu_view, tensor_view) if bound == "alu" else (tensor_view, alu_view)
+    roofline = {"bound": bound, "achieved": main["achieved"], "peak": main["peak"], "unit": main["unit"],
+                "frac": main["frac"], "traffic": None if per_row else gemm_traffic(),
+                "kernel": "gemm_tcgen05_kernel", "peak_source": main["peak_source"], "work": main["work"],
+                "tensor" if bound == "alu" else "alu": other,
+                "floors_ms": {"alu": t_floor_alu * 1e3, "tensor": t_floor_tensor * 1e3},
+                "per_layer_ms": gemm_ms}
 
     # ---- fused activation path (quartz_linear_f16: encode into the operand) -
     fused = None
-    if not args.no_fused:
+    if not args.no_fused and not per_row:
         def fused_step():
             for i in range(nl):
                 Q.linear_f16(x_dev[i], enc_w[i], out=y_dev[i], workspace=workspace)
@@ -384,7 +412,7 @@ def run_ours(args):
         for name, algo in (("tcgen05", Q.ALGO_TCGEN05), ("simt", Q.ALGO_SIMT), ("shift", Q.ALGO_SHIFT)):
             per = []
             for i in range(nl):
-                Q.quantize(x_dev[i], out=enc_a[i], group_s=GROUP_S)
+                Q.quantize(x_dev[i], out=enc_a[i], group_s=GROUP_S, group_q=gq[i])
                 Q.linear(enc_a[i], enc_w[i], out=y_dev[i], workspace=workspace, algo=algo)
                 evs = [(ev(), ev()) for _ in range(3)]
                 for e in evs:
@@ -421,7 +449,7 @@ def run_ours(args):
                     loaded[u] = torch.cuda.Event()
                     loaded[u].record(s_in)
                 stream.wait_event(loaded[u])
-                Q.quantize(x_buf[p][i], out=enc_a[i], group_s=GROUP_S)
+                Q.quantize(x_buf[p][i], out=enc_a[i], group_s=GROUP_S, group_q=gq[i])
                 consumed[u] = torch.cuda.Event()
                 consumed[u].record(stream)
                 if u >= 2:
@@ -462,7 +490,7 @@ def run_ours(args):
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
         rows = 128
-        t, ops = oracle_sample(layers, rows, xs, ws)
+        t, ops = oracle_sample(layers, rows, xs, ws, per_row=per_row)
         cpu = {"value": ops / t / 1e12, "unit": "TOPS", "cores": 1, "kind": "oracle",
                "sample": f"{rows} token rows of each of the 4 layers (encode + linear), "
                          f"{t:.1f} s single-threaded plain C"}
@@ -476,22 +504,10 @@ def run_ours(args):
         "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": t_step * 1e3, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "e4m3/f32", "data": "synthetic",
-        "config": layer_config(layers),
-        "roofline": {"bound": "alu" if t_floor_alu >= t_floor_tensor else "tensor",
-                     "achieved": gemm_alu, "peak": alu_peak, "unit": "Top/s",
-                     "frac": gemm_alu / alu_peak, "traffic": gemm_traffic(),
-                     "kernel": "gemm_tcgen05_kernel",
-                     "peak_source": f"derived: {n_sm} SMs x {FP32_LANES_PER_SM} fp32 lanes x "
-                                    f"{sm_mhz:.0f} MHz ({peak_src} max SM clock)",
-                     "work": "2 fp32 ops (multiply + fused multiply-add) per output per 64-wide group",
-                     "tensor": {"achieved": gemm_tflops, "unit": "TFLOP/s", "peak": fp8_peak,
-                                "frac": gemm_tflops / fp8_peak,
-                                "peak_source": f"{peak_src} bf16 burst {bf16_peak} x {FP8_OVER_BF16} "
-                                               "(nominal FP8 : BF16)"},
-                     "floors_ms": {"alu": t_floor_alu * 1e3, "tensor": t_floor_tensor * 1e3},
-                     "per_layer_ms": gemm_ms},
+        "config": layer_config(layers, per_row),
+        "roofline": roofline,
         "encode": {"kernel": "quantize_kernel", "gbs": enc_gbs, "peak_gbs": hbm_peak,
-                   "frac": enc_gbs / hbm_peak, "bytes_per_elem": encode_bytes_per_elem(),
+                   "frac": enc_gbs / hbm_peak, "bytes_per_elem": enc_bytes / elems,
                    "per_layer_ms": quant_ms, "peak_source": peak_src},
         "clocks": clocks,
         "gpu_launches": launches_per_step * args.steps,

@@ -169,7 +169,8 @@ int32_t quartz_linear_ex(const quartz_encoded_t *a, const quartz_encoded_t *w,
     if (a->K != w->K || a->p.group_q != w->p.group_q || a->p.group_s != w->p.group_s ||
         a->p.mode != w->p.mode)
         return QUARTZ_ERR_INVALID_ARG;
-    if (a->p.group_q != 64) return QUARTZ_ERR_UNSUPPORTED;
+    const bool per_row = a->p.group_q != 64;  // group_q == K (check_shape allows nothing else)
+    if (per_row && o.algo != QUARTZ_ALGO_TCGEN05) return QUARTZ_ERR_UNSUPPORTED;
     const int64_t M = a->rows, N = w->rows, K = a->K;
     if (N <= 0 || N % 8 != 0 || N > (int64_t(1) << 24)) return QUARTZ_ERR_INVALID_ARG;
     if (y_type != QUARTZ_OUT_F16 && y_type != QUARTZ_OUT_BF16 && y_type != QUARTZ_OUT_F32)
@@ -202,7 +203,7 @@ int32_t quartz_linear_ex(const quartz_encoded_t *a, const quartz_encoded_t *w,
         e = launch_gemm_shift(ws, a, w, bias_f16, y, y_type, partials, partials_group, s);
     else
         e = launch_gemm_tcgen05(ws, M, N, K, a->p.mode, bias_f16, y, y_type, partials,
-                                partials_group, dev_err, s);
+                                partials_group, dev_err, s, per_row);
     if (e == cudaSuccess && o.gemm_event_end)
         e = cudaEventRecord(static_cast<cudaEvent_t>(o.gemm_event_end), s);
     return map_cuda(e);

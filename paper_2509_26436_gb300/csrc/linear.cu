@@ -182,7 +182,12 @@ constexpr uint32_t kRegsControl = 32;
 static_assert(kEpiWarps * 32 * kRegsEpilogue + 128 * kRegsControl <= kThreads * kRegsLaunch,
               "register split exceeds the launch allocation");
 constexpr uint32_t kTmemCols = 512;   // two fp32 accumulators of 256 columns
-constexpr int kRasterM = 8;           // tiles are visited in bands of 8 M-tiles
+constexpr int kRasterM = 8;
+// Per-row scales (group_q = K): the MMA accumulates kPerRowChunk stages (256
+// of K) into one TMEM accumulator before the epilogue takes it; each such sum
+// is an integer below 256 * 112^2 < 2^22, exact in fp32 and convertible with
+// the 1.5 * 2^23 rounding addend, and the epilogue adds it to an int32.
+constexpr int kPerRowChunk = 4;           // tiles are visited in bands of 8 M-tiles
 
 struct GemmArgs {
     const float *a_side;  // [nside][G][m_pad]
@@ -196,6 +201,7 @@ struct GemmArgs {
     int32_t *partials;
     int partials_group;
     int *dev_err;
+    int per_row;          // scales per row (group_q = K) rather than per 64-group
 };
 
 // Shared memory: the operand stages, then a ring of side-value slots (one
@@ -279,13 +285,64 @@ __device__ __forceinline__ void epi_half_chunk_sym(uint32_t taddr, float4 sw, ui
         : "memory");
 }
 
+// Per-row-scale epilogue step for half of one 16-column chunk: one
+// 16x128b.x4 TMEM load of an accumulator whose values are exact integers
+// below 2^22, each turned into an int32 with the 1.5 * 2^23 rounding addend
+// (the integer is the float's bit pattern minus 0x4B400000) and added to acc.
+__device__ __forceinline__ void epi_half_chunk_int(uint32_t taddr, int32_t *acc)
+{
+    asm volatile(
+        "{\n\t"
+        ".reg .b32 p<8>;\n\t"
+        ".reg .f32 f<8>;\n\t"
+        "tcgen05.ld.sync.aligned.16x128b.x4.b32 {p0, p1, p2, p3, p4, p5, p6, p7}, [%8];\n\t"
+        "tcgen05.wait::ld.sync.aligned;\n\t"
+        "add.rn.f32 f0, p0, 0f4B400000;\n\t"
+        "add.rn.f32 f1, p1, 0f4B400000;\n\t"
+        "add.rn.f32 f2, p2, 0f4B400000;\n\t"
+        "add.rn.f32 f3, p3, 0f4B400000;\n\t"
+        "add.rn.f32 f4, p4, 0f4B400000;\n\t"
+        "add.rn.f32 f5, p5, 0f4B400000;\n\t"
+        "add.rn.f32 f6, p6, 0f4B400000;\n\t"
+        "add.rn.f32 f7, p7, 0f4B400000;\n\t"
+        "mov.b32 p0, f0;\n\t"
+        "mov.b32 p1, f1;\n\t"
+        "mov.b32 p2, f2;\n\t"
+        "mov.b32 p3, f3;\n\t"
+        "mov.b32 p4, f4;\n\t"
+        "mov.b32 p5, f5;\n\t"
+        "mov.b32 p6, f6;\n\t"
+        "mov.b32 p7, f7;\n\t"
+        "sub.s32 p0, p0, 0x4B400000;\n\t"
+        "sub.s32 p1, p1, 0x4B400000;\n\t"
+        "sub.s32 p2, p2, 0x4B400000;\n\t"
+        "sub.s32 p3, p3, 0x4B400000;\n\t"
+        "sub.s32 p4, p4, 0x4B400000;\n\t"
+        "sub.s32 p5, p5, 0x4B400000;\n\t"
+        "sub.s32 p6, p6, 0x4B400000;\n\t"
+        "sub.s32 p7, p7, 0x4B400000;\n\t"
+        "add.s32 %0, %0, p0;\n\t"
+        "add.s32 %1, %1, p1;\n\t"
+        "add.s32 %2, %2, p2;\n\t"
+        "add.s32 %3, %3, p3;\n\t"
+        "add.s32 %4, %4, p4;\n\t"
+        "add.s32 %5, %5, p5;\n\t"
+        "add.s32 %6, %6, p6;\n\t"
+        "add.s32 %7, %7, p7;\n\t"
+        "}"
+        : "+r"(acc[0]), "+r"(acc[1]), "+r"(acc[2]), "+r"(acc[3]), "+r"(acc[4]), "+r"(acc[5]),
+          "+r"(acc[6]), "+r"(acc[7])
+        : "r"(taddr)
+        : "memory");
+}
+
 // Two 64-bit words from shared memory (one 16-byte load).
 __device__ __forceinline__ void lds_b64x2(uint32_t addr, uint64_t &a, uint64_t &b)
 {
     asm volatile("ld.shared.v2.b64 {%0, %1}, [%2];" : "=l"(a), "=l"(b) : "r"(addr) : "memory");
 }
 
-template <int MODE, int OUT, bool DUMP>
+template <int MODE, int OUT, bool DUMP, bool PERROW>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tmap_a,
                         const __grid_constant__ CUtensorMap tmap_w, const GemmArgs args)
@@ -382,7 +439,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // zero-point terms) go by bulk copy into a ring slot that the
         // epilogue frees.
         // ------------------------------------------------------------------
-        if (lane == 0) {
+        if (!PERROW && lane == 0) {
             constexpr int S = L::kSideSlots;
             const int64_t a_plane = args.m_pad * G;
             const int64_t w_plane = args.n_pad * G;
@@ -426,17 +483,21 @@ __global__ void __launch_bounds__(kThreads, 1)
             constexpr uint32_t idesc = idesc_e4m3_f32(BM, BN);
             int it = 0;
             bool ok = true;
+            constexpr int CH = PERROW ? kPerRowChunk : 1;  // stages per TMEM accumulator
+            int ic = 0;                                    // accumulators handed to the epilogue
             for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
                 for (int g = 0; g < G; ++g, ++it) {
                     const int s = it % kStages;
-                    const int b = it & 1;
+                    const int b = ic & 1;
+                    const bool first = (g % CH) == 0;
+                    const bool last = (g % CH) == CH - 1 || g == G - 1;
                     if (!mbar_wait_bounded(full_bar(s), (it / kStages) & 1, abort_flag, args.dev_err,
                                            kWaitLimitNs)) {
                         ok = false;
                         break;
                     }
-                    if (it >= 2 && !mbar_wait_bounded(acc_empty_bar(b), ((it >> 1) - 1) & 1,
-                                                      abort_flag, args.dev_err, kWaitLimitNs)) {
+                    if (first && ic >= 2 && !mbar_wait_bounded(acc_empty_bar(b), ((ic >> 1) - 1) & 1,
+                                                               abort_flag, args.dev_err, kWaitLimitNs)) {
                         ok = false;
                         break;
                     }
@@ -447,10 +508,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int kk = 0; kk < BK / 32; ++kk) {
                         const uint64_t adesc = sdesc_k_major_sw64(sa + kk * 32);
                         const uint64_t bdesc = sdesc_k_major_sw64(sa + kABytes + kk * 32);
-                        mma_f8_ss(d, adesc, bdesc, idesc, kk > 0 ? 1u : 0u);
+                        mma_f8_ss(d, adesc, bdesc, idesc, (kk > 0 || !first) ? 1u : 0u);
                     }
                     mma_commit(empty_bar(s));
-                    mma_commit(acc_full_bar(b));
+                    if (last) {
+                        mma_commit(acc_full_bar(b));
+                        ++ic;
+                    }
                 }
             }
             // Make sure no MMA is still writing TMEM before it is freed.
@@ -484,7 +548,77 @@ __global__ void __launch_bounds__(kThreads, 1)
 
         // acc[h][j]: output column 16*(j/4) + tq + j%4 of this warp's slice,
         // rows trow + 16h (.x) and trow + 16h + 8 (.y)
-        if constexpr (MODE == QUARTZ_SYMMETRIC && !DUMP) {
+        if constexpr (PERROW) {
+            // Per-row scales (group_q = K, symmetric): each TMEM accumulator
+            // holds the exact integer sum of kPerRowChunk stages; the epilogue
+            // adds it into int32 accumulators and scales once per tile:
+            // y = s_a * (s_w * P).  acci[c][4h + i] = rows trow + 16h (i < 4:
+            // pairs 2i / 2i + 1 are rows +0 / +8) of column 16c + tq + i%4.
+            int32_t acci[4][16];
+            int ic = 0;
+            bool ok = true;
+            const int nchunks = (G + kPerRowChunk - 1) / kPerRowChunk;
+            for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
+#pragma unroll
+                for (int c = 0; c < 4; ++c)
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) acci[c][j] = 0;
+                for (int cc = 0; cc < nchunks; ++cc, ++ic) {
+                    const int b = ic & 1;
+                    if (!mbar_wait_bounded(acc_full_bar(b), (ic >> 1) & 1, abort_flag, args.dev_err,
+                                           kWaitLimitNs)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t tbase = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
+                                           static_cast<uint32_t>(b * BN + slot * kColsPerWarp);
+#pragma unroll
+                    for (int chunk = 0; chunk < 4; ++chunk) {
+                        epi_half_chunk_int(tbase + 16 * chunk, acci[chunk]);
+                        epi_half_chunk_int(tbase + (16u << 16) + 16 * chunk, acci[chunk] + 8);
+                    }
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(acc_empty_bar(b));
+                }
+                if (!ok) break;
+                int mt, nt;
+                tile_coords(tile, args, mt, nt);
+#pragma unroll
+                for (int h = 0; h < 2; ++h)
+#pragma unroll
+                    for (int e = 0; e < 2; ++e) {
+                        const int64_t m = static_cast<int64_t>(mt) * BM + quarter * 32 + 16 * h + 8 * e + trow;
+                        if (m >= args.M) continue;
+                        const float s_a = args.a_side[perm32(m)];
+#pragma unroll
+                        for (int chunk = 0; chunk < 4; ++chunk) {
+                            const int64_t n = static_cast<int64_t>(nt) * BN + slot * kColsPerWarp + 16 * chunk + tq;
+                            if (n >= args.N) continue;
+                            float vv[4];
+#pragma unroll
+                            for (int i = 0; i < 4; ++i) {
+                                const int32_t P = acci[chunk][8 * h + 2 * i + e];
+                                if (DUMP) args.partials[m * args.N + n + i] = P;
+                                const float t = __fmul_rn(static_cast<float>(P), args.w_side[n + i]);
+                                vv[i] = __fmul_rn(t, s_a);
+                            }
+                            float4 v = make_float4(vv[0], vv[1], vv[2], vv[3]);
+                            if (args.bias) {
+                                const uint2 braw = __ldg(reinterpret_cast<const uint2 *>(args.bias + n));
+                                const float2 b0 = __half22float2(*reinterpret_cast<const __half2 *>(&braw.x));
+                                const float2 b1 = __half22float2(*reinterpret_cast<const __half2 *>(&braw.y));
+                                v.x = __fadd_rn(v.x, b0.x);
+                                v.y = __fadd_rn(v.y, b0.y);
+                                v.z = __fadd_rn(v.z, b1.x);
+                                v.w = __fadd_rn(v.w, b1.y);
+                            }
+                            store_quad<OUT>(args.y, m * args.N + n, v);
+                        }
+                    }
+            }
+        } else if constexpr (MODE == QUARTZ_SYMMETRIC && !DUMP) {
             // Symmetric fast path: each half chunk (16 lanes x 16 columns: TMEM
             // load, wait and the scale arithmetic) is one PTX block on
             // explicit 64-bit pairs, which keeps the kernel free of spills.
@@ -925,7 +1059,13 @@ cudaError_t launch_tc(const CUtensorMap &ta, const CUtensorMap &tw, const GemmAr
     constexpr int NSIDE = (MODE == QUARTZ_ASYMMETRIC) ? 3 : 1;
     constexpr int smem = Smem<NSIDE>::kAlloc;
     static_assert(smem <= 227 * 1024, "shared memory budget");
-    auto kern = args.partials ? gemm_tcgen05_kernel<MODE, OUT, true> : gemm_tcgen05_kernel<MODE, OUT, false>;
+    auto kern = args.partials ? gemm_tcgen05_kernel<MODE, OUT, true, false>
+                              : gemm_tcgen05_kernel<MODE, OUT, false, false>;
+    if constexpr (MODE == QUARTZ_SYMMETRIC) {
+        if (args.per_row)
+            kern = args.partials ? gemm_tcgen05_kernel<MODE, OUT, true, true>
+                                 : gemm_tcgen05_kernel<MODE, OUT, false, true>;
+    }
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     const int grid = args.num_tiles < num_sms() ? args.num_tiles : num_sms();
@@ -968,6 +1108,7 @@ GemmArgs make_args(const LinearWorkspace &ws, int64_t M, int64_t N, int64_t K, c
                    void *y, int y_type, int32_t *partials, int partials_group, int *dev_err)
 {
     GemmArgs a;
+    a.per_row = 0;
     a.a_side = ws.a_side;
     a.w_side = ws.w_side;
     a.m_pad = ws.m_pad;
@@ -1024,7 +1165,7 @@ cudaError_t launch_prepare(const quartz_encoded_t *a, const quartz_encoded_t *w,
     const int64_t K = w->K;
     const int64_t upr = K / 16;
     PrepArgs p{};
-    p.G = static_cast<int>(K / kGroupQ);
+    p.G = static_cast<int>(K / w->p.group_q);  // scale groups per row
     p.nside = ws.nside;
     if (a)
         p.ex_a = {reinterpret_cast<const uint2 *>(a->codes), a->flags, static_cast<uint4 *>(ws.a_op),
@@ -1057,13 +1198,15 @@ cudaError_t launch_prepare(const quartz_encoded_t *a, const quartz_encoded_t *w,
 cudaError_t launch_gemm_tcgen05(const LinearWorkspace &ws, int64_t M, int64_t N, int64_t K,
                                 int mode, const void *bias, void *y, int y_type,
                                 int32_t *partials, int partials_group, int *dev_err,
-                                cudaStream_t s)
+                                cudaStream_t s, bool per_row)
 {
     if (M == 0) return cudaSuccess;
     CUtensorMap ta, tw;
     if (!make_operand_map(&ta, ws.a_op, M, K, BM) || !make_operand_map(&tw, ws.w_op, round_up(N, 16), K, BN))
         return cudaErrorInvalidValue;
-    const GemmArgs args = make_args(ws, M, N, K, bias, y, y_type, partials, partials_group, dev_err);
+    GemmArgs args = make_args(ws, M, N, K, bias, y, y_type, partials, partials_group, dev_err);
+    args.per_row = per_row ? 1 : 0;
+    if (per_row) return launch_tc_out<QUARTZ_SYMMETRIC>(ta, tw, args, y_type, s);
     return mode == QUARTZ_ASYMMETRIC ? launch_tc_out<QUARTZ_ASYMMETRIC>(ta, tw, args, y_type, s)
                                      : launch_tc_out<QUARTZ_SYMMETRIC>(ta, tw, args, y_type, s);
 }

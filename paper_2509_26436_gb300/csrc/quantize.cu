@@ -116,6 +116,13 @@ __device__ __forceinline__ int lzs_flag_of(float amax_sub, float r)
     return max(29 - __clz(qmax), 0);
 }
 
+// 16-element units per LZS subgroup (G_s >= 16).
+template <int GS>
+__host__ __device__ constexpr int kUnitsPerSub()
+{
+    return GS >= 16 ? GS / 16 : 1;
+}
+
 // Eq. 1 + Eq. 2 on the 16 elements of one unit (lo, hi: eight fp16 pairs):
 // the group scale and, per 8-element half, the FLAG and the eight codes.  All
 // 32 lanes must call it together (group and subgroup maxima are shuffles).
@@ -217,8 +224,8 @@ __device__ __forceinline__ void store_unit_sym(const UnitCodes &u, int64_t unit,
         reinterpret_cast<uint16_t *>(flags)[unit] = static_cast<uint16_t>(u.flag0 | (u.flag1 << 8));
     } else if (GS == 16) {
         flags[unit] = static_cast<uint8_t>(u.flag0);
-    } else if ((lane & (GS / 16 - 1)) == 0) {
-        flags[unit / (GS / 16)] = static_cast<uint8_t>(u.flag0);
+    } else if ((lane & (kUnitsPerSub<GS>() - 1)) == 0) {
+        flags[unit / kUnitsPerSub<GS>()] = static_cast<uint8_t>(u.flag0);
     }
     if ((lane & 3) == 0) scales[unit >> 2] = u.s16;
 }
@@ -306,8 +313,8 @@ __global__ void __launch_bounds__(kThreads) quantize_row_sym_kernel(const uint4 
             reinterpret_cast<uint16_t *>(flags)[u] = static_cast<uint16_t>(c.flag0 | (c.flag1 << 8));
         } else if (GS == 16) {
             flags[u] = static_cast<uint8_t>(c.flag0);
-        } else if ((lane & (GS / 16 - 1)) == 0) {
-            flags[u / (GS / 16)] = static_cast<uint8_t>(c.flag0);
+        } else if ((lane & (kUnitsPerSub<GS>() - 1)) == 0) {
+            flags[u / kUnitsPerSub<GS>()] = static_cast<uint8_t>(c.flag0);
         }
         if ((j * 16) % group_q == 0) scales[(u * 16) / group_q] = s16;
     }

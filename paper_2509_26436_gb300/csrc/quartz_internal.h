@@ -62,10 +62,11 @@ cudaError_t launch_gemm_shift(const LinearWorkspace &ws, const quartz_encoded_t 
 // side values; `enc` (may be NULL) also receives the encoded tensor.
 cudaError_t launch_encode_operand(const void *x, int64_t M, int64_t K, const quartz_params_t *p,
                                   const LinearWorkspace &ws, const quartz_encoded_t *enc, cudaStream_t s);
+// per_row: one scale per row of both operands (group_q = K, symmetric).
 cudaError_t launch_gemm_tcgen05(const LinearWorkspace &ws, int64_t M, int64_t N, int64_t K,
                                 int mode, const void *bias, void *y, int y_type,
                                 int32_t *partials, int partials_group, int *dev_err,
-                                cudaStream_t s);
+                                cudaStream_t s, bool per_row = false);
 cudaError_t launch_gemm_simt(const LinearWorkspace &ws, int64_t M, int64_t N, int64_t K, int mode,
                              const void *bias, void *y, int y_type, int32_t *partials,
                              int partials_group, cudaStream_t s);

@@ -287,3 +287,53 @@ def test_shift_schedule_lzs_extremes(Q, seed):
         _, part = Q.linear(a, w, out_dtype=torch.float32, partials_group=g, algo=Q.ALGO_SHIFT)
         ref = O.group_partials(va[:, g * 64:(g + 1) * 64], vw[:, g * 64:(g + 1) * 64], 64)[0]
         assert np.array_equal(part.cpu().numpy().astype(np.int64), ref), f"group {g}"
+
+
+@pytest.mark.parametrize("gs", [8, 16, 64])
+@pytest.mark.parametrize("M,N,K", [(1, 8, 64), (200, 264, 640), (300, 520, 3072), (129, 256, 12288)])
+def test_per_row_scales_linear(Q, gs, M, N, K):
+    """group_q = K on both operands (per-token activations, per-channel
+    weights): the whole-K integer partial sum is exact (it is accumulated in
+    exact 256-wide pieces) and y matches the oracle."""
+    xa = inputs.laplace_activations(M, K, seed=M + N + K + gs)
+    xw = inputs.gaussian_weights(N, K, seed=3 * N + K)
+    bias = inputs.gaussian_weights(1, N, seed=N + 1)[0]
+    a = Q.quantize(torch.from_numpy(xa).cuda(), group_s=gs, group_q=K)
+    w = Q.encode_weights(torch.from_numpy(xw).cuda(), group_s=gs, group_q=K)
+    y, part = Q.linear(a, w, torch.from_numpy(bias).cuda(), out_dtype=torch.float32, partials_group=0)
+    assert Q.device_status() == 0
+    ea, ew = O.encode(xa, K, gs), O.encode(xw, K, gs)
+    ref, rabs = O.linear(ea, ew, bias, with_abs=True)
+    _tol_check(y.cpu().numpy(), ref, rabs, 1, "float32")
+    P = O.group_partials(O.decode_values(ea), O.decode_values(ew), K)[0]
+    assert np.array_equal(part.cpu().numpy().astype(np.int64), P)
+    y16 = Q.linear(a, w, torch.from_numpy(bias).cuda())
+    _tol_check(y16.float().cpu().numpy(), ref, rabs, 1, "float16")
+
+
+def test_per_row_scales_extreme_partials(Q):
+    """Whole-K partials far beyond 2^24 (every decoded value +-112): exact."""
+    M, N, K = 128, 64, 12288
+    xa = np.where(np.random.default_rng(1).random((M, K)) < 0.9, 1.0, -1.0).astype(np.float16)
+    xw = np.ones((N, K), np.float16)
+    a = Q.quantize(torch.from_numpy(xa).cuda(), group_s=16, group_q=K)
+    w = Q.encode_weights(torch.from_numpy(xw).cuda(), group_s=16, group_q=K)
+    _, part = Q.linear(a, w, out_dtype=torch.float32, partials_group=0)
+    P = O.group_partials(O.decode_values(O.encode(xa, K, 16)), O.decode_values(O.encode(xw, K, 16)), K)[0]
+    assert np.abs(P).max() > 2 ** 24
+    assert np.array_equal(part.cpu().numpy().astype(np.int64), P)
+
+
+def test_static_activation_per_channel_weight_linear(Q):
+    """Appendix C's latent-diffusion setting: activations quantized with one
+    static calibrated scale, weights per output channel."""
+    M, N, K = 256, 320, 1152
+    xa = inputs.laplace_activations(M, K, seed=17)
+    xw = inputs.gaussian_weights(N, K, seed=18)
+    scale = np.float16(np.abs(xa.astype(np.float32)).max() / 127 * 0.8)   # clips the largest 20%
+    a = Q.quantize_static(torch.from_numpy(xa).cuda(), scale, group_s=16, group_q=K)
+    w = Q.encode_weights(torch.from_numpy(xw).cuda(), group_s=16, group_q=K)
+    y = Q.linear(a, w, out_dtype=torch.float32)
+    assert Q.device_status() == 0
+    ref, rabs = O.linear(O.encode_static(xa, scale, K, 16), O.encode(xw, K, 16), with_abs=True)
+    _tol_check(y.cpu().numpy(), ref, rabs, 1, "float32")
