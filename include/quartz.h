@@ -70,6 +70,9 @@ typedef struct {
                       * weights; SYMMETRIC only) */
     int32_t group_s; /* LZS subgroup G_s along K: 8, 16, 32 or 64 (Section 3, Table 1) */
     int32_t mode;    /* quartz_mode_t */
+    int32_t flag_bits; /* FLAG storage: 0 or 8 = one byte per subgroup (Section
+                        * 4.4); 4 = two FLAGs per byte (values 0..4 fit in 4
+                        * bits), 4 + 4/G_s + 16/group_q bits per element */
 } quartz_params_t;
 
 /* One encoded tensor of `rows` rows and `K` columns (Section 4.4: "packed
@@ -77,7 +80,11 @@ typedef struct {
  * memory owned by the caller; sizes in elements:
  *   codes  uint8 [rows, K/2]        two's-complement 4-bit codes in [-7, 7],
  *                                   element 2j in the low nibble of byte j
- *   flags  uint8 [rows, K/group_s]  FLAG of Eq. 2, values 0..4
+ *   flags  uint8 [rows, K/group_s]  FLAG of Eq. 2, values 0..4; with
+ *                                   flag_bits = 4: uint8 [ceil(rows*K/group_s
+ *                                   / 2)], FLAG of subgroup 2j (counted over
+ *                                   the whole tensor, row after row) in the
+ *                                   low nibble of byte j, 2j + 1 in the high
  *   scales fp16  [rows, K/group_q]  16-bit scale s of each group (bits)
  *   zeros  int8  [rows, K/group_q]  stored zero point z (ASYMMETRIC only;
  *                                   may be NULL in SYMMETRIC mode)

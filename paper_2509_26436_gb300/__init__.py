@@ -33,14 +33,17 @@ def _torch():
 
 @dataclass(frozen=True)
 class Params:
-    """group_q: min-max group along K (64, Appendix C); group_s: LZS
-    subgroup G_s (8/16/32/64, Section 3); mode: SYMMETRIC or ASYMMETRIC."""
+    """group_q: min-max group along K (64, Appendix C, or K for one scale per
+    row); group_s: LZS subgroup G_s (8/16/32/64, Section 3); mode: SYMMETRIC
+    or ASYMMETRIC; flag_bits: 8 (one FLAG byte per subgroup) or 4 (two FLAGs
+    per byte)."""
     group_q: int = 64
     group_s: int = 16
     mode: int = SYMMETRIC
+    flag_bits: int = 8
 
     def c(self) -> N.QuartzParams:
-        return N.QuartzParams(self.group_q, self.group_s, self.mode)
+        return N.QuartzParams(self.group_q, self.group_s, self.mode, self.flag_bits)
 
 
 class Encoded:
@@ -71,7 +74,10 @@ def empty_encoded(rows: int, K: int, params: Params = Params(), device="cuda") -
     N.check(N.load().quartz_encoded_sizes(rows, K, C.byref(p), sizes), "quartz_encoded_sizes")
     G = K // params.group_q
     codes = torch.empty((rows, K // 2), dtype=torch.uint8, device=device)
-    flags = torch.empty((rows, K // params.group_s), dtype=torch.uint8, device=device)
+    if params.flag_bits == 4:
+        flags = torch.empty((max(int(sizes[1]), 1),), dtype=torch.uint8, device=device)
+    else:
+        flags = torch.empty((rows, K // params.group_s), dtype=torch.uint8, device=device)
     scales = torch.empty((rows, G), dtype=torch.float16, device=device)
     zeros = gsum = None
     if params.mode == ASYMMETRIC:
@@ -93,32 +99,33 @@ def _check_f16(x, name):
 
 
 def quantize(x, group_s: int = 16, mode: int = SYMMETRIC, out: Encoded | None = None,
-             stream=None, _entry="quartz_quantize", group_q: int = 64) -> Encoded:
+             stream=None, _entry="quartz_quantize", group_q: int = 64, flag_bits: int = 8) -> Encoded:
     """Eq. 1 + Eq. 2 on fp16 activations [M, K] (K % 64 == 0); group_q = 64
     or K (one scale per row)."""
     _check_f16(x, "x")
     rows, K = x.shape
-    e = out if out is not None else empty_encoded(rows, K, Params(group_q, group_s, mode), x.device)
+    e = out if out is not None else empty_encoded(rows, K, Params(group_q, group_s, mode, flag_bits), x.device)
     ec = e.c()
     N.check(getattr(N.load(), _entry)(x.data_ptr(), C.byref(ec), _stream(stream)), _entry)
     return e
 
 
 def encode_weights(w, group_s: int = 16, mode: int = SYMMETRIC, out: Encoded | None = None,
-                   stream=None, group_q: int = 64) -> Encoded:
+                   stream=None, group_q: int = 64, flag_bits: int = 8) -> Encoded:
     """The same encoder applied to nn.Linear weights [N, K], run offline
     (group_q = K gives per-output-channel scales)."""
-    return quantize(w, group_s, mode, out, stream, _entry="quartz_encode_weights", group_q=group_q)
+    return quantize(w, group_s, mode, out, stream, _entry="quartz_encode_weights", group_q=group_q,
+                    flag_bits=flag_bits)
 
 
 def quantize_static(x, scale, group_s: int = 16, group_q: int = 64, out: Encoded | None = None,
-                    stream=None) -> Encoded:
+                    stream=None, flag_bits: int = 8) -> Encoded:
     """Static per-tensor quantization: Eq. 1 with the given calibrated fp16
     scale for every element (symmetric), then Eq. 2."""
     import numpy as np
     _check_f16(x, "x")
     rows, K = x.shape
-    e = out if out is not None else empty_encoded(rows, K, Params(group_q, group_s, SYMMETRIC), x.device)
+    e = out if out is not None else empty_encoded(rows, K, Params(group_q, group_s, SYMMETRIC, flag_bits), x.device)
     ec = e.c()
     bits = int(np.float16(scale).view(np.uint16))
     N.check(N.load().quartz_quantize_static(x.data_ptr(), bits, C.byref(ec), _stream(stream)),

@@ -19,6 +19,7 @@ int32_t check_params(const quartz_params_t *p)
 {
     if (!p) return QUARTZ_ERR_INVALID_ARG;
     if (p->mode != QUARTZ_SYMMETRIC && p->mode != QUARTZ_ASYMMETRIC) return QUARTZ_ERR_INVALID_ARG;
+    if (p->flag_bits != 0 && p->flag_bits != 4 && p->flag_bits != 8) return QUARTZ_ERR_INVALID_ARG;
     if (p->group_s != 8 && p->group_s != 16 && p->group_s != 32 && p->group_s != 64)
         return QUARTZ_ERR_INVALID_ARG;
     if (p->group_q <= 0 || p->group_q % p->group_s != 0) return QUARTZ_ERR_INVALID_ARG;
@@ -90,7 +91,7 @@ const char *quartz_status_string(int32_t status)
     }
 }
 
-int32_t quartz_version(void) { return (1 << 16) | 1; }
+int32_t quartz_version(void) { return (1 << 16) | 2; }
 
 int32_t quartz_encoded_sizes(int64_t rows, int64_t K, const quartz_params_t *p, size_t out[5])
 {
@@ -99,7 +100,7 @@ int32_t quartz_encoded_sizes(int64_t rows, int64_t K, const quartz_params_t *p, 
     if (rc) return rc;
     const int64_t G = K / p->group_q;
     out[0] = static_cast<size_t>(rows * (K / 2));
-    out[1] = static_cast<size_t>(rows * (K / p->group_s));
+    out[1] = static_cast<size_t>(p->flag_bits == 4 ? (rows * (K / p->group_s) + 1) / 2 : rows * (K / p->group_s));
     out[2] = static_cast<size_t>(rows * G * 2);
     out[3] = static_cast<size_t>(rows * G);
     out[4] = static_cast<size_t>(rows * G * 4);

@@ -68,6 +68,7 @@ struct ExpandJob {
     uint4 *out;                  // [rows_out, K/16] units of 16 E4M3 values
     int64_t units, units_pad, units_per_row;
     int permute;
+    int packed_flags;            // FLAGs two per byte
 };
 struct SideJob {
     const __half *scales;
@@ -102,11 +103,17 @@ __device__ __forceinline__ void run_expand(const ExpandJob &j, int64_t u)
     const uint2 c = j.codes[u];
     int f0, f1;
     if (GS == 8) {
-        const uint32_t ff = reinterpret_cast<const uint16_t *>(j.flags)[u];
-        f0 = static_cast<int>(ff & 0xFFu);
-        f1 = static_cast<int>(ff >> 8);
+        if (j.packed_flags) {
+            const uint32_t ff = j.flags[u];
+            f0 = static_cast<int>(ff & 0xFu);
+            f1 = static_cast<int>(ff >> 4);
+        } else {
+            const uint32_t ff = reinterpret_cast<const uint16_t *>(j.flags)[u];
+            f0 = static_cast<int>(ff & 0xFFu);
+            f1 = static_cast<int>(ff >> 8);
+        }
     } else {
-        f0 = f1 = j.flags[(u * 16) / GS];
+        f0 = f1 = load_flag(j.flags, (u * 16) / GS, j.packed_flags != 0);
     }
     uint4 o;
     e4m3_from_codes8(c.x, f0, o.x, o.y);
@@ -915,7 +922,7 @@ __global__ void __launch_bounds__(256) gemm_shift_kernel(const uint32_t *__restr
                                                          const uint8_t *__restrict__ a_flags,
                                                          const uint32_t *__restrict__ w_codes,
                                                          const uint8_t *__restrict__ w_flags,
-                                                         const GemmArgs args, int K)
+                                                         const GemmArgs args, int K, int a_packed, int w_packed)
 {
     constexpr int kSub = kGroupQ / GS;            // subgroups per group
     constexpr int kWordsPerSub = GS / 4;          // int8x4 words per subgroup
@@ -943,8 +950,8 @@ __global__ void __launch_bounds__(256) gemm_shift_kernel(const uint32_t *__restr
         for (int i = threadIdx.x; i < 64 * kSub; i += 256) {
             const int r = i / kSub, j = i % kSub;
             const int64_t col = static_cast<int64_t>(g) * kSub + j;
-            fa[r][j] = (m0 + r < args.M) ? a_flags[(m0 + r) * flags_per_row + col] : 0;
-            fw[r][j] = (n0 + r < args.N) ? w_flags[(n0 + r) * flags_per_row + col] : 0;
+            fa[r][j] = (m0 + r < args.M) ? load_flag(a_flags, (m0 + r) * flags_per_row + col, a_packed != 0) : 0;
+            fw[r][j] = (n0 + r < args.N) ? load_flag(w_flags, (n0 + r) * flags_per_row + col, w_packed != 0) : 0;
         }
         __syncthreads();
         int p[4][4] = {};
@@ -1169,10 +1176,10 @@ cudaError_t launch_prepare(const quartz_encoded_t *a, const quartz_encoded_t *w,
     p.nside = ws.nside;
     if (a)
         p.ex_a = {reinterpret_cast<const uint2 *>(a->codes), a->flags, static_cast<uint4 *>(ws.a_op),
-                  a->rows * upr, a->rows * upr, upr, 0};
+                  a->rows * upr, a->rows * upr, upr, 0, a->p.flag_bits == 4};
     // the weight operand is row-permuted and padded to a multiple of 16 rows
     p.ex_w = {reinterpret_cast<const uint2 *>(w->codes), w->flags, static_cast<uint4 *>(ws.w_op),
-              w->rows * upr, round_up(w->rows, 16) * upr, upr, 1};
+              w->rows * upr, round_up(w->rows, 16) * upr, upr, 1, w->p.flag_bits == 4};
     if (a)
         p.sd_a = {reinterpret_cast<const __half *>(a->scales), a->zeros, a->gsum, ws.a_side, a->rows, ws.m_pad, 1};
     p.sd_w = {reinterpret_cast<const __half *>(w->scales), w->zeros, w->gsum, ws.w_side, w->rows, ws.n_pad, 0};
@@ -1230,7 +1237,7 @@ cudaError_t launch_shift(const quartz_encoded_t *a, const quartz_encoded_t *w, c
     dim3 grid(static_cast<unsigned>((args.N + 63) / 64), static_cast<unsigned>((args.M + 63) / 64));
     gemm_shift_kernel<GS, MODE, OUT><<<grid, 256, 0, s>>>(
         reinterpret_cast<const uint32_t *>(a->codes), a->flags, reinterpret_cast<const uint32_t *>(w->codes),
-        w->flags, args, static_cast<int>(a->K));
+        w->flags, args, static_cast<int>(a->K), a->p.flag_bits == 4, w->p.flag_bits == 4);
     return cudaGetLastError();
 }
 

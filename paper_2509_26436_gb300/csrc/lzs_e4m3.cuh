@@ -46,4 +46,11 @@ __device__ __forceinline__ void e4m3_from_codes8(uint32_t word, int flag, uint32
     hi = prmt_b32(ev, od, 0x7362u);
 }
 
+// FLAG of subgroup k (global index over the flattened [rows, K/G_s] array):
+// one byte per FLAG, or packed two per byte (subgroup 2j in the low nibble).
+__device__ __forceinline__ int load_flag(const uint8_t *flags, int64_t k, bool packed)
+{
+    return packed ? (flags[k >> 1] >> ((k & 1) * 4)) & 0xF : flags[k];
+}
+
 }  // namespace quartz

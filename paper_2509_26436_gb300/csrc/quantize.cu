@@ -129,6 +129,7 @@ __host__ __device__ constexpr int kUnitsPerSub()
 struct UnitCodes {
     uint32_t c0, c1;   // codes of elements 0-7 and 8-15 (element k in bits 4k..4k+3)
     int flag0, flag1;  // their FLAGs (equal unless G_s = 8)
+    int flag_next;     // G_s >= 16: FLAG of the next subgroup (packed FLAG storage)
     __half s16;        // the group's fp16 scale
 };
 
@@ -171,6 +172,8 @@ __device__ __forceinline__ UnitCodes encode_unit_sym(const uint4 lo, const uint4
         u.c0 = lzs_word8<false>(w, a, r, u.flag0);
         u.c1 = lzs_word8<false>(w + 4, a + 4, r, u.flag1);
     }
+    u.flag_next = 0;
+    if (GS >= 16) u.flag_next = __shfl_down_sync(0xffffffffu, u.flag0, kUnitsPerSub<GS>());
     return u;
 }
 
@@ -210,23 +213,39 @@ __device__ __forceinline__ UnitCodes encode_unit_sym_scaled(const uint4 lo, cons
         u.c0 = lzs_word8<false>(w, a, r, u.flag0);
         u.c1 = lzs_word8<false>(w + 4, a + 4, r, u.flag1);
     }
+    u.flag_next = 0;
+    if (GS >= 16) u.flag_next = __shfl_down_sync(0xffffffffu, u.flag0, kUnitsPerSub<GS>());
     return u;
 }
 
-// Store one unit's encoding: codes, FLAG byte(s), and the scale once per group.
+// Store one unit's FLAGs: one byte per subgroup, or (packed) two per byte,
+// subgroup 2j in the low nibble of byte j; a packed byte is written by the
+// lane holding its first subgroup.
+template <int GS>
+__device__ __forceinline__ void store_unit_flags(const UnitCodes &u, int64_t unit, int lane,
+                                                 uint8_t *__restrict__ flags, bool packed)
+{
+    constexpr int ups = kUnitsPerSub<GS>();
+    if (GS == 8) {
+        if (packed)
+            flags[unit] = static_cast<uint8_t>(u.flag0 | (u.flag1 << 4));
+        else
+            reinterpret_cast<uint16_t *>(flags)[unit] = static_cast<uint16_t>(u.flag0 | (u.flag1 << 8));
+    } else if (packed) {
+        if ((lane & (2 * ups - 1)) == 0) flags[unit / (2 * ups)] = static_cast<uint8_t>(u.flag0 | (u.flag_next << 4));
+    } else if ((lane & (ups - 1)) == 0) {
+        flags[unit / ups] = static_cast<uint8_t>(u.flag0);
+    }
+}
+
+// Store one unit's encoding: codes, FLAGs, and the scale once per group.
 template <int GS>
 __device__ __forceinline__ void store_unit_sym(const UnitCodes &u, int64_t unit, int lane,
                                                uint2 *__restrict__ codes, uint8_t *__restrict__ flags,
-                                               __half *__restrict__ scales)
+                                               __half *__restrict__ scales, bool packed)
 {
     codes[unit] = make_uint2(u.c0, u.c1);
-    if (GS == 8) {
-        reinterpret_cast<uint16_t *>(flags)[unit] = static_cast<uint16_t>(u.flag0 | (u.flag1 << 8));
-    } else if (GS == 16) {
-        flags[unit] = static_cast<uint8_t>(u.flag0);
-    } else if ((lane & (kUnitsPerSub<GS>() - 1)) == 0) {
-        flags[unit / kUnitsPerSub<GS>()] = static_cast<uint8_t>(u.flag0);
-    }
+    store_unit_flags<GS>(u, unit, lane, flags, packed);
     if ((lane & 3) == 0) scales[unit >> 2] = u.s16;
 }
 
@@ -234,7 +253,7 @@ template <int GS>
 __global__ void __launch_bounds__(kThreads) quantize_sym_kernel(const uint4 *__restrict__ x, int64_t n_units,
                                                                 uint2 *__restrict__ codes,
                                                                 uint8_t *__restrict__ flags,
-                                                                __half *__restrict__ scales)
+                                                                __half *__restrict__ scales, int packed)
 {
     const int lane = threadIdx.x & 31;
     const int64_t base = static_cast<int64_t>(blockIdx.x) * (kThreads * kUnitsPerThread) + threadIdx.x;
@@ -250,7 +269,7 @@ __global__ void __launch_bounds__(kThreads) quantize_sym_kernel(const uint4 *__r
     for (int j = 0; j < kUnitsPerThread; ++j) {
         const int64_t u = base + j * kThreads;
         const UnitCodes c = encode_unit_sym<GS>(raw[j][0], raw[j][1]);
-        if (u < n_units) store_unit_sym<GS>(c, u, lane, codes, flags, scales);
+        if (u < n_units) store_unit_sym<GS>(c, u, lane, codes, flags, scales, packed != 0);
     }
 }
 
@@ -265,7 +284,7 @@ __global__ void __launch_bounds__(kThreads) quantize_row_sym_kernel(const uint4 
                                                                     unsigned short static_s16,
                                                                     uint2 *__restrict__ codes,
                                                                     uint8_t *__restrict__ flags,
-                                                                    __half *__restrict__ scales)
+                                                                    __half *__restrict__ scales, int packed)
 {
     __shared__ float warp_max[kThreads / 32];
     const int lane = threadIdx.x & 31;
@@ -309,13 +328,7 @@ __global__ void __launch_bounds__(kThreads) quantize_row_sym_kernel(const uint4 
         if (!in) continue;
         const int64_t u = row * U + j;
         codes[u] = make_uint2(c.c0, c.c1);
-        if (GS == 8) {
-            reinterpret_cast<uint16_t *>(flags)[u] = static_cast<uint16_t>(c.flag0 | (c.flag1 << 8));
-        } else if (GS == 16) {
-            flags[u] = static_cast<uint8_t>(c.flag0);
-        } else if ((lane & (kUnitsPerSub<GS>() - 1)) == 0) {
-            flags[u / kUnitsPerSub<GS>()] = static_cast<uint8_t>(c.flag0);
-        }
+        store_unit_flags<GS>(c, u, lane, flags, packed != 0);
         if ((j * 16) % group_q == 0) scales[(u * 16) / group_q] = s16;
     }
 }
@@ -329,7 +342,7 @@ template <int GS>
 __global__ void __launch_bounds__(kThreads) encode_operand_kernel(
     const uint4 *__restrict__ x, int64_t n_units, int64_t n_units_pad, int64_t units_per_row, int64_t m_pad,
     uint4 *__restrict__ a_op, float *__restrict__ a_side, uint2 *__restrict__ codes,
-    uint8_t *__restrict__ flags, __half *__restrict__ scales)
+    uint8_t *__restrict__ flags, __half *__restrict__ scales, int packed)
 {
     const int lane = threadIdx.x & 31;
     const int64_t base = static_cast<int64_t>(blockIdx.x) * (kThreads * kUnitsPerThread) + threadIdx.x;
@@ -356,7 +369,7 @@ __global__ void __launch_bounds__(kThreads) encode_operand_kernel(
         e4m3_from_codes8(c.c0, c.flag0, o.x, o.y);
         e4m3_from_codes8(c.c1, c.flag1, o.z, o.w);
         a_op[u] = o;
-        if (codes) store_unit_sym<GS>(c, u, lane, codes, flags, scales);
+        if (codes) store_unit_sym<GS>(c, u, lane, codes, flags, scales, packed != 0);
     }
 }
 
@@ -380,7 +393,7 @@ __device__ __forceinline__ void encode_chunk(const uint4 raw, int64_t chunk, boo
                                              uint8_t *__restrict__ flags,
                                              __half *__restrict__ scales,
                                              int8_t *__restrict__ zeros,
-                                             int32_t *__restrict__ gsum)
+                                             int32_t *__restrict__ gsum, bool packed)
 {
     float x[8];
     unpack8(raw, x);
@@ -445,11 +458,17 @@ __device__ __forceinline__ void encode_chunk(const uint4 raw, int64_t chunk, boo
         vsum += __shfl_xor_sync(0xffffffffu, vsum, 2);
         vsum += __shfl_xor_sync(0xffffffffu, vsum, 4);
     }
+    constexpr int kChunksPerSub = GS / 8;
+    const int flag_next = __shfl_down_sync(0xffffffffu, flag, kChunksPerSub);  // next subgroup's
     if (!valid) return;
 
     codes[chunk] = word;
-    constexpr int kChunksPerSub = GS / 8;
-    if ((lane & (kChunksPerSub - 1)) == 0) flags[chunk / kChunksPerSub] = static_cast<uint8_t>(flag);
+    if (packed) {
+        if ((lane & (2 * kChunksPerSub - 1)) == 0)
+            flags[chunk / (2 * kChunksPerSub)] = static_cast<uint8_t>(flag | (flag_next << 4));
+    } else if ((lane & (kChunksPerSub - 1)) == 0) {
+        flags[chunk / kChunksPerSub] = static_cast<uint8_t>(flag);
+    }
     if ((lane & 7) == 0) {
         const int64_t g = chunk >> 3;
         scales[g] = s16;
@@ -467,7 +486,7 @@ __global__ void __launch_bounds__(kThreads) quantize_kernel(const uint4 *__restr
                                                             uint8_t *__restrict__ flags,
                                                             __half *__restrict__ scales,
                                                             int8_t *__restrict__ zeros,
-                                                            int32_t *__restrict__ gsum)
+                                                            int32_t *__restrict__ gsum, int packed)
 {
     const int lane = threadIdx.x & 31;
     const int64_t base = static_cast<int64_t>(blockIdx.x) * (kThreads * kChunksPerThread) + threadIdx.x;
@@ -480,7 +499,7 @@ __global__ void __launch_bounds__(kThreads) quantize_kernel(const uint4 *__restr
 #pragma unroll
     for (int j = 0; j < kChunksPerThread; ++j) {
         const int64_t c = base + j * kThreads;
-        encode_chunk<GS, MODE>(raw[j], c, c < n_chunks, lane, codes, flags, scales, zeros, gsum);
+        encode_chunk<GS, MODE>(raw[j], c, c < n_chunks, lane, codes, flags, scales, zeros, gsum, packed != 0);
     }
 }
 
@@ -488,12 +507,12 @@ __global__ void __launch_bounds__(kThreads) quantize_kernel(const uint4 *__restr
 __global__ void __launch_bounds__(kThreads) dequantize_kernel(
     const uint32_t *__restrict__ codes, const uint8_t *__restrict__ flags,
     const __half *__restrict__ scales, const int8_t *__restrict__ zeros, int group_s, int group_q,
-    int64_t n_chunks, uint4 *__restrict__ out)
+    int packed, int64_t n_chunks, uint4 *__restrict__ out)
 {
     const int64_t c = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x;
     if (c >= n_chunks) return;
     const uint32_t word = codes[c];
-    const int flag = flags[(c * 8) / group_s];
+    const int flag = load_flag(flags, (c * 8) / group_s, packed != 0);
     const int64_t g = (c * 8) / group_q;
     const float s = __half2float(scales[g]);
     const int z = zeros ? zeros[g] : 0;
@@ -519,7 +538,7 @@ cudaError_t launch_q(const void *x, const quartz_encoded_t *e, cudaStream_t s)
         const int64_t blocks = (n_units + per_block - 1) / per_block;
         quantize_sym_kernel<GS><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(
             static_cast<const uint4 *>(x), n_units, reinterpret_cast<uint2 *>(e->codes), e->flags,
-            reinterpret_cast<__half *>(e->scales));
+            reinterpret_cast<__half *>(e->scales), e->p.flag_bits == 4);
         return cudaGetLastError();
     } else {
         const int64_t n_chunks = e->rows * e->K / 8;
@@ -527,7 +546,7 @@ cudaError_t launch_q(const void *x, const quartz_encoded_t *e, cudaStream_t s)
         const int64_t blocks = (n_chunks + per_block - 1) / per_block;
         quantize_kernel<GS, MODE><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(
             static_cast<const uint4 *>(x), n_chunks, reinterpret_cast<uint32_t *>(e->codes), e->flags,
-            reinterpret_cast<__half *>(e->scales), e->zeros, e->gsum);
+            reinterpret_cast<__half *>(e->scales), e->zeros, e->gsum, e->p.flag_bits == 4);
         return cudaGetLastError();
     }
 }
@@ -549,7 +568,7 @@ cudaError_t launch_row(const void *x, const quartz_encoded_t *e, int use_static,
 {
     quantize_row_sym_kernel<GS><<<static_cast<unsigned>(e->rows), kThreads, 0, s>>>(
         static_cast<const uint4 *>(x), e->K, e->p.group_q, use_static, s16, reinterpret_cast<uint2 *>(e->codes),
-        e->flags, reinterpret_cast<__half *>(e->scales));
+        e->flags, reinterpret_cast<__half *>(e->scales), e->p.flag_bits == 4);
     return cudaGetLastError();
 }
 
@@ -594,11 +613,12 @@ cudaError_t launch_encode_operand(const void *x, int64_t M, int64_t K, const qua
     uint2 *codes = enc ? reinterpret_cast<uint2 *>(enc->codes) : nullptr;
     uint8_t *flags = enc ? enc->flags : nullptr;
     __half *scales = enc ? reinterpret_cast<__half *>(enc->scales) : nullptr;
+    const int packed = enc && enc->p.flag_bits == 4;
     switch (p->group_s) {
-        case 8: encode_operand_kernel<8><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales); break;
-        case 16: encode_operand_kernel<16><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales); break;
-        case 32: encode_operand_kernel<32><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales); break;
-        default: encode_operand_kernel<64><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales); break;
+        case 8: encode_operand_kernel<8><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
+        case 16: encode_operand_kernel<16><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
+        case 32: encode_operand_kernel<32><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
+        default: encode_operand_kernel<64><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
     }
     return cudaGetLastError();
 }
@@ -611,7 +631,7 @@ cudaError_t launch_dequantize(const quartz_encoded_t *e, void *y, cudaStream_t s
     dequantize_kernel<<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(
         reinterpret_cast<const uint32_t *>(e->codes), e->flags,
         reinterpret_cast<const __half *>(e->scales),
-        e->p.mode == QUARTZ_ASYMMETRIC ? e->zeros : nullptr, e->p.group_s, e->p.group_q, n_chunks,
+        e->p.mode == QUARTZ_ASYMMETRIC ? e->zeros : nullptr, e->p.group_s, e->p.group_q, e->p.flag_bits == 4, n_chunks,
         static_cast<uint4 *>(y));
     return cudaGetLastError();
 }

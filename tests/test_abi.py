@@ -57,6 +57,14 @@ def test_encoded_sizes(lib):
     assert list(out) == [10 * 64, 10 * 8, 10 * 2 * 2, 10 * 2, 10 * 2 * 4]
     p = N.QuartzParams(64, 12, 0)
     assert lib.quartz_encoded_sizes(10, 128, C.byref(p), out) == N.QUARTZ_ERR_INVALID_ARG
+    p = N.QuartzParams(64, 16, 0, 4)             # FLAGs two per byte
+    assert lib.quartz_encoded_sizes(10, 128, C.byref(p), out) == 0
+    assert out[1] == 10 * 8 // 2
+    p = N.QuartzParams(64, 64, 0, 4)             # an odd number of subgroups in all
+    assert lib.quartz_encoded_sizes(3, 64, C.byref(p), out) == 0
+    assert out[1] == 2
+    p = N.QuartzParams(64, 16, 0, 5)
+    assert lib.quartz_encoded_sizes(10, 128, C.byref(p), out) == N.QUARTZ_ERR_INVALID_ARG
 
 
 def test_host_validation_rejects_before_launch(lib):

@@ -164,3 +164,35 @@ def test_encode_static_scale_bit_exact(Q, gs, group_q):
         e = Q.quantize_static(torch.from_numpy(x).cuda(), scale, group_s=gs, group_q=gq)
         torch.cuda.synchronize()
         _assert_encoded_equal(e, O.encode_static(x, scale, gq, gs), O.SYMMETRIC)
+
+
+@pytest.mark.parametrize("mode", [O.SYMMETRIC, O.ASYMMETRIC])
+@pytest.mark.parametrize("gs", [8, 16, 32, 64])
+@pytest.mark.parametrize("shape", [(1, 64), (3, 576), (37, 1152), (129, 4096)])
+def test_encode_packed_flags(Q, mode, gs, shape):
+    """flag_bits = 4: FLAGs two per byte, subgroup 2j in the low nibble of
+    byte j over the whole tensor; codes and scales unchanged."""
+    x = inputs.mixture_activations(*shape, seed=4000 + shape[0] + gs)
+    e = Q.quantize(torch.from_numpy(x).cuda(), group_s=gs, mode=mode, flag_bits=4)
+    torch.cuda.synchronize()
+    ref = O.encode(x, 64, gs, mode)
+    assert np.array_equal(e.flags.cpu().numpy(), O.pack_nibbles(ref.flags.reshape(-1).astype(np.int8)))
+    assert np.array_equal(e.codes.cpu().numpy(), ref.codes)
+    assert np.array_equal(e.scales.cpu().numpy().view(np.uint16), ref.scales.view(np.uint16))
+    xh = Q.dequantize(e)
+    assert torch.equal(xh.cpu(), torch.from_numpy(O.dequantize(ref).astype(np.float16)))
+
+
+@pytest.mark.parametrize("gs", [8, 16, 64])
+def test_encode_packed_flags_per_row_and_static(Q, gs):
+    x = inputs.mixture_activations(33, 3072, seed=5000 + gs)
+    xt = torch.from_numpy(x).cuda()
+    e = Q.quantize(xt, group_s=gs, group_q=3072, flag_bits=4)
+    ref = O.encode(x, 3072, gs)
+    assert np.array_equal(e.flags.cpu().numpy(), O.pack_nibbles(ref.flags.reshape(-1).astype(np.int8)))
+    assert np.array_equal(e.codes.cpu().numpy(), ref.codes)
+    s = np.float16(0.01)
+    e = Q.quantize_static(xt, s, group_s=gs, flag_bits=4)
+    ref = O.encode_static(x, s, 64, gs)
+    assert np.array_equal(e.flags.cpu().numpy(), O.pack_nibbles(ref.flags.reshape(-1).astype(np.int8)))
+    assert np.array_equal(e.codes.cpu().numpy(), ref.codes)

@@ -337,3 +337,34 @@ def test_static_activation_per_channel_weight_linear(Q):
     assert Q.device_status() == 0
     ref, rabs = O.linear(O.encode_static(xa, scale, K, 16), O.encode(xw, K, 16), with_abs=True)
     _tol_check(y.cpu().numpy(), ref, rabs, 1, "float32")
+
+
+@pytest.mark.parametrize("algo", list(ALGOS))
+@pytest.mark.parametrize("mode", [O.SYMMETRIC, O.ASYMMETRIC])
+@pytest.mark.parametrize("gs", [8, 16, 64])
+def test_linear_packed_flags_identical(Q, algo, mode, gs):
+    """Operands stored with FLAGs two per byte give the same bits as with
+    one FLAG byte per subgroup (each operand independently)."""
+    M, N, K = 200, 264, 576
+    xa = inputs.mixture_activations(M, K, seed=M + gs)
+    xw = inputs.gaussian_weights(N, K, seed=N + gs)
+    a8 = Q.quantize(torch.from_numpy(xa).cuda(), group_s=gs, mode=mode)
+    w8 = Q.encode_weights(torch.from_numpy(xw).cuda(), group_s=gs, mode=mode)
+    a4 = Q.quantize(torch.from_numpy(xa).cuda(), group_s=gs, mode=mode, flag_bits=4)
+    w4 = Q.encode_weights(torch.from_numpy(xw).cuda(), group_s=gs, mode=mode, flag_bits=4)
+    ref = Q.linear(a8, w8, out_dtype=torch.float32, algo=ALGOS[algo])
+    for a, w in ((a4, w4), (a4, w8), (a8, w4)):
+        y = Q.linear(a, w, out_dtype=torch.float32, algo=ALGOS[algo])
+        assert Q.device_status() == 0
+        assert torch.equal(y, ref)
+
+
+def test_linear_f16_packed_flag_output(Q):
+    M, N, K = 128, 256, 1152
+    x = torch.from_numpy(inputs.mixture_activations(M, K, seed=11)).cuda()
+    w = Q.encode_weights(torch.from_numpy(inputs.gaussian_weights(N, K, seed=12)).cuda(), flag_bits=4)
+    a_out = Q.empty_encoded(M, K, Q.Params(64, 16, O.SYMMETRIC, 4), x.device)
+    y = Q.linear_f16(x, w, a_out=a_out)
+    a = Q.quantize(x, flag_bits=4)
+    assert torch.equal(a_out.flags, a.flags) and torch.equal(a_out.codes, a.codes)
+    assert torch.equal(y, Q.linear(a, w))
