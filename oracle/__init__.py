@@ -10,6 +10,8 @@ Every function follows a passage of arXiv 2509.26436:
   lzs_encode      Section 3, Eq. 2 (FLAG = max(29 - clz(m), 0), shift)
   lzs_decode      Section 3 (the equal shift of a group is undone by FLAG)
   encode          Eq. 1 then Eq. 2 then nibble packing (Section 4.4 format)
+  quantize16      Section 5 LLM variant: Eq. 1 with 16-bit codes
+  lzs_encode16    Eq. 2 on 16-bit codes (FLAG 0..12)
   group_partials  Section 4.4 (integer MMA per 64-wide group)
   linear          Section 4.4 + Appendix C (16-bit group scales)
 """
@@ -66,6 +68,9 @@ def _load():
             lib.oracle_unpack_nibbles.restype = None
             lib.oracle_encode.argtypes = [P, i64, i64, i32, i32, i32, P, P, P, P, P]
             lib.oracle_quantize_static.argtypes = [P, i64, C.c_uint16, P]
+            lib.oracle_quantize16.argtypes = [P, i64, i64, i32, P, P]
+            lib.oracle_lzs_encode16.argtypes = [P, i64, i32, P, P]
+            lib.oracle_encode16.argtypes = [P, i64, i64, i32, i32, P, P, P]
             lib.oracle_encode_static.argtypes = [P, i64, i64, C.c_uint16, i32, i32, P, P, P]
             lib.oracle_decode_codes.argtypes = [P, P, i64, i64, i32, P]
             lib.oracle_dequantize.argtypes = [P, P, P, P, i64, i64, i32, i32, P]
@@ -214,6 +219,41 @@ def encode_static(x16: np.ndarray, s16, group_q: int = 64, group_s: int = 16) ->
     scales = np.empty((R, G), np.uint16)
     _check(_load().oracle_encode_static(_ptr(xb), R, K, int(np.float16(s16).view(np.uint16)), group_q,
                                         group_s, _ptr(codes), _ptr(flags), _ptr(scales)))
+    return Encoded(codes, flags, scales.view(np.float16), np.zeros((R, G), np.int8),
+                   np.zeros((R, G), np.int32), group_q, group_s, SYMMETRIC)
+
+
+def quantize16(x16: np.ndarray, group_q: int = 64):
+    """LLM variant stage 1: 16-bit codes q int16 [R, K] and fp16 scales [R, K/gq]."""
+    xb = _as_u16(x16)
+    R, K = xb.shape
+    q = np.empty((R, K), np.int16)
+    s = np.empty((R, K // group_q), np.uint16)
+    _check(_load().oracle_quantize16(_ptr(xb), R, K, group_q, _ptr(q), _ptr(s)))
+    return q, s.view(np.float16)
+
+
+def lzs_encode16(q: np.ndarray, group_s: int):
+    """Eq. 2 on 16-bit codes: (flags uint8 0..12, c int8 in [-7, 7])."""
+    q = np.ascontiguousarray(q, dtype=np.int16).ravel()
+    flags = np.empty(q.size // group_s, np.uint8)
+    c = np.empty(q.size, np.int8)
+    rc = _load().oracle_lzs_encode16(_ptr(q), q.size, group_s, _ptr(flags), _ptr(c))
+    if rc == -2:
+        raise ValueError("code -32768 has no 4-bit LZS form")
+    _check(rc)
+    return flags, c
+
+
+def encode16(x16: np.ndarray, group_q: int = 64, group_s: int = 8) -> Encoded:
+    """LLM-variant encoder (16-bit codes, FLAGs 0..12), symmetric."""
+    xb = _as_u16(x16)
+    R, K = xb.shape
+    G = K // group_q
+    codes = np.empty((R, K // 2), np.uint8)
+    flags = np.empty((R, K // group_s), np.uint8)
+    scales = np.empty((R, G), np.uint16)
+    _check(_load().oracle_encode16(_ptr(xb), R, K, group_q, group_s, _ptr(codes), _ptr(flags), _ptr(scales)))
     return Encoded(codes, flags, scales.view(np.float16), np.zeros((R, G), np.int8),
                    np.zeros((R, G), np.int32), group_q, group_s, SYMMETRIC)
 

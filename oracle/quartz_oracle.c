@@ -5,6 +5,7 @@
  * linear layer computes (arXiv 2509.26436):
  *   stage 1  per-group 8-bit min-max quantization        (Section 3, Eq. 1)
  *   stage 2  Leading Zero Suppression to 4-bit + FLAG    (Section 3, Eq. 2)
+ *   LLM variant  16-bit codes straight to 4 bits, FLAG 0..12   (Section 5)
  *   GEMM     s4 x s4 -> integer partial sums per 64-wide group, then the
  *            16-bit-scale / zero-point dequantisation    (Section 4.4;
  *            Appendix C: groups of 64 along K with 16-bit scales)
@@ -322,6 +323,87 @@ int oracle_encode_static(const uint16_t *x, int64_t rows, int64_t K, uint16_t s1
         if (rc) return rc;
         oracle_pack_nibbles(c, K, codes + row * (K / 2));
         for (int64_t g = 0; g < G; ++g) scales[row * G + g] = s16;
+    }
+    return ORACLE_OK;
+}
+
+/* ---------------------------------------------------------------------------
+ * LLM variant (Section 5, "Potential Applications to LLMs": 16-bit
+ * activations compressed directly to 4 bits, G_s = 8).  Stage 1 quantizes
+ * each group to 16-bit integers, symmetric: s = fp16(max|x| / 32767),
+ * q = clamp(round(x * r), -32767, 32767) with r = RN(1/s) (R3); a zero scale
+ * gives all-zero codes (R5).  Stage 2 is Eq. 2 unchanged on the wider codes:
+ * FLAG = max(29 - clz(m), 0) now ranges over 0..12, and the 4-bit code keeps
+ * the three bits below the leading one: c = sgn(q) (|q| >> FLAG).
+ * ------------------------------------------------------------------------- */
+int oracle_quantize16(const uint16_t *x, int64_t rows, int64_t K, int group_q, int16_t *q,
+                      uint16_t *scales)
+{
+    if (rows < 0 || K <= 0 || group_q <= 0 || K % group_q != 0) return ORACLE_ERR_ARG;
+    int64_t G = K / group_q;
+    for (int64_t row = 0; row < rows; ++row) {
+        for (int64_t g = 0; g < G; ++g) {
+            const uint16_t *xg = x + row * K + g * group_q;
+            int16_t *qg = q + row * K + g * group_q;
+            float amax = 0.0f;
+            for (int k = 0; k < group_q; ++k) {
+                float v = fabsf(oracle_half_to_float(xg[k]));
+                if (v > amax) amax = v;
+            }
+            uint16_t s16 = oracle_float_to_half_rn(amax / 32767.0f);
+            float s = oracle_half_to_float(s16);
+            if (s == 0.0f) {
+                for (int k = 0; k < group_q; ++k) qg[k] = 0;
+            } else {
+                float r = 1.0f / s;
+                for (int k = 0; k < group_q; ++k) {
+                    float t = clamp_float(oracle_half_to_float(xg[k]) * r, -65536.0f, 65536.0f);
+                    qg[k] = (int16_t)clamp_int(rne_int(t), -32767, 32767);
+                }
+            }
+            scales[row * G + g] = s16;
+        }
+    }
+    return ORACLE_OK;
+}
+
+/* Eq. 2 on 16-bit codes q [n]: flags [n/gs] (0..12), 4-bit values c [n] */
+int oracle_lzs_encode16(const int16_t *q, int64_t n, int gs, uint8_t *flags, int8_t *c)
+{
+    if (gs <= 0 || n % gs != 0) return ORACLE_ERR_ARG;
+    for (int64_t b = 0; b < n / gs; ++b) {
+        uint32_t m = 0;
+        for (int i = 0; i < gs; ++i) {
+            int v = q[b * gs + i];
+            if (v == -32768) return ORACLE_ERR_CODE128;
+            m |= (uint32_t)(v < 0 ? -v : v);
+        }
+        int flag = 29 - oracle_clz32(m);
+        if (flag < 0) flag = 0;
+        flags[b] = (uint8_t)flag;
+        for (int i = 0; i < gs; ++i) {
+            int v = q[b * gs + i];
+            int mag = v < 0 ? -v : v;
+            c[b * gs + i] = (int8_t)((v < 0 ? -1 : 1) * (mag >> flag));
+        }
+    }
+    return ORACLE_OK;
+}
+
+/* Full LLM-variant encoder: codes [rows, K/2], flags [rows, K/gs], scales [rows, K/gq] */
+int oracle_encode16(const uint16_t *x, int64_t rows, int64_t K, int gq, int gs, uint8_t *codes,
+                    uint8_t *flags, uint16_t *scales)
+{
+    if (gs <= 0 || gq % gs != 0 || K % gq != 0 || K % 2 != 0 || K > 65536) return ORACLE_ERR_ARG;
+    int16_t q[65536];
+    int8_t c[65536];
+    int64_t G = K / gq;
+    for (int64_t row = 0; row < rows; ++row) {
+        int rc = oracle_quantize16(x + row * K, 1, K, gq, q, scales + row * G);
+        if (rc) return rc;
+        rc = oracle_lzs_encode16(q, K, gs, flags + row * (K / gs), c);
+        if (rc) return rc;
+        oracle_pack_nibbles(c, K, codes + row * (K / 2));
     }
     return ORACLE_OK;
 }

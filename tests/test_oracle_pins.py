@@ -489,3 +489,115 @@ def test_static_scale_codes_follow_lzs_of_saturated_values():
     e = O.encode_static(x, np.float16(0.01), 64, 16)
     v = O.decode_values(e)
     assert np.all(np.abs(v) == 112) and np.all(e.flags == 4)
+
+
+# --- LLM variant (Section 5): 16-bit codes compressed straight to 4 bits ---
+
+def test_lzs16_exhaustive_all_16bit_codes():
+    """Every code in [-32767, 32767] at G_s = 1: FLAG = max(H(m) - 3, 0) with
+    Appendix A's bit length H, now ranging over 0..12, and FLAG is also the
+    smallest right shift that leaves the magnitude within 3 bits."""
+    q = np.arange(-32767, 32768, dtype=np.int16)
+    flags, c = O.lzs_encode16(q, 1)
+    qi = q.astype(np.int64)
+    mag = np.abs(qi)
+    H = np.array([int(m).bit_length() for m in mag])
+    f = flags.astype(np.int64)
+    assert np.array_equal(f, np.maximum(H - 3, 0))
+    f_min = np.full(mag.size, -1)
+    for t in range(15, -1, -1):
+        f_min = np.where((mag >> t) <= 7, t, f_min)
+    assert np.array_equal(f, f_min)
+    assert f.max() == 12 and (np.abs(c) <= 7).all()
+    assert np.array_equal(c.astype(np.int64), np.sign(qi) * (mag >> f))
+    v = O.lzs_decode(c, flags, 1).astype(np.int64)
+    assert np.abs(v).max() == 7 << 12 == 28672
+    assert ((mag - np.abs(v)) < (1 << f)).all() and ((mag - np.abs(v)) >= 0).all()
+    # FLAG histogram over magnitudes 0..32767 is fixed by H: 2^(F+2) codes per FLAG >= 1
+    hist = np.bincount(f[qi >= 0], minlength=13)
+    assert hist[0] == 8 and all(hist[F] == 1 << (F + 2) for F in range(1, 13))
+    # the 8-bit codes are a subset: same FLAG and value on [-127, 127]
+    f8, c8 = O.lzs_encode(np.arange(-127, 128, dtype=np.int8), 1)
+    mid = slice(32767 - 127, 32767 + 128)
+    assert np.array_equal(f8, flags[mid]) and np.array_equal(c8, c[mid])
+    with pytest.raises(ValueError):
+        O.lzs_encode16(np.array([5, -32768], np.int16), 2)
+
+
+def test_quantize16_closed_form_on_exact_units():
+    """Closed form of the 16-bit symmetric quantizer where every quantity is
+    exact: max|x| = 4 gives s = binary16(4 / 32767) = 2^-13 (the quotient is
+    2^-13 (1 + 1/32767), far below half a binary16 step), r = 2^13, and each
+    x = u 2^-13 maps to clamp(round-half-even(u), -32767, 32767).  The value
+    4.0 itself lands on 32768 and must saturate to 32767 (not wrap)."""
+    units = np.array([0, 1, -1, 0.5, 1.5, 2.5, -2.5, 3.5, 513.5, 1000.5, 1001.5, 1543, 12344,
+                      -12344, 20000, 32752, -32752, 32768, -32768])
+    x = np.zeros((1, 64), np.float16)
+    x[0, :units.size] = (units * 2.0 ** -13).astype(np.float16)
+    exact = x[0, :units.size].astype(np.float64) * 2.0 ** 13
+    assert np.array_equal(exact, units)    # binary16 holds every unit exactly
+    q, s = O.quantize16(x, 64)
+    assert s.view(np.uint16)[0, 0] == np.float16(2.0 ** -13).view(np.uint16)
+    expect = np.clip(np.round(exact), -32767, 32767)   # numpy: half to even
+    assert np.array_equal(q[0, :units.size].astype(np.int64), expect.astype(np.int64))
+    assert q[0, list(units).index(32768)] == 32767 and q[0, list(units).index(-32768)] == -32767
+    assert (q[0, units.size:] == 0).all()
+
+
+def test_quantize16_against_exact_rounding():
+    """16-bit codes against exact rational rounding of x / s: equal except
+    within 2^-12 of a half-integer (binary32 reciprocal-multiply at 16-bit
+    magnitudes), |x - s q| <= s / 2 for unsaturated elements, and the largest
+    element of a group lands on 32767 up to the relative rounding error of
+    the binary16 scale."""
+    x = inputs.laplace_activations(4, 512, seed=13)
+    q, s = O.quantize16(x, 64)
+    mism = 0
+    for i in range(4):
+        for g in range(8):
+            sv = Fraction(float(s[i, g]))
+            xs = x[i, g * 64:(g + 1) * 64].astype(np.float64)
+            for k in range(64):
+                t = Fraction(float(xs[k])) / sv
+                fl = t.numerator // t.denominator
+                frac = t - fl
+                ex = fl + (1 if frac > Fraction(1, 2) or (frac == Fraction(1, 2) and fl % 2) else 0)
+                ex = max(-32767, min(32767, ex))
+                if ex != int(q[i, g * 64 + k]):
+                    mism += 1
+                    assert abs(frac - Fraction(1, 2)) < Fraction(1, 2 ** 12)
+                if abs(t) < 32767:
+                    assert abs(Fraction(float(xs[k])) - sv * int(q[i, g * 64 + k])) <= sv / 2 * (1 + Fraction(1, 2 ** 10))
+            # the binary16 scale is off max|x| / 32767 by at most half its own
+            # spacing (2^-24 absolute once it is subnormal, i.e. max|x| < 2)
+            rel = float(np.spacing(s[i, g])) / 2 / float(s[i, g])
+            top = np.abs(q[i, g * 64:(g + 1) * 64].astype(np.int64)).max()
+            assert 32767 * (1 - rel) / (1 + rel) - 1 <= top <= 32767
+    assert mism <= 4
+
+
+def test_encode16_truncation_bound_and_linear_exact():
+    """LLM-variant encoding (G_s = 8): every decoded value is the 16-bit code
+    truncated toward zero by its subgroup's FLAG (error < 2^FLAG steps, no
+    sign error), and the W4A4 linear of two such operands equals the binary64
+    product of the dequantised operands.  All-saturated rows make each
+    64-wide group sum 64 x 28672^2 (> 2^31): an int32 accumulator would wrap."""
+    xa = inputs.mixture_activations(6, 256, seed=17)
+    xw = inputs.gaussian_weights(10, 256, seed=18)
+    xa[0, :] = 8.0
+    xw[0, :] = -2.0
+    a = O.encode16(xa, 64, 8)
+    w = O.encode16(xw, 64, 8)
+    assert a.flags.max() == 12
+    q, _ = O.quantize16(xa, 64)
+    v = O.decode_values(a).astype(np.int64)
+    qi = q.astype(np.int64)
+    F = np.repeat(a.flags.astype(np.int64), 8, axis=1)
+    err = np.abs(qi) - np.abs(v)
+    assert (err >= 0).all() and (err < (1 << F)).all()
+    assert ((np.sign(v) == np.sign(qi)) | (v == 0)).all()
+    y = O.linear(a, w)
+    ref = O.dequantize(a) @ O.dequantize(w).T
+    assert np.allclose(y, ref, rtol=1e-12, atol=1e-12 * np.abs(ref).max())
+    P = O.group_partials(O.decode_values(a), O.decode_values(w), 64)
+    assert P[0, 0, 0] == -64 * 28672 * 28672 and abs(P[0, 0, 0]) > 2 ** 31
