@@ -51,6 +51,9 @@ def parse():
     p.add_argument("--compare-algos", action="store_true",
                    help="also time the three GEMM algorithms (tcgen05, simt, shift) on each layer")
     p.add_argument("--layers", default="", help="comma-separated subset of layer names (profiling)")
+    p.add_argument("--llm", action="store_true",
+                   help="also time the LLM variant (Section 5: 16-bit codes straight to 4 bits, "
+                        "G_s = 8) on LLaMA-2-7B block linears")
     return p.parse_args()
 
 
@@ -423,6 +426,9 @@ def run_ours(args):
             algos[name] = per
         assert Q.device_status() == 0
 
+    # ---- LLM variant (optional) ---------------------------------------------
+    llm = run_llm_variant(args, Q, inputs, dev, n_sm, sm_mhz, peak_src) if args.llm else None
+
     # ---- end to end through the public API with host buffers ---------------
     # Each (step, layer) unit copies its activations from pinned host memory,
     # encodes them, runs the linear layer and copies the fp16 output back to
@@ -513,10 +519,78 @@ def run_ours(args):
         "gpu_launches": launches_per_step * args.steps,
         "fused": fused,
         "gemm_algos": algos,
+        "llm_variant": llm,
         "e2e": e2e,
         "cpu_baseline": cpu,
     }
     print(json.dumps(out), flush=True)
+
+
+LLM_GROUP_S = 8
+
+
+def run_llm_variant(args, Q, inputs, dev, n_sm, sm_mhz, peak_src):
+    """One step = encode (16-bit codes, G_s = 8) + linear of each of the four
+    LLaMA-2-7B block linears at 2048 tokens; per-kernel CUDA-event times."""
+    import torch
+    layers = inputs.CONFIG_LLM
+    nl = len(layers)
+    x_dev = [torch.from_numpy(l.activations()).to(dev) for l in layers]
+    enc_w = [Q.encode_weights(torch.from_numpy(l.weights()).to(dev), group_s=LLM_GROUP_S, code_bits=16)
+             for l in layers]
+    enc_a = [Q.empty_encoded(l.M, l.K, Q.Params(GROUP_Q, LLM_GROUP_S, code_bits=16), dev) for l in layers]
+    y_dev = [torch.empty((l.M, l.N), dtype=torch.float16, device=dev) for l in layers]
+    workspace = torch.empty(max(Q.linear_workspace_size(l.M, l.N, l.K, enc_a[0].params) for l in layers),
+                            dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+    ev = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
+    steps = max(1, min(args.steps, 10))
+
+    def step(rec=None):
+        for i in range(nl):
+            if rec is not None:
+                rec[i][0].record(stream)
+            Q.quantize(x_dev[i], out=enc_a[i], group_s=LLM_GROUP_S, code_bits=16)
+            if rec is not None:
+                rec[i][1].record(stream)
+            Q.linear(enc_a[i], enc_w[i], out=y_dev[i], workspace=workspace,
+                     gemm_events=None if rec is None else rec[i][2:])
+
+    for _ in range(max(1, args.warmup)):
+        step()
+    torch.cuda.synchronize()
+    recs = [[(ev(), ev(), ev(), ev()) for _ in range(nl)] for _ in range(steps)]
+    t0, t1 = ev(), ev()
+    t0.record(stream)
+    for k in range(steps):
+        step(recs[k])
+    t1.record(stream)
+    torch.cuda.synchronize()
+    assert Q.device_status() == 0
+    t_step = t0.elapsed_time(t1) / 1e3 / steps
+    gemm_ms = [statistics.mean(r[i][2].elapsed_time(r[i][3]) for r in recs) for i in range(nl)]
+    quant_ms = [statistics.mean(r[i][0].elapsed_time(r[i][1]) for r in recs) for i in range(nl)]
+    ops = sum(l.ops for l in layers)
+    t_gemm = sum(gemm_ms) / 1e3
+    # accumulator-shift GEMM: per output and 8-wide subgroup two dp4a, one
+    # shift and one 64-bit add, against the 128 integer lanes of each SM
+    int_ops = sum(l.M * l.N * (l.K // LLM_GROUP_S) * 4 for l in layers)
+    int_peak = n_sm * FP32_LANES_PER_SM * sm_mhz * 1e6 / 1e12
+    enc_bytes = sum(l.M * l.K * encode_bytes_per_elem(LLM_GROUP_S, GROUP_Q) for l in layers)
+    return {"workload": "llama2_7b_block_linears", "tokens": layers[0].M,
+            "layers": [f"{l.name}:{l.K}->{l.N}" for l in layers], "group_q": GROUP_Q,
+            "group_s": LLM_GROUP_S, "code_bits": 16, "gemm": "accumulator-shift (64-bit group sums)",
+            "value": ops / t_step / 1e12, "unit": "TOPS", "ms_per_step": t_step * 1e3, "steps": steps,
+            "gemm_tops": ops / t_gemm / 1e12, "gemm_per_layer_ms": gemm_ms,
+            "roofline": {"bound": "alu", "kernel": "gemm_shift_kernel",
+                         "achieved": int_ops / t_gemm / 1e12, "peak": int_peak, "unit": "Top/s",
+                         "frac": int_ops / t_gemm / 1e12 / int_peak,
+                         "work": "2 dp4a + 1 shift + 1 add per output per 8-wide subgroup",
+                         "peak_source": f"derived: {n_sm} SMs x {FP32_LANES_PER_SM} lanes x "
+                                        f"{sm_mhz:.0f} MHz ({peak_src} max SM clock)"},
+            "encode": {"kernel": "quantize_kernel<8, sym, wide>", "per_layer_ms": quant_ms,
+                       "gbs": enc_bytes / (sum(quant_ms) / 1e3) / 1e9},
+            "inputs": "seeded synthetic Laplace(0,0.05), 0.2% channels x100; weights N(0,0.02)"}
 
 
 def main():

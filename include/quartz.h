@@ -73,6 +73,13 @@ typedef struct {
     int32_t flag_bits; /* FLAG storage: 0 or 8 = one byte per subgroup (Section
                         * 4.4); 4 = two FLAGs per byte (values 0..4 fit in 4
                         * bits), 4 + 4/G_s + 16/group_q bits per element */
+    int32_t code_bits; /* width of the stage-1 codes: 0 or 8 = Eq. 1's 8-bit
+                        * codes; 16 = the LLM variant of Section 5 (16-bit
+                        * activations compressed straight to 4 bits; the
+                        * paper uses G_s = 8): s = fp16(max|x| / 32767),
+                        * q = clamp(round(x/s), -32767, 32767), Eq. 2 gives
+                        * FLAG in 0..12 and decoded values up to 7 << 12.
+                        * 16 requires SYMMETRIC mode and group_q == 64. */
 } quartz_params_t;
 
 /* One encoded tensor of `rows` rows and `K` columns (Section 4.4: "packed
@@ -80,7 +87,8 @@ typedef struct {
  * memory owned by the caller; sizes in elements:
  *   codes  uint8 [rows, K/2]        two's-complement 4-bit codes in [-7, 7],
  *                                   element 2j in the low nibble of byte j
- *   flags  uint8 [rows, K/group_s]  FLAG of Eq. 2, values 0..4; with
+ *   flags  uint8 [rows, K/group_s]  FLAG of Eq. 2, values 0..4 (0..12 with
+ *                                   16-bit codes); with
  *                                   flag_bits = 4: uint8 [ceil(rows*K/group_s
  *                                   / 2)], FLAG of subgroup 2j (counted over
  *                                   the whole tensor, row after row) in the
@@ -119,17 +127,19 @@ int32_t quartz_encoded_sizes(int64_t rows, int64_t K, const quartz_params_t *p, 
  * K, then Eq. 2 per subgroup of p->group_s, then nibble packing.
  *   x_f16  fp16 [out->rows, out->K] device, 16-byte aligned
  *   out    describes the destination: rows, K, p and the buffers above
- * Requirements: rows >= 0, K > 0, K % 64 == 0, group_q == 64, group_s in
- * {8,16,32,64}.  rows == 0 is a no-op. */
+ * Requirements: rows >= 0, K > 0, K % 64 == 0, group_q == 64 (or K: one
+ * scale per row, symmetric), group_s in {8,16,32,64}.  With code_bits = 16
+ * the stage-1 codes are 16 bits wide (the LLM variant above).  rows == 0 is
+ * a no-op. */
 int32_t quartz_quantize(const void *x_f16, const quartz_encoded_t *out, void *stream);
 
 /* Static per-tensor quantization (Appendix C: the latent-diffusion models
  * quantize activations with one static, calibrated scale per tensor): Eq. 1
  * with the given fp16 scale `scale_f16` (bits; finite, >= 0) for every
  * element instead of a scale computed from the data, then Eq. 2.  Elements
- * beyond 127 * scale saturate to +-127 before LZS.  SYMMETRIC mode; any
- * group_q; every stored scale of `out` is `scale_f16`.  A zero scale gives
- * all-zero codes. */
+ * beyond 127 * scale saturate to +-127 before LZS.  SYMMETRIC mode, 8-bit
+ * codes (else QUARTZ_ERR_UNSUPPORTED); any group_q; every stored scale of
+ * `out` is `scale_f16`.  A zero scale gives all-zero codes. */
 int32_t quartz_quantize_static(const void *x_f16, uint16_t scale_f16, const quartz_encoded_t *out, void *stream);
 
 /* The same encoder applied to nn.Linear weights [N, K] (one quantization
@@ -161,7 +171,10 @@ size_t quartz_linear_workspace_size(int64_t M, int64_t N, int64_t K, const quart
  *              16-byte aligned, owned by the caller; contents are scratch
  * Requirements: N % 8 == 0, K % 64 == 0, M >= 0.  The per-group partials
  * P_g are exact; the scaled sum is accumulated in binary32 and rounded once
- * to y_type. */
+ * to y_type.  Operands with 16-bit stage-1 codes (code_bits = 16, both
+ * operands) run on QUARTZ_ALGO_SHIFT only, with 64-bit integer partials (a
+ * group sum reaches 64 * 28672^2 > 2^31); quartz_linear, whose algorithm
+ * is TCGEN05, returns QUARTZ_ERR_UNSUPPORTED for them. */
 int32_t quartz_linear(const quartz_encoded_t *a, const quartz_encoded_t *w, const void *bias_f16,
                       void *y, int32_t y_type, void *workspace, size_t workspace_bytes,
                       void *stream);
@@ -170,6 +183,8 @@ int32_t quartz_linear(const quartz_encoded_t *a, const quartz_encoded_t *w, cons
  *   partials          NULL, or int32 [M, N] device buffer that receives
  *                     P_g[m, n] of group `partials_group` (0 <= g < K/64), the
  *                     raw integer MMA result before any scale or zero point
+ *                     (8-bit codes only: QUARTZ_ERR_UNSUPPORTED with 16-bit
+ *                     codes, whose partials need 64 bits)
  *   algo              quartz_algo_t: which GEMM kernel runs
  *   gemm_event_begin  NULL, or a cudaEvent_t recorded on `stream` right before
  *   gemm_event_end    / right after the GEMM kernel (after operand expansion),
@@ -195,8 +210,8 @@ int32_t quartz_linear_ex(const quartz_encoded_t *a, const quartz_encoded_t *w,
  * quartz_quantize followed by quartz_linear with the same parameters.
  *   x_f16      fp16 [M, K] device, 16-byte aligned
  *   w          encoded weights [N, K]; its params (group_s, mode) are used
- *              for the activations; SYMMETRIC mode only (else
- *              QUARTZ_ERR_UNSUPPORTED)
+ *              for the activations; SYMMETRIC mode, group_q == 64 and 8-bit
+ *              codes only (else QUARTZ_ERR_UNSUPPORTED)
  *   bias_f16, y, y_type, workspace, workspace_bytes: as quartz_linear
  *              (quartz_linear_workspace_size(M, N, K, &w->p) bytes)
  *   a_out      NULL, or an encoded [M, K] tensor with w's params that also

@@ -36,14 +36,16 @@ class Params:
     """group_q: min-max group along K (64, Appendix C, or K for one scale per
     row); group_s: LZS subgroup G_s (8/16/32/64, Section 3); mode: SYMMETRIC
     or ASYMMETRIC; flag_bits: 8 (one FLAG byte per subgroup) or 4 (two FLAGs
-    per byte)."""
+    per byte); code_bits: 8 (Eq. 1's codes) or 16 (the LLM variant of
+    Section 5: 16-bit codes compressed straight to 4 bits, symmetric)."""
     group_q: int = 64
     group_s: int = 16
     mode: int = SYMMETRIC
     flag_bits: int = 8
+    code_bits: int = 8
 
     def c(self) -> N.QuartzParams:
-        return N.QuartzParams(self.group_q, self.group_s, self.mode, self.flag_bits)
+        return N.QuartzParams(self.group_q, self.group_s, self.mode, self.flag_bits, self.code_bits)
 
 
 class Encoded:
@@ -99,23 +101,25 @@ def _check_f16(x, name):
 
 
 def quantize(x, group_s: int = 16, mode: int = SYMMETRIC, out: Encoded | None = None,
-             stream=None, _entry="quartz_quantize", group_q: int = 64, flag_bits: int = 8) -> Encoded:
+             stream=None, _entry="quartz_quantize", group_q: int = 64, flag_bits: int = 8,
+             code_bits: int = 8) -> Encoded:
     """Eq. 1 + Eq. 2 on fp16 activations [M, K] (K % 64 == 0); group_q = 64
-    or K (one scale per row)."""
+    or K (one scale per row); code_bits = 16 for Section 5's LLM variant."""
     _check_f16(x, "x")
     rows, K = x.shape
-    e = out if out is not None else empty_encoded(rows, K, Params(group_q, group_s, mode, flag_bits), x.device)
+    e = out if out is not None else empty_encoded(rows, K, Params(group_q, group_s, mode, flag_bits, code_bits),
+                                                  x.device)
     ec = e.c()
     N.check(getattr(N.load(), _entry)(x.data_ptr(), C.byref(ec), _stream(stream)), _entry)
     return e
 
 
 def encode_weights(w, group_s: int = 16, mode: int = SYMMETRIC, out: Encoded | None = None,
-                   stream=None, group_q: int = 64, flag_bits: int = 8) -> Encoded:
+                   stream=None, group_q: int = 64, flag_bits: int = 8, code_bits: int = 8) -> Encoded:
     """The same encoder applied to nn.Linear weights [N, K], run offline
     (group_q = K gives per-output-channel scales)."""
     return quantize(w, group_s, mode, out, stream, _entry="quartz_encode_weights", group_q=group_q,
-                    flag_bits=flag_bits)
+                    flag_bits=flag_bits, code_bits=code_bits)
 
 
 def quantize_static(x, scale, group_s: int = 16, group_q: int = 64, out: Encoded | None = None,
@@ -151,15 +155,19 @@ _OUT = {"float16": OUT_F16, "bfloat16": OUT_BF16, "float32": OUT_F32}
 
 
 def linear(a: Encoded, w: Encoded, bias=None, out_dtype=None, out=None, workspace=None,
-           partials_group: int | None = None, algo: int = ALGO_TCGEN05, stream=None,
+           partials_group: int | None = None, algo: int | None = None, stream=None,
            gemm_events=None):
     """W4A4 QuaRTZ linear: y = dequant(a) @ dequant(w)^T (+ bias), computed as
     exact integer group partials scaled by the 16-bit group scales.
 
     Returns y, or (y, partials) when `partials_group` is given (int32 [M, N]
     raw integer MMA sums of that 64-wide K group).  `gemm_events` = a pair
-    of torch.cuda.Event recorded around the GEMM kernel alone."""
+    of torch.cuda.Event recorded around the GEMM kernel alone.  `algo`
+    defaults to ALGO_TCGEN05, or ALGO_SHIFT (the only GEMM built for them)
+    for operands with 16-bit codes."""
     torch = _torch()
+    if algo is None:
+        algo = ALGO_SHIFT if a.params.code_bits == 16 else ALGO_TCGEN05
     out_dtype = out_dtype or torch.float16
     M, Nn = a.rows, w.rows
     dev = a.codes.device

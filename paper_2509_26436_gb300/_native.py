@@ -39,7 +39,7 @@ _SZ = C.c_size_t
 
 class QuartzParams(C.Structure):
     _fields_ = [("group_q", C.c_int32), ("group_s", C.c_int32), ("mode", C.c_int32),
-                ("flag_bits", C.c_int32)]
+                ("flag_bits", C.c_int32), ("code_bits", C.c_int32)]
 
 
 class QuartzEncoded(C.Structure):

@@ -24,8 +24,13 @@ int32_t check_params(const quartz_params_t *p)
         return QUARTZ_ERR_INVALID_ARG;
     if (p->group_q <= 0 || p->group_q % p->group_s != 0) return QUARTZ_ERR_INVALID_ARG;
     if (p->group_q % 64 != 0) return QUARTZ_ERR_UNSUPPORTED;
+    if (p->code_bits != 0 && p->code_bits != 8 && p->code_bits != 16) return QUARTZ_ERR_INVALID_ARG;
+    // 16-bit stage-1 codes (Section 5 LLM variant): symmetric groups of 64
+    if (p->code_bits == 16 && (p->mode != QUARTZ_SYMMETRIC || p->group_q != 64)) return QUARTZ_ERR_UNSUPPORTED;
     return QUARTZ_OK;
 }
+
+bool wide_codes(const quartz_params_t &p) { return p.code_bits == 16; }
 
 int32_t check_shape(int64_t rows, int64_t K, const quartz_params_t *p)
 {
@@ -91,7 +96,7 @@ const char *quartz_status_string(int32_t status)
     }
 }
 
-int32_t quartz_version(void) { return (1 << 16) | 2; }
+int32_t quartz_version(void) { return (1 << 16) | 3; }
 
 int32_t quartz_encoded_sizes(int64_t rows, int64_t K, const quartz_params_t *p, size_t out[5])
 {
@@ -121,7 +126,7 @@ int32_t quartz_quantize_static(const void *x_f16, uint16_t scale_f16, const quar
 {
     int32_t rc = check_encoded(out);
     if (rc) return rc;
-    if (out->p.mode != QUARTZ_SYMMETRIC) return QUARTZ_ERR_UNSUPPORTED;
+    if (out->p.mode != QUARTZ_SYMMETRIC || wide_codes(out->p)) return QUARTZ_ERR_UNSUPPORTED;
     // a finite, non-negative fp16 scale
     if ((scale_f16 & 0x8000u) && scale_f16 != 0x8000u) return QUARTZ_ERR_INVALID_ARG;
     if ((scale_f16 & 0x7C00u) == 0x7C00u) return QUARTZ_ERR_INVALID_ARG;
@@ -168,8 +173,11 @@ int32_t quartz_linear_ex(const quartz_encoded_t *a, const quartz_encoded_t *w,
     rc = check_encoded(w);
     if (rc) return rc;
     if (a->K != w->K || a->p.group_q != w->p.group_q || a->p.group_s != w->p.group_s ||
-        a->p.mode != w->p.mode)
+        a->p.mode != w->p.mode || wide_codes(a->p) != wide_codes(w->p))
         return QUARTZ_ERR_INVALID_ARG;
+    const bool wide = wide_codes(a->p);
+    // 16-bit codes: decoded values up to 7 << 12 and group sums beyond int32
+    if (wide && (o.algo != QUARTZ_ALGO_SHIFT || partials)) return QUARTZ_ERR_UNSUPPORTED;
     const bool per_row = a->p.group_q != 64;  // group_q == K (check_shape allows nothing else)
     if (per_row && o.algo != QUARTZ_ALGO_TCGEN05) return QUARTZ_ERR_UNSUPPORTED;
     const int64_t M = a->rows, N = w->rows, K = a->K;
@@ -201,7 +209,7 @@ int32_t quartz_linear_ex(const quartz_encoded_t *a, const quartz_encoded_t *w,
     if (algo == QUARTZ_ALGO_SIMT)
         e = launch_gemm_simt(ws, M, N, K, a->p.mode, bias_f16, y, y_type, partials, partials_group, s);
     else if (algo == QUARTZ_ALGO_SHIFT)
-        e = launch_gemm_shift(ws, a, w, bias_f16, y, y_type, partials, partials_group, s);
+        e = launch_gemm_shift(ws, a, w, bias_f16, y, y_type, partials, partials_group, s, wide);
     else
         e = launch_gemm_tcgen05(ws, M, N, K, a->p.mode, bias_f16, y, y_type, partials,
                                 partials_group, dev_err, s, per_row);
@@ -223,7 +231,7 @@ int32_t quartz_linear_f16(const void *x_f16, int64_t M, const quartz_encoded_t *
 {
     int32_t rc = check_encoded(w);
     if (rc) return rc;
-    if (w->p.mode != QUARTZ_SYMMETRIC || w->p.group_q != 64) return QUARTZ_ERR_UNSUPPORTED;
+    if (w->p.mode != QUARTZ_SYMMETRIC || w->p.group_q != 64 || wide_codes(w->p)) return QUARTZ_ERR_UNSUPPORTED;
     const int64_t N = w->rows, K = w->K;
     rc = check_shape(M, K, &w->p);
     if (rc) return rc;

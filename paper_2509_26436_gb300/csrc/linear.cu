@@ -27,6 +27,7 @@
 // floating-point pipe.)
 #include <cuda.h>
 #include <cuda_fp16.h>
+#include <type_traits>
 #include <cuda_bf16.h>
 #include <cuda_fp8.h>
 
@@ -915,9 +916,11 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const __nv_fp8_e4m3 *__r
 //    products run on dp4a over the codes placed in the high nibble of each
 //    byte (int8 value 16c, so a dot product is 256 x the code dot product).
 //    The dequant arithmetic is the SIMT kernel's.  64x64 output tile per
-//    256-thread block, 4x4 outputs per thread.
+//    256-thread block, 4x4 outputs per thread.  WIDE: operands with 16-bit
+//    stage-1 codes (Section 5 LLM variant), FLAGs up to 12, so a shifted
+//    subgroup product reaches 392 << 24 and the group sums are 64-bit.
 // ---------------------------------------------------------------------------
-template <int GS, int MODE, int OUT>
+template <int GS, int MODE, int OUT, bool WIDE>
 __global__ void __launch_bounds__(256) gemm_shift_kernel(const uint32_t *__restrict__ a_codes,
                                                          const uint8_t *__restrict__ a_flags,
                                                          const uint32_t *__restrict__ w_codes,
@@ -954,7 +957,8 @@ __global__ void __launch_bounds__(256) gemm_shift_kernel(const uint32_t *__restr
             fw[r][j] = (n0 + r < args.N) ? load_flag(w_flags, (n0 + r) * flags_per_row + col, w_packed != 0) : 0;
         }
         __syncthreads();
-        int p[4][4] = {};
+        using Acc = typename std::conditional<WIDE, long long, int>::type;
+        Acc p[4][4] = {};
 #pragma unroll
         for (int j = 0; j < kSub; ++j) {
 #pragma unroll
@@ -966,7 +970,7 @@ __global__ void __launch_bounds__(256) gemm_shift_kernel(const uint32_t *__restr
                     for (int q = 0; q < kWordsPerSub; ++q)
                         dot = __dp4a(static_cast<int>(sa[ty * 4 + i][j * kWordsPerSub + q]),
                                      static_cast<int>(sw[tx * 4 + jj][j * kWordsPerSub + q]), dot);
-                    p[i][jj] += (dot >> 8) * (1 << (fa[ty * 4 + i][j] + fw[tx * 4 + jj][j]));
+                    p[i][jj] += static_cast<Acc>(dot >> 8) << (fa[ty * 4 + i][j] + fw[tx * 4 + jj][j]);
                 }
         }
 #pragma unroll
@@ -979,7 +983,8 @@ __global__ void __launch_bounds__(256) gemm_shift_kernel(const uint32_t *__restr
                 const int n = n0 + tx * 4 + jj;
                 if (n >= args.N) continue;
                 float P = static_cast<float>(p[i][jj]);
-                if (args.partials && g == args.partials_group) args.partials[(int64_t)m * args.N + n] = p[i][jj];
+                if (!WIDE && args.partials && g == args.partials_group)
+                    args.partials[(int64_t)m * args.N + n] = static_cast<int32_t>(p[i][jj]);
                 if (MODE == QUARTZ_ASYMMETRIC) {
                     const float za = args.a_side[a_plane + (int64_t)g * args.m_pad + perm32(m)];
                     const float ua = args.a_side[2 * a_plane + (int64_t)g * args.m_pad + perm32(m)];
@@ -1230,49 +1235,50 @@ cudaError_t launch_gemm_simt(const LinearWorkspace &ws, int64_t M, int64_t N, in
 }
 
 namespace {
-template <int GS, int MODE, int OUT>
+template <int GS, int MODE, int OUT, bool WIDE>
 cudaError_t launch_shift(const quartz_encoded_t *a, const quartz_encoded_t *w, const GemmArgs &args,
                          cudaStream_t s)
 {
     dim3 grid(static_cast<unsigned>((args.N + 63) / 64), static_cast<unsigned>((args.M + 63) / 64));
-    gemm_shift_kernel<GS, MODE, OUT><<<grid, 256, 0, s>>>(
+    gemm_shift_kernel<GS, MODE, OUT, WIDE><<<grid, 256, 0, s>>>(
         reinterpret_cast<const uint32_t *>(a->codes), a->flags, reinterpret_cast<const uint32_t *>(w->codes),
         w->flags, args, static_cast<int>(a->K), a->p.flag_bits == 4, w->p.flag_bits == 4);
     return cudaGetLastError();
 }
 
-template <int GS, int MODE>
+template <int GS, int MODE, bool WIDE>
 cudaError_t launch_shift_out(const quartz_encoded_t *a, const quartz_encoded_t *w, const GemmArgs &args,
                              int y_type, cudaStream_t s)
 {
     switch (y_type) {
-        case QUARTZ_OUT_F16: return launch_shift<GS, MODE, QUARTZ_OUT_F16>(a, w, args, s);
-        case QUARTZ_OUT_BF16: return launch_shift<GS, MODE, QUARTZ_OUT_BF16>(a, w, args, s);
-        default: return launch_shift<GS, MODE, QUARTZ_OUT_F32>(a, w, args, s);
+        case QUARTZ_OUT_F16: return launch_shift<GS, MODE, QUARTZ_OUT_F16, WIDE>(a, w, args, s);
+        case QUARTZ_OUT_BF16: return launch_shift<GS, MODE, QUARTZ_OUT_BF16, WIDE>(a, w, args, s);
+        default: return launch_shift<GS, MODE, QUARTZ_OUT_F32, WIDE>(a, w, args, s);
     }
 }
 
 template <int GS>
 cudaError_t launch_shift_mode(const quartz_encoded_t *a, const quartz_encoded_t *w, const GemmArgs &args,
-                              int y_type, cudaStream_t s)
+                              int y_type, bool wide, cudaStream_t s)
 {
-    return a->p.mode == QUARTZ_ASYMMETRIC ? launch_shift_out<GS, QUARTZ_ASYMMETRIC>(a, w, args, y_type, s)
-                                          : launch_shift_out<GS, QUARTZ_SYMMETRIC>(a, w, args, y_type, s);
+    if (wide) return launch_shift_out<GS, QUARTZ_SYMMETRIC, true>(a, w, args, y_type, s);
+    return a->p.mode == QUARTZ_ASYMMETRIC ? launch_shift_out<GS, QUARTZ_ASYMMETRIC, false>(a, w, args, y_type, s)
+                                          : launch_shift_out<GS, QUARTZ_SYMMETRIC, false>(a, w, args, y_type, s);
 }
 }  // namespace
 
 cudaError_t launch_gemm_shift(const LinearWorkspace &ws, const quartz_encoded_t *a, const quartz_encoded_t *w,
                               const void *bias, void *y, int y_type, int32_t *partials, int partials_group,
-                              cudaStream_t s)
+                              cudaStream_t s, bool wide)
 {
     const int64_t M = a->rows, N = w->rows, K = a->K;
     if (M == 0) return cudaSuccess;
     const GemmArgs args = make_args(ws, M, N, K, bias, y, y_type, partials, partials_group, nullptr);
     switch (a->p.group_s) {
-        case 8: return launch_shift_mode<8>(a, w, args, y_type, s);
-        case 16: return launch_shift_mode<16>(a, w, args, y_type, s);
-        case 32: return launch_shift_mode<32>(a, w, args, y_type, s);
-        default: return launch_shift_mode<64>(a, w, args, y_type, s);
+        case 8: return launch_shift_mode<8>(a, w, args, y_type, wide, s);
+        case 16: return launch_shift_mode<16>(a, w, args, y_type, wide, s);
+        case 32: return launch_shift_mode<32>(a, w, args, y_type, wide, s);
+        default: return launch_shift_mode<64>(a, w, args, y_type, wide, s);
     }
 }
 

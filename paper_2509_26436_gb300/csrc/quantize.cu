@@ -14,8 +14,9 @@
 // permutes, shifted right by FLAG in one 32-bit shift, and the sign applied
 // per byte in 4-bit two's complement.
 //
-// Asymmetric mode uses one thread per 8-element chunk (eight lanes per group)
-// with the same arithmetic written per element.
+// Asymmetric mode, and the 16-bit-code LLM variant of Section 5, use one
+// thread per 8-element chunk (eight lanes per group) with the same arithmetic
+// written per element.
 #include <cuda_fp16.h>
 
 #include "lzs_e4m3.cuh"
@@ -386,8 +387,10 @@ __device__ __forceinline__ void unpack8(const uint4 &raw, float (&x)[8])
 
 // Encode the 8 elements of one chunk.  All 32 lanes must call this together
 // (the group and subgroup reductions are warp shuffles); `valid` only gates
-// the stores.
-template <int GS, int MODE>
+// the stores.  WIDE selects the LLM variant of Section 5 (symmetric only):
+// stage 1 quantizes to 16-bit codes (32767 levels) and Eq. 2 compresses them
+// straight to 4 bits, FLAG = max(29 - clz(m), 0) in 0..12.
+template <int GS, int MODE, bool WIDE>
 __device__ __forceinline__ void encode_chunk(const uint4 raw, int64_t chunk, bool valid, int lane,
                                              uint32_t *__restrict__ codes,
                                              uint8_t *__restrict__ flags,
@@ -407,7 +410,7 @@ __device__ __forceinline__ void encode_chunk(const uint4 raw, int64_t chunk, boo
         amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, 1));
         amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, 2));
         amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, 4));
-        s32 = __fdiv_rn(amax, 127.0f);
+        s32 = __fdiv_rn(amax, WIDE ? 32767.0f : 127.0f);
     } else {
         float hi = 0.f;  // the range always contains 0
 #pragma unroll
@@ -432,8 +435,10 @@ __device__ __forceinline__ void encode_chunk(const uint4 raw, int64_t chunk, boo
     uint32_t m = 0;
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
-        const float t = fminf(fmaxf(__fmul_rn(x[i], r), -1024.0f), 1024.0f);
-        q[i] = min(max(__float2int_rn(t) + z, -127), 127);
+        constexpr float kT = WIDE ? 65536.0f : 1024.0f;  // beyond the cap, below int overflow
+        constexpr int kQ = WIDE ? 32767 : 127;
+        const float t = fminf(fmaxf(__fmul_rn(x[i], r), -kT), kT);
+        q[i] = min(max(__float2int_rn(t) + z, -kQ), kQ);
         m |= static_cast<uint32_t>(abs(q[i]));
     }
 
@@ -479,7 +484,7 @@ __device__ __forceinline__ void encode_chunk(const uint4 raw, int64_t chunk, boo
     }
 }
 
-template <int GS, int MODE>
+template <int GS, int MODE, bool WIDE>
 __global__ void __launch_bounds__(kThreads) quantize_kernel(const uint4 *__restrict__ x,
                                                             int64_t n_chunks,
                                                             uint32_t *__restrict__ codes,
@@ -499,7 +504,8 @@ __global__ void __launch_bounds__(kThreads) quantize_kernel(const uint4 *__restr
 #pragma unroll
     for (int j = 0; j < kChunksPerThread; ++j) {
         const int64_t c = base + j * kThreads;
-        encode_chunk<GS, MODE>(raw[j], c, c < n_chunks, lane, codes, flags, scales, zeros, gsum, packed != 0);
+        encode_chunk<GS, MODE, WIDE>(raw[j], c, c < n_chunks, lane, codes, flags, scales, zeros, gsum,
+                                     packed != 0);
     }
 }
 
@@ -529,10 +535,10 @@ __global__ void __launch_bounds__(kThreads) dequantize_kernel(
     out[c] = make_uint4(o[0], o[1], o[2], o[3]);
 }
 
-template <int GS, int MODE>
+template <int GS, int MODE, bool WIDE = false>
 cudaError_t launch_q(const void *x, const quartz_encoded_t *e, cudaStream_t s)
 {
-    if constexpr (MODE == QUARTZ_SYMMETRIC) {
+    if constexpr (MODE == QUARTZ_SYMMETRIC && !WIDE) {
         const int64_t n_units = e->rows * e->K / 16;
         const int64_t per_block = kThreads * kUnitsPerThread;
         const int64_t blocks = (n_units + per_block - 1) / per_block;
@@ -544,7 +550,7 @@ cudaError_t launch_q(const void *x, const quartz_encoded_t *e, cudaStream_t s)
         const int64_t n_chunks = e->rows * e->K / 8;
         const int64_t per_block = kThreads * kChunksPerThread;
         const int64_t blocks = (n_chunks + per_block - 1) / per_block;
-        quantize_kernel<GS, MODE><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(
+        quantize_kernel<GS, MODE, WIDE><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(
             static_cast<const uint4 *>(x), n_chunks, reinterpret_cast<uint32_t *>(e->codes), e->flags,
             reinterpret_cast<__half *>(e->scales), e->zeros, e->gsum, e->p.flag_bits == 4);
         return cudaGetLastError();
@@ -559,6 +565,16 @@ cudaError_t launch_q_mode(const void *x, const quartz_encoded_t *e, cudaStream_t
         case 16: return launch_q<16, MODE>(x, e, s);
         case 32: return launch_q<32, MODE>(x, e, s);
         default: return launch_q<64, MODE>(x, e, s);
+    }
+}
+
+cudaError_t launch_q_wide(const void *x, const quartz_encoded_t *e, cudaStream_t s)
+{
+    switch (e->p.group_s) {
+        case 8: return launch_q<8, QUARTZ_SYMMETRIC, true>(x, e, s);
+        case 16: return launch_q<16, QUARTZ_SYMMETRIC, true>(x, e, s);
+        case 32: return launch_q<32, QUARTZ_SYMMETRIC, true>(x, e, s);
+        default: return launch_q<64, QUARTZ_SYMMETRIC, true>(x, e, s);
     }
 }
 
@@ -595,6 +611,7 @@ cudaError_t launch_quantize(const void *x, const quartz_encoded_t *out, cudaStre
 {
     static_assert(kGroupQ == 64, "one quantization group is 8 lanes x 8 elements");
     if (out->rows == 0) return cudaSuccess;
+    if (out->p.code_bits == 16) return launch_q_wide(x, out, s);   // Section 5 LLM variant
     if (out->p.group_q != kGroupQ) return launch_quantize_row(x, out, 0, 0, s);  // group_q == K
     return out->p.mode == QUARTZ_SYMMETRIC ? launch_q_mode<QUARTZ_SYMMETRIC>(x, out, s)
                                            : launch_q_mode<QUARTZ_ASYMMETRIC>(x, out, s);

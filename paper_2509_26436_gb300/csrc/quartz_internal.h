@@ -53,10 +53,11 @@ void linear_workspace_carve(void *base, int64_t M, int64_t N, int64_t K, int mod
 // `expand` false only the scales are transposed (accumulator-shift GEMM).
 cudaError_t launch_prepare(const quartz_encoded_t *a, const quartz_encoded_t *w, const LinearWorkspace &ws,
                            cudaStream_t s, bool expand = true);
-// The paper's accumulator-shift schedule on CUDA cores, from the packed codes.
+// The paper's accumulator-shift schedule on CUDA cores, from the packed codes;
+// `wide`: 16-bit stage-1 codes (FLAGs up to 12, 64-bit group sums).
 cudaError_t launch_gemm_shift(const LinearWorkspace &ws, const quartz_encoded_t *a, const quartz_encoded_t *w,
                               const void *bias, void *y, int y_type, int32_t *partials, int partials_group,
-                              cudaStream_t s);
+                              cudaStream_t s, bool wide = false);
 // Fused activation path (quantize.cu, symmetric mode): Eq. 1 + Eq. 2 on fp16
 // x [M, K] written straight into the workspace as E4M3 operand and scale
 // side values; `enc` (may be NULL) also receives the encoded tensor.

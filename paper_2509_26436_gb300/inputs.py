@@ -18,7 +18,10 @@ available; these recipes stand in for them:
 * the encode sweep: an i.i.d. mixture 89% Laplace(0,0.05), 10% N(0,0.3),
   1% U(-8,8);
 * UNet convolutions: SiLU(N(0,1)) feature maps with sparse x10 channels,
-  lowered to a GEMM by im2col with K ordered (kh, kw, c_in), padding 1.
+  lowered to a GEMM by im2col with K ordered (kh, kw, c_in), padding 1;
+* LLM layers (Section 5 variant; the paper's Qwen2 / LLaMA checkpoints and
+  its perplexity corpus are not available): the Laplace recipe with 0.2% of
+  the channels x100, the few very large channels of LLM hidden states.
 """
 from __future__ import annotations
 
@@ -150,7 +153,17 @@ CONFIG4 = [
     Layer("flux_fc2", 18432, 3072, 12288, 4, 3, outlier_frac=0.001, outlier_scale=50.0),
 ]
 
+# LLaMA-2-7B decoder block linears (Section 5 LLM variant, 16-bit codes,
+# G_s = 8) at a 2048-token prefill: hidden 4096, MLP 11008 (gate and up
+# fused), activations with a few strong outlier channels.
+CONFIG_LLM = [
+    Layer("llama2_qkv", 2048, 12288, 4096, 5, 0, outlier_frac=0.002, outlier_scale=100.0),
+    Layer("llama2_o", 2048, 4096, 4096, 5, 1, outlier_frac=0.002, outlier_scale=100.0),
+    Layer("llama2_gate_up", 2048, 22016, 4096, 5, 2, outlier_frac=0.002, outlier_scale=100.0),
+    Layer("llama2_down", 2048, 4096, 11008, 5, 3, outlier_frac=0.002, outlier_scale=100.0),
+]
+
 # Encode sweep sizes: 1M, 16M and 128M fp16 elements as [rows, 4096].
 ENCODE_SWEEP = [(2 ** 20 // 4096, 4096), (4096, 4096), (32768, 4096)]
 
-GEMM_CONFIGS = {0: CONFIG0, 2: CONFIG2, 3: CONFIG3, 4: CONFIG4}
+GEMM_CONFIGS = {0: CONFIG0, 2: CONFIG2, 3: CONFIG3, 4: CONFIG4, 5: CONFIG_LLM}

@@ -134,6 +134,38 @@ def test_linear_validation(lib):
     assert lib.quartz_selftest_timeout(10, None) == N.QUARTZ_ERR_INVALID_ARG
 
 
+def test_code_bits_validation(lib):
+    """16-bit stage-1 codes (Section 5 LLM variant): symmetric groups of 64;
+    only the accumulator-shift GEMM takes them, without int32 partials."""
+    out = (C.c_size_t * 5)()
+    for bits, rc in ((0, 0), (8, 0), (16, 0), (12, N.QUARTZ_ERR_INVALID_ARG), (4, N.QUARTZ_ERR_INVALID_ARG)):
+        p = N.QuartzParams(64, 8, 0, 8, bits)
+        assert lib.quartz_encoded_sizes(10, 128, C.byref(p), out) == rc
+    p = N.QuartzParams(64, 8, 0, 4, 16)          # FLAGs 0..12 still fit in 4 bits
+    assert lib.quartz_encoded_sizes(10, 128, C.byref(p), out) == 0 and out[1] == 10 * 16 // 2
+    q = lib.quartz_quantize
+
+    def enc(rows, K, gq=64, mode=0, bits=16):
+        return N.QuartzEncoded(0x1000, 0x1000, 0x1000, 0x1000, 0x1000, rows, K, N.QuartzParams(gq, 8, mode, 8, bits))
+
+    assert q(0x1000, C.byref(enc(4, 128, mode=1)), None) == N.QUARTZ_ERR_UNSUPPORTED   # asymmetric
+    assert q(0x1000, C.byref(enc(4, 128, gq=128)), None) == N.QUARTZ_ERR_UNSUPPORTED   # per-row scales
+    assert lib.quartz_quantize_static(0x1000, 0x3C00, C.byref(enc(4, 128)), None) == N.QUARTZ_ERR_UNSUPPORTED
+    L = lib.quartz_linear_ex
+
+    def lin(a, w, algo, part=None):
+        o = N.QuartzLinearOpts(part, 0, algo, None, None)
+        return L(C.byref(a), C.byref(w), None, 0x2000, 0, 0x3000, 1 << 30, C.byref(o), None)
+
+    a, w = enc(16, 128), enc(24, 128)
+    assert lin(a, w, N.ALGO_TCGEN05) == N.QUARTZ_ERR_UNSUPPORTED
+    assert lin(a, w, N.ALGO_SIMT) == N.QUARTZ_ERR_UNSUPPORTED
+    assert lin(a, w, N.ALGO_SHIFT, part=0x4000) == N.QUARTZ_ERR_UNSUPPORTED
+    assert lin(a, enc(24, 128, bits=8), N.ALGO_SHIFT) == N.QUARTZ_ERR_INVALID_ARG  # mixed widths
+    assert lib.quartz_linear_f16(0x1000, 16, C.byref(w), None, 0x2000, 0, None, 0x3000, 1 << 30,
+                                 None) == N.QUARTZ_ERR_UNSUPPORTED
+
+
 def test_linear_f16_validation(lib):
     """Host checks of the fused activation path: nothing is launched on error."""
     L = lib.quartz_linear_f16

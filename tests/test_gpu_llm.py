@@ -1,0 +1,192 @@
+"""GPU parity of the LLM variant (Section 5: 16-bit activations compressed
+straight to 4 bits, G_s = 8) against the CPU oracle.
+
+* Encoder: codes, FLAGs (0..12) and fp16 scale bits bit-exact against
+  oracle.encode16, including saturated groups, subnormal scales and packed
+  FLAG storage; the dequantiser bit-exact against the oracle's binary64
+  value rounded once to fp16.
+* Linear (accumulator-shift GEMM, 64-bit group sums): outputs against the
+  oracle's binary64 y.  Tolerance from the kernel's arithmetic: P_g is exact
+  in 64 bits and is rounded once to binary32; s_a*(s_w*P_g) adds two more
+  roundings and the G-term running sum G more, so |y_gpu - y| <=
+  (G + 5) 2^-24 sum_g |s_a s_w D_g| before the output conversion (relative
+  2^-11 for fp16, 2^-8 for bf16).
+"""
+import numpy as np
+import pytest
+
+import oracle as O
+from paper_2509_26436_gb300 import inputs
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+REL = {"float16": 1e-3, "bfloat16": 4e-3, "float32": 1e-5}
+
+
+@pytest.fixture(scope="module")
+def Q():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2509_26436_gb300 as Q
+    return Q
+
+
+def _enc(Q, x16, gs=8, flag_bits=8):
+    e = Q.quantize(torch.from_numpy(x16).cuda(), group_s=gs, code_bits=16, flag_bits=flag_bits)
+    torch.cuda.synchronize()
+    return e
+
+
+def _assert_equal(e, ref):
+    assert np.array_equal(e.codes.cpu().numpy(), ref.codes)
+    assert np.array_equal(e.flags.cpu().numpy(), ref.flags)
+    assert np.array_equal(e.scales.cpu().numpy().view(np.uint16), ref.scales.view(np.uint16))
+
+
+def _pack_flags(flags):
+    f = flags.reshape(-1).astype(np.uint8)
+    if f.size % 2:
+        f = np.concatenate([f, np.zeros(1, np.uint8)])
+    return f[0::2] | (f[1::2] << 4)
+
+
+@pytest.mark.parametrize("gs", [8, 16, 32, 64])
+@pytest.mark.parametrize("shape", [(1, 64), (3, 128), (37, 1152), (129, 4096), (1000, 640)])
+def test_encode16_bit_exact(Q, gs, shape):
+    x = inputs.mixture_activations(*shape, seed=5000 + shape[0] + gs)
+    _assert_equal(_enc(Q, x, gs), O.encode16(x, 64, gs))
+
+
+def test_encode16_edge_values(Q):
+    """Zero groups, scale underflow, subnormal scales (max|x| < 2), fp16
+    extremes (x r lands on 32768 and saturates), ties and all-equal groups."""
+    rows = [np.zeros(256), np.full(256, 1e-7), np.linspace(-3e-4, 3e-4, 256),
+            np.concatenate([np.full(64, 65504.0), -np.full(64, 65504.0), np.full(64, 4.0),
+                            np.linspace(-4, 4, 64)]),
+            np.concatenate([np.full(64, 0.5), np.arange(64) * 2.0 ** -13, np.arange(64) * 1.5 * 2.0 ** -14,
+                            -np.arange(64) * 2.0 ** -10]),
+            np.tile([1.0, -1.0, 1e-3, -1e-3], 64)]
+    x = np.stack(rows).astype(np.float16)
+    for gs in (8, 16, 32, 64):
+        ref = O.encode16(x, 64, gs)
+        _assert_equal(_enc(Q, x, gs), ref)
+    assert ref.flags.max() == 12
+
+
+@pytest.mark.parametrize("gs", [8, 16, 64])
+@pytest.mark.parametrize("shape", [(1, 64), (3, 576), (129, 4096)])
+def test_encode16_packed_flags(Q, gs, shape):
+    x = inputs.mixture_activations(*shape, seed=5100 + gs)
+    ref = O.encode16(x, 64, gs)
+    e = _enc(Q, x, gs, flag_bits=4)
+    assert np.array_equal(e.codes.cpu().numpy(), ref.codes)
+    assert np.array_equal(e.flags.cpu().numpy(), _pack_flags(ref.flags))
+    assert np.array_equal(e.scales.cpu().numpy().view(np.uint16), ref.scales.view(np.uint16))
+
+
+@pytest.mark.parametrize("gs", [8, 32])
+def test_dequantize16_bit_exact(Q, gs):
+    x = inputs.laplace_activations(77, 1152, seed=5200 + gs, outlier_frac=0.002, outlier_scale=100.0)
+    e = _enc(Q, x, gs)
+    y = Q.dequantize(e)
+    torch.cuda.synchronize()
+    ref = O.dequantize(O.encode16(x, 64, gs)).astype(np.float16)
+    assert np.array_equal(y.cpu().numpy().view(np.uint16), ref.view(np.uint16))
+
+
+def _tol_check(y_gpu, y_ref, y_abs, G, dtype_name):
+    y_gpu = y_gpu.astype(np.float64)
+    tol = REL[dtype_name] * np.abs(y_ref) + (G + 5) * 2.0 ** -24 * y_abs + 2.0 ** -24
+    err = np.abs(y_gpu - y_ref)
+    bad = err > tol
+    assert not bad.any(), (f"{bad.sum()} of {bad.size} outside tolerance; worst "
+                           f"{(err / np.maximum(tol, 1e-30)).max():.3g}x")
+
+
+def _linear16(Q, xa, xw, gs, bias=None, out_dtype="float16", flag_bits=8):
+    a = _enc(Q, xa, gs, flag_bits)
+    w = Q.encode_weights(torch.from_numpy(xw).cuda(), group_s=gs, code_bits=16, flag_bits=flag_bits)
+    b = None if bias is None else torch.from_numpy(bias).cuda()
+    y = Q.linear(a, w, b, out_dtype=getattr(torch, out_dtype))
+    assert Q.device_status() == 0
+    return y.float().cpu().numpy()
+
+
+@pytest.mark.parametrize("gs", [8, 16, 64])
+@pytest.mark.parametrize("M,N,K", [(1, 8, 64), (200, 264, 640), (129, 520, 1216)])
+def test_linear16_ragged_shapes(Q, gs, M, N, K):
+    xa = inputs.laplace_activations(M, K, seed=5300 + M, outlier_frac=0.002, outlier_scale=100.0)
+    xw = inputs.gaussian_weights(N, K, seed=5301 + N)
+    bias = np.random.default_rng(M).normal(0, 0.1, N).astype(np.float16)
+    y = _linear16(Q, xa, xw, gs, bias)
+    ref, rabs = O.linear(O.encode16(xa, 64, gs), O.encode16(xw, 64, gs), bias, with_abs=True)
+    _tol_check(y, ref, rabs, K // 64, "float16")
+
+
+@pytest.mark.parametrize("out_dtype", ["float16", "bfloat16", "float32"])
+def test_linear16_out_dtypes_and_packed_flags(Q, out_dtype):
+    xa = inputs.laplace_activations(256, 1152, seed=5400, outlier_frac=0.002, outlier_scale=100.0)
+    xw = inputs.gaussian_weights(384, 1152, seed=5401)
+    ref, rabs = O.linear(O.encode16(xa, 64, 8), O.encode16(xw, 64, 8), with_abs=True)
+    y = _linear16(Q, xa, xw, 8, out_dtype=out_dtype)
+    _tol_check(y, ref, rabs, 18, out_dtype)
+    y4 = _linear16(Q, xa, xw, 8, out_dtype=out_dtype, flag_bits=4)
+    assert np.array_equal(y4, y)
+
+
+def test_linear16_group_sums_beyond_int32(Q):
+    """Saturated rows decode to +-28672 everywhere, so a 64-wide group sum is
+    64 x 28672^2 > 2^31; rows with mixed FLAG 0..12 subgroups interleave."""
+    xa = inputs.mixture_activations(40, 512, seed=5500)
+    xw = inputs.gaussian_weights(64, 512, seed=5501)
+    xa[0, :] = 8.0
+    xa[1, ::2], xa[1, 1::2] = -3.0, 3.0
+    xw[0, :] = -2.0
+    xw[1, :] = 0.5
+    xa[2, :] = (np.arange(512) % 8 - 3.5).astype(np.float16) * np.float16(2.0 ** -12)
+    ea, ew = O.encode16(xa, 64, 8), O.encode16(xw, 64, 8)
+    P = O.group_partials(O.decode_values(ea), O.decode_values(ew), 64)
+    assert np.abs(P).max() > 2 ** 31
+    y = _linear16(Q, xa, xw, 8, out_dtype="float32")
+    ref, rabs = O.linear(ea, ew, with_abs=True)
+    _tol_check(y, ref, rabs, 8, "float32")
+
+
+def test_linear16_other_algorithms_rejected(Q):
+    """Only the 64-bit accumulator-shift GEMM takes 16-bit codes; mixing
+    8-bit and 16-bit operands is an argument error."""
+    x = torch.from_numpy(inputs.mixture_activations(16, 128, seed=5600)).cuda()
+    a = Q.quantize(x, group_s=8, code_bits=16)
+    w = Q.encode_weights(x[:8].contiguous(), group_s=8, code_bits=16)
+    w8 = Q.encode_weights(x[:8].contiguous(), group_s=8)
+    for algo in (Q.ALGO_TCGEN05, Q.ALGO_SIMT):
+        with pytest.raises(Q.QuartzError, match="UNSUPPORTED"):
+            Q.linear(a, w, algo=algo)
+    with pytest.raises(Q.QuartzError, match="UNSUPPORTED"):
+        Q.linear(a, w, algo=Q.ALGO_SHIFT, partials_group=0)
+    with pytest.raises(Q.QuartzError, match="INVALID_ARG"):
+        Q.linear(a, w8, algo=Q.ALGO_SHIFT)
+    torch.cuda.synchronize()
+    assert Q.device_status() == 0
+
+
+@pytest.mark.parametrize("layer", inputs.CONFIG_LLM, ids=[l.name for l in inputs.CONFIG_LLM])
+def test_linear16_llama_layers_sampled(Q, layer):
+    """Full-size LLaMA-2-7B block linears (G_s = 8, fp16 out) in the
+    benchmark's launch configuration: codes of sampled rows bit-exact and
+    their outputs within tolerance of the oracle."""
+    xa, xw = layer.activations(), layer.weights()
+    a = Q.quantize(torch.from_numpy(xa).cuda(), group_s=8, code_bits=16)
+    w = Q.encode_weights(torch.from_numpy(xw).cuda(), group_s=8, code_bits=16)
+    y = Q.linear(a, w)
+    assert Q.device_status() == 0
+    rows = np.unique(np.concatenate([np.arange(3), np.arange(layer.M - 3, layer.M),
+                                     np.linspace(3, layer.M - 4, 6).astype(np.int64)]))
+    rt = torch.from_numpy(rows).cuda()
+    ea, ew = O.encode16(xa[rows], 64, 8), O.encode16(xw, 64, 8)
+    assert np.array_equal(a.codes[rt].cpu().numpy(), ea.codes)
+    assert np.array_equal(a.flags[rt].cpu().numpy(), ea.flags)
+    assert np.array_equal(w.codes.cpu().numpy(), ew.codes)
+    ref, rabs = O.linear(ea, ew, with_abs=True)
+    _tol_check(y[rt].float().cpu().numpy(), ref, rabs, layer.K // 64, "float16")
