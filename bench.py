@@ -427,7 +427,7 @@ def run_ours(args):
         assert Q.device_status() == 0
 
     # ---- LLM variant (optional) ---------------------------------------------
-    llm = run_llm_variant(args, Q, inputs, dev, n_sm, sm_mhz, peak_src) if args.llm else None
+    llm = run_llm_variant(args, Q, inputs, dev, n_sm, sm_mhz, peak_src, fp8_peak) if args.llm else None
 
     # ---- end to end through the public API with host buffers ---------------
     # Each (step, layer) unit copies its activations from pinned host memory,
@@ -529,9 +529,10 @@ def run_ours(args):
 LLM_GROUP_S = 8
 
 
-def run_llm_variant(args, Q, inputs, dev, n_sm, sm_mhz, peak_src):
+def run_llm_variant(args, Q, inputs, dev, n_sm, sm_mhz, peak_src, fp8_peak):
     """One step = encode (16-bit codes, G_s = 8) + linear of each of the four
-    LLaMA-2-7B block linears at 2048 tokens; per-kernel CUDA-event times."""
+    LLaMA-2-7B block linears at 2048 tokens; per-kernel CUDA-event times, for
+    the tcgen05 GEMM (E5M2 operands) and the exact accumulator-shift GEMM."""
     import torch
     layers = inputs.CONFIG_LLM
     nl = len(layers)
@@ -544,50 +545,67 @@ def run_llm_variant(args, Q, inputs, dev, n_sm, sm_mhz, peak_src):
                             dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream()
     ev = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
-    steps = max(1, min(args.steps, 10))
-
-    def step(rec=None):
-        for i in range(nl):
-            if rec is not None:
-                rec[i][0].record(stream)
-            Q.quantize(x_dev[i], out=enc_a[i], group_s=LLM_GROUP_S, code_bits=16)
-            if rec is not None:
-                rec[i][1].record(stream)
-            Q.linear(enc_a[i], enc_w[i], out=y_dev[i], workspace=workspace,
-                     gemm_events=None if rec is None else rec[i][2:])
-
-    for _ in range(max(1, args.warmup)):
-        step()
-    torch.cuda.synchronize()
-    recs = [[(ev(), ev(), ev(), ev()) for _ in range(nl)] for _ in range(steps)]
-    t0, t1 = ev(), ev()
-    t0.record(stream)
-    for k in range(steps):
-        step(recs[k])
-    t1.record(stream)
-    torch.cuda.synchronize()
-    assert Q.device_status() == 0
-    t_step = t0.elapsed_time(t1) / 1e3 / steps
-    gemm_ms = [statistics.mean(r[i][2].elapsed_time(r[i][3]) for r in recs) for i in range(nl)]
-    quant_ms = [statistics.mean(r[i][0].elapsed_time(r[i][1]) for r in recs) for i in range(nl)]
     ops = sum(l.ops for l in layers)
-    t_gemm = sum(gemm_ms) / 1e3
-    # accumulator-shift GEMM: per output and 8-wide subgroup two dp4a, one
-    # shift and one 64-bit add, against the 128 integer lanes of each SM
-    int_ops = sum(l.M * l.N * (l.K // LLM_GROUP_S) * 4 for l in layers)
-    int_peak = n_sm * FP32_LANES_PER_SM * sm_mhz * 1e6 / 1e12
+    alu_peak = n_sm * FP32_LANES_PER_SM * sm_mhz * 1e6 / 1e12
     enc_bytes = sum(l.M * l.K * encode_bytes_per_elem(LLM_GROUP_S, GROUP_Q) for l in layers)
+
+    def timed(algo, steps):
+        def step(rec=None):
+            for i in range(nl):
+                if rec is not None:
+                    rec[i][0].record(stream)
+                Q.quantize(x_dev[i], out=enc_a[i], group_s=LLM_GROUP_S, code_bits=16)
+                if rec is not None:
+                    rec[i][1].record(stream)
+                Q.linear(enc_a[i], enc_w[i], out=y_dev[i], workspace=workspace, algo=algo,
+                         gemm_events=None if rec is None else rec[i][2:])
+
+        for _ in range(max(3, args.warmup)):
+            step()
+        torch.cuda.synchronize()
+        recs = [[(ev(), ev(), ev(), ev()) for _ in range(nl)] for _ in range(steps)]
+        t0, t1 = ev(), ev()
+        t0.record(stream)
+        for k in range(steps):
+            step(recs[k])
+        t1.record(stream)
+        torch.cuda.synchronize()
+        assert Q.device_status() == 0
+        t_step = t0.elapsed_time(t1) / 1e3 / steps
+        gemm_ms = [statistics.mean(r[i][2].elapsed_time(r[i][3]) for r in recs) for i in range(nl)]
+        quant_ms = [statistics.mean(r[i][0].elapsed_time(r[i][1]) for r in recs) for i in range(nl)]
+        return t_step, gemm_ms, quant_ms
+
+    t_tc, gemm_tc, quant_ms = timed(Q.ALGO_TCGEN05, max(3, min(args.steps, 50)))
+    t_sh, gemm_sh, _ = timed(Q.ALGO_SHIFT, max(1, min(args.steps, 5)))
+    t_gemm = sum(gemm_tc) / 1e3
+    epi_ops = sum(2 * l.M * l.N * (l.K // GROUP_Q) for l in layers)
+    t_floor_alu, t_floor_tensor = epi_ops / (alu_peak * 1e12), ops / (fp8_peak * 1e12)
+    alu_view = {"achieved": epi_ops / t_gemm / 1e12, "peak": alu_peak, "unit": "Top/s",
+                "frac": epi_ops / t_gemm / 1e12 / alu_peak,
+                "work": "2 fp32 ops (multiply + fused multiply-add) per output per 64-wide group"}
+    tensor_view = {"achieved": ops / t_gemm / 1e12, "peak": fp8_peak, "unit": "TFLOP/s",
+                   "frac": ops / t_gemm / 1e12 / fp8_peak, "work": "2 M N K FP8 (E5M2) MMA flops"}
+    bound = "alu" if t_floor_alu >= t_floor_tensor else "tensor"
+    main, other = (alu_view, tensor_view) if bound == "alu" else (tensor_view, alu_view)
+    sh_ops = sum(l.M * l.N * (l.K // LLM_GROUP_S) * 4 for l in layers)
+    t_sh_gemm = sum(gemm_sh) / 1e3
     return {"workload": "llama2_7b_block_linears", "tokens": layers[0].M,
             "layers": [f"{l.name}:{l.K}->{l.N}" for l in layers], "group_q": GROUP_Q,
-            "group_s": LLM_GROUP_S, "code_bits": 16, "gemm": "accumulator-shift (64-bit group sums)",
-            "value": ops / t_step / 1e12, "unit": "TOPS", "ms_per_step": t_step * 1e3, "steps": steps,
-            "gemm_tops": ops / t_gemm / 1e12, "gemm_per_layer_ms": gemm_ms,
-            "roofline": {"bound": "alu", "kernel": "gemm_shift_kernel",
-                         "achieved": int_ops / t_gemm / 1e12, "peak": int_peak, "unit": "Top/s",
-                         "frac": int_ops / t_gemm / 1e12 / int_peak,
-                         "work": "2 dp4a + 1 shift + 1 add per output per 8-wide subgroup",
-                         "peak_source": f"derived: {n_sm} SMs x {FP32_LANES_PER_SM} lanes x "
-                                        f"{sm_mhz:.0f} MHz ({peak_src} max SM clock)"},
+            "group_s": LLM_GROUP_S, "code_bits": 16, "gemm": "tcgen05 (E5M2 operands)",
+            "value": ops / t_tc / 1e12, "unit": "TOPS", "ms_per_step": t_tc * 1e3,
+            "gemm_tops": ops / t_gemm / 1e12, "gemm_per_layer_ms": gemm_tc,
+            "roofline": dict(main, bound=bound, kernel="gemm_tcgen05_kernel",
+                             **{("tensor" if bound == "alu" else "alu"): other},
+                             floors_ms={"alu": t_floor_alu * 1e3, "tensor": t_floor_tensor * 1e3}),
+            "shift": {"gemm": "accumulator-shift (exact 64-bit group sums)", "value": ops / t_sh / 1e12,
+                      "ms_per_step": t_sh * 1e3, "gemm_per_layer_ms": gemm_sh,
+                      "roofline": {"bound": "alu", "kernel": "gemm_shift_kernel",
+                                   "achieved": sh_ops / t_sh_gemm / 1e12, "peak": alu_peak,
+                                   "unit": "Top/s", "frac": sh_ops / t_sh_gemm / 1e12 / alu_peak,
+                                   "work": "2 dp4a + 1 shift + 1 add per output per 8-wide subgroup"}},
+            "peak_source": f"alu: {n_sm} SMs x {FP32_LANES_PER_SM} lanes x {sm_mhz:.0f} MHz ({peak_src} "
+                           f"max SM clock); tensor: {peak_src} bf16 burst x {FP8_OVER_BF16}",
             "encode": {"kernel": "quantize_kernel<8, sym, wide>", "per_layer_ms": quant_ms,
                        "gbs": enc_bytes / (sum(quant_ms) / 1e3) / 1e9},
             "inputs": "seeded synthetic Laplace(0,0.05), 0.2% channels x100; weights N(0,0.02)"}

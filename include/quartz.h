@@ -172,9 +172,11 @@ size_t quartz_linear_workspace_size(int64_t M, int64_t N, int64_t K, const quart
  * Requirements: N % 8 == 0, K % 64 == 0, M >= 0.  The per-group partials
  * P_g are exact; the scaled sum is accumulated in binary32 and rounded once
  * to y_type.  Operands with 16-bit stage-1 codes (code_bits = 16, both
- * operands) run on QUARTZ_ALGO_SHIFT only, with 64-bit integer partials (a
- * group sum reaches 64 * 28672^2 > 2^31); quartz_linear, whose algorithm
- * is TCGEN05, returns QUARTZ_ERR_UNSUPPORTED for them. */
+ * operands; decoded values up to 7 << 12, a group sum up to
+ * 64 * 28672^2 > 2^31): QUARTZ_ALGO_SHIFT keeps P_g exact in 64-bit
+ * integers; TCGEN05 (E5M2 operands) multiplies exactly but sums each group
+ * in the tensor cores' fp32 accumulator, so P_g is then rounded like any
+ * fp32 sum; SIMT returns QUARTZ_ERR_UNSUPPORTED. */
 int32_t quartz_linear(const quartz_encoded_t *a, const quartz_encoded_t *w, const void *bias_f16,
                       void *y, int32_t y_type, void *workspace, size_t workspace_bytes,
                       void *stream);

@@ -155,19 +155,17 @@ _OUT = {"float16": OUT_F16, "bfloat16": OUT_BF16, "float32": OUT_F32}
 
 
 def linear(a: Encoded, w: Encoded, bias=None, out_dtype=None, out=None, workspace=None,
-           partials_group: int | None = None, algo: int | None = None, stream=None,
+           partials_group: int | None = None, algo: int = ALGO_TCGEN05, stream=None,
            gemm_events=None):
     """W4A4 QuaRTZ linear: y = dequant(a) @ dequant(w)^T (+ bias), computed as
     exact integer group partials scaled by the 16-bit group scales.
 
     Returns y, or (y, partials) when `partials_group` is given (int32 [M, N]
     raw integer MMA sums of that 64-wide K group).  `gemm_events` = a pair
-    of torch.cuda.Event recorded around the GEMM kernel alone.  `algo`
-    defaults to ALGO_TCGEN05, or ALGO_SHIFT (the only GEMM built for them)
-    for operands with 16-bit codes."""
+    of torch.cuda.Event recorded around the GEMM kernel alone.  Operands
+    with 16-bit codes (Section 5 LLM variant) run on ALGO_TCGEN05 (E5M2
+    operands, fp32 group sums) or ALGO_SHIFT (exact 64-bit group sums)."""
     torch = _torch()
-    if algo is None:
-        algo = ALGO_SHIFT if a.params.code_bits == 16 else ALGO_TCGEN05
     out_dtype = out_dtype or torch.float16
     M, Nn = a.rows, w.rows
     dev = a.codes.device

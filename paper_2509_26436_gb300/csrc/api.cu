@@ -176,8 +176,9 @@ int32_t quartz_linear_ex(const quartz_encoded_t *a, const quartz_encoded_t *w,
         a->p.mode != w->p.mode || wide_codes(a->p) != wide_codes(w->p))
         return QUARTZ_ERR_INVALID_ARG;
     const bool wide = wide_codes(a->p);
-    // 16-bit codes: decoded values up to 7 << 12 and group sums beyond int32
-    if (wide && (o.algo != QUARTZ_ALGO_SHIFT || partials)) return QUARTZ_ERR_UNSUPPORTED;
+    // 16-bit codes: decoded values up to 7 << 12 (E5M2 operands for the
+    // tensor cores, no E4M3 SIMT path) and group sums beyond int32
+    if (wide && (o.algo == QUARTZ_ALGO_SIMT || partials)) return QUARTZ_ERR_UNSUPPORTED;
     const bool per_row = a->p.group_q != 64;  // group_q == K (check_shape allows nothing else)
     if (per_row && o.algo != QUARTZ_ALGO_TCGEN05) return QUARTZ_ERR_UNSUPPORTED;
     const int64_t M = a->rows, N = w->rows, K = a->K;
@@ -212,7 +213,7 @@ int32_t quartz_linear_ex(const quartz_encoded_t *a, const quartz_encoded_t *w,
         e = launch_gemm_shift(ws, a, w, bias_f16, y, y_type, partials, partials_group, s, wide);
     else
         e = launch_gemm_tcgen05(ws, M, N, K, a->p.mode, bias_f16, y, y_type, partials,
-                                partials_group, dev_err, s, per_row);
+                                partials_group, dev_err, s, per_row, wide);
     if (e == cudaSuccess && o.gemm_event_end)
         e = cudaEventRecord(static_cast<cudaEvent_t>(o.gemm_event_end), s);
     return map_cuda(e);

@@ -25,6 +25,13 @@
 // accumulator, so the tensor-core sum equals the integer sum.  (sm_103a has
 // no integer tcgen05 MMA kind; this is why the integer GEMM runs on the
 // floating-point pipe.)
+//
+// 16-bit stage-1 codes (Section 5 LLM variant): decoded values reach
+// 7 * 2^12 and are expanded to E5M2 instead (exact, see lzs_e4m3.cuh).
+// Each product is still exact, but a group sum can need more than fp32's 24
+// significant bits (products from 2^0 to 49 * 2^24), so P_g is the fp32
+// tensor-core sum of exact products rather than the exact integer; the
+// accumulator-shift GEMM below is the exact path for those operands.
 #include <cuda.h>
 #include <cuda_fp16.h>
 #include <type_traits>
@@ -88,7 +95,7 @@ struct PrepArgs {
 constexpr int kPrepThreads = 256;
 constexpr int kSideGroupsPerThread = 8;
 
-template <int GS>
+template <int GS, bool WIDE>
 __device__ __forceinline__ void run_expand(const ExpandJob &j, int64_t u)
 {
     if (u >= j.units_pad) return;
@@ -117,8 +124,13 @@ __device__ __forceinline__ void run_expand(const ExpandJob &j, int64_t u)
         f0 = f1 = load_flag(j.flags, (u * 16) / GS, j.packed_flags != 0);
     }
     uint4 o;
-    e4m3_from_codes8(c.x, f0, o.x, o.y);
-    e4m3_from_codes8(c.y, f1, o.z, o.w);
+    if (WIDE) {
+        e5m2_from_codes8(c.x, f0, o.x, o.y);
+        e5m2_from_codes8(c.y, f1, o.z, o.w);
+    } else {
+        e4m3_from_codes8(c.x, f0, o.x, o.y);
+        e4m3_from_codes8(c.y, f1, o.z, o.w);
+    }
     j.out[dst] = o;
 }
 
@@ -143,14 +155,14 @@ __device__ __forceinline__ void run_side(const SideJob &j, int64_t t, int G, int
     }
 }
 
-template <int GS>
+template <int GS, bool WIDE>
 __global__ void __launch_bounds__(kPrepThreads) prep_kernel(const __grid_constant__ PrepArgs args)
 {
     const int64_t bid = blockIdx.x;
     if (bid < args.block_end[0]) {
-        run_expand<GS>(args.ex_a, bid * kPrepThreads + threadIdx.x);
+        run_expand<GS, WIDE>(args.ex_a, bid * kPrepThreads + threadIdx.x);
     } else if (bid < args.block_end[1]) {
-        run_expand<GS>(args.ex_w, (bid - args.block_end[0]) * kPrepThreads + threadIdx.x);
+        run_expand<GS, WIDE>(args.ex_w, (bid - args.block_end[0]) * kPrepThreads + threadIdx.x);
     } else if (bid < args.block_end[2]) {
         run_side(args.sd_a, (bid - args.block_end[1]) * kPrepThreads + threadIdx.x, args.G, args.nside);
     } else {
@@ -210,6 +222,7 @@ struct GemmArgs {
     int partials_group;
     int *dev_err;
     int per_row;          // scales per row (group_q = K) rather than per 64-group
+    int wide;             // E5M2 operands (16-bit stage-1 codes) instead of E4M3
 };
 
 // Shared memory: the operand stages, then a ring of side-value slots (one
@@ -488,7 +501,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // frees the operand stage, one hands P_g to the epilogue.
         // ------------------------------------------------------------------
         if (lane == 0) {
-            constexpr uint32_t idesc = idesc_e4m3_f32(BM, BN);
+            const uint32_t idesc = args.wide ? idesc_e5m2_f32(BM, BN) : idesc_e4m3_f32(BM, BN);
             int it = 0;
             bool ok = true;
             constexpr int CH = PERROW ? kPerRowChunk : 1;  // stages per TMEM accumulator
@@ -1121,6 +1134,7 @@ GemmArgs make_args(const LinearWorkspace &ws, int64_t M, int64_t N, int64_t K, c
 {
     GemmArgs a;
     a.per_row = 0;
+    a.wide = 0;
     a.a_side = ws.a_side;
     a.w_side = ws.w_side;
     a.m_pad = ws.m_pad;
@@ -1198,11 +1212,20 @@ cudaError_t launch_prepare(const quartz_encoded_t *a, const quartz_encoded_t *w,
     }
     if (acc == 0) return cudaSuccess;
     const unsigned blocks = static_cast<unsigned>(acc);
+    if (w->p.code_bits == 16) {  // 16-bit stage-1 codes: E5M2 operands
+        switch (w->p.group_s) {
+            case 8: prep_kernel<8, true><<<blocks, kPrepThreads, 0, s>>>(p); break;
+            case 16: prep_kernel<16, true><<<blocks, kPrepThreads, 0, s>>>(p); break;
+            case 32: prep_kernel<32, true><<<blocks, kPrepThreads, 0, s>>>(p); break;
+            default: prep_kernel<64, true><<<blocks, kPrepThreads, 0, s>>>(p); break;
+        }
+        return cudaGetLastError();
+    }
     switch (w->p.group_s) {
-        case 8: prep_kernel<8><<<blocks, kPrepThreads, 0, s>>>(p); break;
-        case 16: prep_kernel<16><<<blocks, kPrepThreads, 0, s>>>(p); break;
-        case 32: prep_kernel<32><<<blocks, kPrepThreads, 0, s>>>(p); break;
-        default: prep_kernel<64><<<blocks, kPrepThreads, 0, s>>>(p); break;
+        case 8: prep_kernel<8, false><<<blocks, kPrepThreads, 0, s>>>(p); break;
+        case 16: prep_kernel<16, false><<<blocks, kPrepThreads, 0, s>>>(p); break;
+        case 32: prep_kernel<32, false><<<blocks, kPrepThreads, 0, s>>>(p); break;
+        default: prep_kernel<64, false><<<blocks, kPrepThreads, 0, s>>>(p); break;
     }
     return cudaGetLastError();
 }
@@ -1210,7 +1233,7 @@ cudaError_t launch_prepare(const quartz_encoded_t *a, const quartz_encoded_t *w,
 cudaError_t launch_gemm_tcgen05(const LinearWorkspace &ws, int64_t M, int64_t N, int64_t K,
                                 int mode, const void *bias, void *y, int y_type,
                                 int32_t *partials, int partials_group, int *dev_err,
-                                cudaStream_t s, bool per_row)
+                                cudaStream_t s, bool per_row, bool wide)
 {
     if (M == 0) return cudaSuccess;
     CUtensorMap ta, tw;
@@ -1218,6 +1241,7 @@ cudaError_t launch_gemm_tcgen05(const LinearWorkspace &ws, int64_t M, int64_t N,
         return cudaErrorInvalidValue;
     GemmArgs args = make_args(ws, M, N, K, bias, y, y_type, partials, partials_group, dev_err);
     args.per_row = per_row ? 1 : 0;
+    args.wide = wide ? 1 : 0;
     if (per_row) return launch_tc_out<QUARTZ_SYMMETRIC>(ta, tw, args, y_type, s);
     return mode == QUARTZ_ASYMMETRIC ? launch_tc_out<QUARTZ_ASYMMETRIC>(ta, tw, args, y_type, s)
                                      : launch_tc_out<QUARTZ_SYMMETRIC>(ta, tw, args, y_type, s);

@@ -1,5 +1,6 @@
 // Device helpers shared by the encoder and the operand preparation: decode
-// of 4-bit LZS codes (Eq. 2) to FP8 E4M3 tensor-core operands.
+// of 4-bit LZS codes (Eq. 2) to FP8 E4M3 (or, for 16-bit stage-1 codes,
+// E5M2) tensor-core operands.
 #pragma once
 #include <cstdint>
 
@@ -42,6 +43,26 @@ __device__ __forceinline__ void e4m3_from_codes8(uint32_t word, int flag, uint32
     const uint32_t t3 = 0xB8C0C4C8u + add;                  // -4, -3, -2, -1
     const uint32_t ev = lut16(word & 0x0F0F0F0Fu, t0, t1, t2, t3);         // codes 0, 2, 4, 6
     const uint32_t od = lut16((word >> 4) & 0x0F0F0F0Fu, t0, t1, t2, t3);  // codes 1, 3, 5, 7
+    lo = prmt_b32(ev, od, 0x5140u);
+    hi = prmt_b32(ev, od, 0x7362u);
+}
+
+// The same for codes with FLAGs up to 12 (16-bit stage-1 codes, Section 5
+// LLM variant), to E5M2 bytes: |v| reaches 7 * 2^12 = 28672, beyond E4M3's
+// range but exact in E5M2, whose 2-bit mantissa holds every |c| <= 7
+// (1, 1.5 or 1.75 times a power of two) and whose exponent reaches 2^15.
+// The byte of a nonzero c is sign | (15 + e + flag) << 2 | m, so FLAG f adds
+// 4 f to every nonzero entry (largest 0x47 + 48 = 0x77: no carry leaves a
+// byte).
+__device__ __forceinline__ void e5m2_from_codes8(uint32_t word, int flag, uint32_t &lo, uint32_t &hi)
+{
+    const uint32_t add = (static_cast<uint32_t>(flag) << 2) * 0x01010101u;
+    const uint32_t t0 = 0x42403C00u + (add & 0xFFFFFF00u);  //  0,  1,  2,  3
+    const uint32_t t1 = 0x47464544u + add;                  //  4,  5,  6,  7
+    const uint32_t t2 = 0xC5C6C700u + (add & 0xFFFFFF00u);  // -8, -7, -6, -5
+    const uint32_t t3 = 0xBCC0C2C4u + add;                  // -4, -3, -2, -1
+    const uint32_t ev = lut16(word & 0x0F0F0F0Fu, t0, t1, t2, t3);
+    const uint32_t od = lut16((word >> 4) & 0x0F0F0F0Fu, t0, t1, t2, t3);
     lo = prmt_b32(ev, od, 0x5140u);
     hi = prmt_b32(ev, od, 0x7362u);
 }

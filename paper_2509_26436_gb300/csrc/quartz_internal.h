@@ -67,7 +67,7 @@ cudaError_t launch_encode_operand(const void *x, int64_t M, int64_t K, const qua
 cudaError_t launch_gemm_tcgen05(const LinearWorkspace &ws, int64_t M, int64_t N, int64_t K,
                                 int mode, const void *bias, void *y, int y_type,
                                 int32_t *partials, int partials_group, int *dev_err,
-                                cudaStream_t s, bool per_row = false);
+                                cudaStream_t s, bool per_row = false, bool wide = false);
 cudaError_t launch_gemm_simt(const LinearWorkspace &ws, int64_t M, int64_t N, int64_t K, int mode,
                              const void *bias, void *y, int y_type, int32_t *partials,
                              int partials_group, cudaStream_t s);

@@ -136,7 +136,7 @@ def test_linear_validation(lib):
 
 def test_code_bits_validation(lib):
     """16-bit stage-1 codes (Section 5 LLM variant): symmetric groups of 64;
-    only the accumulator-shift GEMM takes them, without int32 partials."""
+    no SIMT GEMM and no int32 partials for them."""
     out = (C.c_size_t * 5)()
     for bits, rc in ((0, 0), (8, 0), (16, 0), (12, N.QUARTZ_ERR_INVALID_ARG), (4, N.QUARTZ_ERR_INVALID_ARG)):
         p = N.QuartzParams(64, 8, 0, 8, bits)
@@ -158,9 +158,9 @@ def test_code_bits_validation(lib):
         return L(C.byref(a), C.byref(w), None, 0x2000, 0, 0x3000, 1 << 30, C.byref(o), None)
 
     a, w = enc(16, 128), enc(24, 128)
-    assert lin(a, w, N.ALGO_TCGEN05) == N.QUARTZ_ERR_UNSUPPORTED
     assert lin(a, w, N.ALGO_SIMT) == N.QUARTZ_ERR_UNSUPPORTED
     assert lin(a, w, N.ALGO_SHIFT, part=0x4000) == N.QUARTZ_ERR_UNSUPPORTED
+    assert lin(a, w, N.ALGO_TCGEN05, part=0x4000) == N.QUARTZ_ERR_UNSUPPORTED
     assert lin(a, enc(24, 128, bits=8), N.ALGO_SHIFT) == N.QUARTZ_ERR_INVALID_ARG  # mixed widths
     assert lib.quartz_linear_f16(0x1000, 16, C.byref(w), None, 0x2000, 0, None, 0x3000, 1 << 30,
                                  None) == N.QUARTZ_ERR_UNSUPPORTED

@@ -5,12 +5,16 @@ straight to 4 bits, G_s = 8) against the CPU oracle.
   oracle.encode16, including saturated groups, subnormal scales and packed
   FLAG storage; the dequantiser bit-exact against the oracle's binary64
   value rounded once to fp16.
-* Linear (accumulator-shift GEMM, 64-bit group sums): outputs against the
+* Linear, accumulator-shift GEMM (64-bit group sums): outputs against the
   oracle's binary64 y.  Tolerance from the kernel's arithmetic: P_g is exact
   in 64 bits and is rounded once to binary32; s_a*(s_w*P_g) adds two more
   roundings and the G-term running sum G more, so |y_gpu - y| <=
   (G + 5) 2^-24 sum_g |s_a s_w D_g| before the output conversion (relative
   2^-11 for fp16, 2^-8 for bf16).
+* Linear, tcgen05 GEMM on E5M2 operands: every product is exact, but the
+  64 products of a group are summed in the tensor cores' fp32 accumulator;
+  at most one rounding per product gives a further 64 2^-24
+  sum_g s_a s_w sum_k |v_a v_w| (the magnitude of the group's products).
 """
 import numpy as np
 import pytest
@@ -104,11 +108,28 @@ def _tol_check(y_gpu, y_ref, y_abs, G, dtype_name):
                            f"{(err / np.maximum(tol, 1e-30)).max():.3g}x")
 
 
-def _linear16(Q, xa, xw, gs, bias=None, out_dtype="float16", flag_bits=8):
+def _products_magnitude(ea, ew):
+    """sum_g s_a s_w sum_{k in g} |v_a v_w| for every output (binary64)."""
+    va = np.abs(O.decode_values(ea).astype(np.float64))
+    vw = np.abs(O.decode_values(ew).astype(np.float64))
+    sa, sw = ea.scales.astype(np.float64), ew.scales.astype(np.float64)
+    out = np.zeros((va.shape[0], vw.shape[0]))
+    for g in range(va.shape[1] // 64):
+        blk = va[:, 64 * g:64 * g + 64] @ vw[:, 64 * g:64 * g + 64].T
+        out += sa[:, g:g + 1] * sw[:, g][None, :] * blk
+    return out
+
+
+def _tc_tol_check(y_gpu, ea, ew, bias, G, dtype_name):
+    ref, rabs = O.linear(ea, ew, bias, with_abs=True)
+    _tol_check(y_gpu, ref, rabs + 64 * _products_magnitude(ea, ew), G, dtype_name)
+
+
+def _linear16(Q, xa, xw, gs, bias=None, out_dtype="float16", flag_bits=8, algo=None):
     a = _enc(Q, xa, gs, flag_bits)
     w = Q.encode_weights(torch.from_numpy(xw).cuda(), group_s=gs, code_bits=16, flag_bits=flag_bits)
     b = None if bias is None else torch.from_numpy(bias).cuda()
-    y = Q.linear(a, w, b, out_dtype=getattr(torch, out_dtype))
+    y = Q.linear(a, w, b, out_dtype=getattr(torch, out_dtype), algo=Q.ALGO_SHIFT if algo is None else algo)
     assert Q.device_status() == 0
     return y.float().cpu().numpy()
 
@@ -154,17 +175,17 @@ def test_linear16_group_sums_beyond_int32(Q):
 
 
 def test_linear16_other_algorithms_rejected(Q):
-    """Only the 64-bit accumulator-shift GEMM takes 16-bit codes; mixing
-    8-bit and 16-bit operands is an argument error."""
+    """No SIMT GEMM and no int32 partials for 16-bit codes; mixing 8-bit and
+    16-bit operands is an argument error."""
     x = torch.from_numpy(inputs.mixture_activations(16, 128, seed=5600)).cuda()
     a = Q.quantize(x, group_s=8, code_bits=16)
     w = Q.encode_weights(x[:8].contiguous(), group_s=8, code_bits=16)
     w8 = Q.encode_weights(x[:8].contiguous(), group_s=8)
-    for algo in (Q.ALGO_TCGEN05, Q.ALGO_SIMT):
-        with pytest.raises(Q.QuartzError, match="UNSUPPORTED"):
-            Q.linear(a, w, algo=algo)
     with pytest.raises(Q.QuartzError, match="UNSUPPORTED"):
-        Q.linear(a, w, algo=Q.ALGO_SHIFT, partials_group=0)
+        Q.linear(a, w, algo=Q.ALGO_SIMT)
+    for algo in (Q.ALGO_SHIFT, Q.ALGO_TCGEN05):
+        with pytest.raises(Q.QuartzError, match="UNSUPPORTED"):
+            Q.linear(a, w, algo=algo, partials_group=0)
     with pytest.raises(Q.QuartzError, match="INVALID_ARG"):
         Q.linear(a, w8, algo=Q.ALGO_SHIFT)
     torch.cuda.synchronize()
@@ -179,7 +200,7 @@ def test_linear16_llama_layers_sampled(Q, layer):
     xa, xw = layer.activations(), layer.weights()
     a = Q.quantize(torch.from_numpy(xa).cuda(), group_s=8, code_bits=16)
     w = Q.encode_weights(torch.from_numpy(xw).cuda(), group_s=8, code_bits=16)
-    y = Q.linear(a, w)
+    y = Q.linear(a, w, algo=Q.ALGO_SHIFT)
     assert Q.device_status() == 0
     rows = np.unique(np.concatenate([np.arange(3), np.arange(layer.M - 3, layer.M),
                                      np.linspace(3, layer.M - 4, 6).astype(np.int64)]))
@@ -190,3 +211,44 @@ def test_linear16_llama_layers_sampled(Q, layer):
     assert np.array_equal(w.codes.cpu().numpy(), ew.codes)
     ref, rabs = O.linear(ea, ew, with_abs=True)
     _tol_check(y[rt].float().cpu().numpy(), ref, rabs, layer.K // 64, "float16")
+
+
+# --- tcgen05 GEMM on E5M2 operands ------------------------------------------
+
+@pytest.mark.parametrize("gs", [8, 16, 64])
+@pytest.mark.parametrize("M,N,K", [(1, 8, 64), (200, 264, 640), (129, 520, 1216), (300, 1024, 4096)])
+def test_linear16_tcgen05_ragged_shapes(Q, gs, M, N, K):
+    xa = inputs.laplace_activations(M, K, seed=5700 + M, outlier_frac=0.002, outlier_scale=100.0)
+    xw = inputs.gaussian_weights(N, K, seed=5701 + N)
+    bias = np.random.default_rng(M).normal(0, 0.1, N).astype(np.float16)
+    y = _linear16(Q, xa, xw, gs, bias, algo=Q.ALGO_TCGEN05)
+    _tc_tol_check(y, O.encode16(xa, 64, gs), O.encode16(xw, 64, gs), bias, K // 64, "float16")
+
+
+def test_linear16_tcgen05_extremes_and_packed_flags(Q):
+    """Saturated rows (group sums 64 x 28672^2) and mixed FLAG 0..12 rows
+    through the E5M2 operands; packed FLAGs give the identical output."""
+    xa = inputs.mixture_activations(130, 512, seed=5800)
+    xw = inputs.gaussian_weights(264, 512, seed=5801)
+    xa[0, :] = 8.0
+    xa[1, ::2], xa[1, 1::2] = -3.0, 3.0
+    xw[0, :] = -2.0
+    xa[2, :] = (np.arange(512) % 8 - 3.5).astype(np.float16) * np.float16(2.0 ** -12)
+    y = _linear16(Q, xa, xw, 8, out_dtype="float32", algo=Q.ALGO_TCGEN05)
+    _tc_tol_check(y, O.encode16(xa, 64, 8), O.encode16(xw, 64, 8), None, 8, "float32")
+    y4 = _linear16(Q, xa, xw, 8, out_dtype="float32", flag_bits=4, algo=Q.ALGO_TCGEN05)
+    assert np.array_equal(y4, y)
+
+
+@pytest.mark.parametrize("layer", inputs.CONFIG_LLM, ids=[l.name for l in inputs.CONFIG_LLM])
+def test_linear16_tcgen05_llama_layers_sampled(Q, layer):
+    xa, xw = layer.activations(), layer.weights()
+    a = Q.quantize(torch.from_numpy(xa).cuda(), group_s=8, code_bits=16)
+    w = Q.encode_weights(torch.from_numpy(xw).cuda(), group_s=8, code_bits=16)
+    y = Q.linear(a, w, algo=Q.ALGO_TCGEN05)
+    assert Q.device_status() == 0
+    rows = np.unique(np.concatenate([np.arange(3), np.arange(layer.M - 3, layer.M),
+                                     np.linspace(3, layer.M - 4, 6).astype(np.int64)]))
+    rt = torch.from_numpy(rows).cuda()
+    _tc_tol_check(y[rt].float().cpu().numpy(), O.encode16(xa[rows], 64, 8), O.encode16(xw, 64, 8), None,
+                  layer.K // 64, "float16")
