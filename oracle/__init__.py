@@ -14,6 +14,8 @@ Every function follows a passage of arXiv 2509.26436:
   lzs_encode16    Eq. 2 on 16-bit codes (FLAG 0..12)
   group_partials  Section 4.4 (integer MMA per 64-wide group)
   linear          Section 4.4 + Appendix C (16-bit group scales)
+  attention_decode  Appendix D, Table 6: attention of one query per head over
+                  an encoded key / value cache (reading in quartz_oracle.c)
 """
 from __future__ import annotations
 
@@ -72,6 +74,8 @@ def _load():
             lib.oracle_lzs_encode16.argtypes = [P, i64, i32, P, P]
             lib.oracle_encode16.argtypes = [P, i64, i64, i32, i32, P, P, P]
             lib.oracle_encode_static.argtypes = [P, i64, i64, C.c_uint16, i32, i32, P, P, P]
+            lib.oracle_attention_decode.argtypes = [P, P, P, P, P, P, P, P, P, i64, i64, i64, i64, i32,
+                                                    i32, C.c_double, P, P]
             lib.oracle_decode_codes.argtypes = [P, P, i64, i64, i32, P]
             lib.oracle_dequantize.argtypes = [P, P, P, P, i64, i64, i32, i32, P]
             lib.oracle_group_partials.argtypes = [P, P, i64, i64, i64, i32, P, i64, P]
@@ -310,3 +314,24 @@ def linear(a: Encoded, w: Encoded, bias16=None, rows=None, with_abs: bool = Fals
                                  0 if sel is None else sel.size, _ptr(scratch), _ptr(y),
                                  _ptr(yabs)))
     return (y, yabs) if with_abs else y
+
+
+# --- attention (Appendix D, Table 6) ---------------------------------------
+
+def attention_decode(q: Encoded, k: Encoded, v: Encoded, L_max: int, L: int, scale: float,
+                     with_abs: bool = False):
+    """o [BH, d] binary64: one query per (batch x head) row of `q` against the
+    first L tokens of that head's rows (bh * L_max + t) of the caches."""
+    if not (q.K == k.K == v.K and q.group_q == k.group_q == v.group_q and
+            q.group_s == k.group_s == v.group_s and q.mode == k.mode == v.mode == SYMMETRIC):
+        raise ValueError("q, k, v must share d, group sizes and the symmetric mode")
+    BH, d = q.rows, q.K
+    if k.rows != BH * L_max or v.rows != BH * L_max:
+        raise ValueError("caches must hold BH * L_max rows")
+    o = np.empty((BH, d), np.float64)
+    oabs = np.empty((BH, d), np.float64) if with_abs else None
+    _check(_load().oracle_attention_decode(
+        _ptr(q.codes), _ptr(q.flags), _ptr(_as_u16(q.scales)), _ptr(k.codes), _ptr(k.flags),
+        _ptr(_as_u16(k.scales)), _ptr(v.codes), _ptr(v.flags), _ptr(_as_u16(v.scales)), BH, L_max, L, d,
+        q.group_q, q.group_s, float(scale), _ptr(o), _ptr(oabs)))
+    return (o, oabs) if with_abs else o

@@ -523,3 +523,73 @@ int oracle_linear(const uint8_t *a_codes, const uint8_t *a_flags, const uint16_t
     }
     return ORACLE_OK;
 }
+
+/* ---------------------------------------------------------------------------
+ * QuaRTZ attention, one decode step (Appendix D, Table 6: QuaRTZ kernels for
+ * attention with heads x 128 dimensions and LZS groups of 8 / 16 / 32).  The
+ * paper gives no formula; the reading used here (R18): the query and the
+ * key / value caches are encoded with Eq. 1 + Eq. 2 per token, groups of
+ * `gq` along the head dimension d, and for each of the BH (batch x head)
+ * rows
+ *     score_t = scale * sum_g s_q[g] s_k[t,g] sum_{k in g} v_q[k] v_k[t,k]
+ *     p_t     = exp(score_t - max_t score) / sum_t exp(score_t - max_t score)
+ *     o[k]    = sum_t p_t * s_v[t,g(k)] * v_v[t,k]
+ * over the first L tokens of the head, the integer group sums in int64 and
+ * everything else in binary64.  The caches hold the tokens of head bh in
+ * rows bh * L_max .. bh * L_max + L - 1.  Output o [BH, d]; when `oabs` is
+ * not NULL it receives sum_t p_t |s_v v_v[t,k]|, the magnitude a rounding
+ * error bound of o scales with.  Symmetric encodings (no zero points).
+ * ------------------------------------------------------------------------- */
+int oracle_attention_decode(const uint8_t *q_codes, const uint8_t *q_flags, const uint16_t *q_scales,
+                            const uint8_t *k_codes, const uint8_t *k_flags, const uint16_t *k_scales,
+                            const uint8_t *v_codes, const uint8_t *v_flags, const uint16_t *v_scales,
+                            int64_t BH, int64_t L_max, int64_t L, int64_t d, int gq, int gs,
+                            double scale, double *o, double *oabs)
+{
+    static double score[65536];
+    int16_t vq[4096], vk[4096];
+    if (d <= 0 || d > 4096 || gq <= 0 || d % gq != 0 || gs <= 0 || gq % gs != 0 || L <= 0 ||
+        L > L_max || L > 65536 || BH < 0)
+        return ORACLE_ERR_ARG;
+    int64_t G = d / gq;
+    for (int64_t bh = 0; bh < BH; ++bh) {
+        int rc = oracle_decode_codes(q_codes + bh * (d / 2), q_flags + bh * (d / gs), 1, d, gs, vq);
+        if (rc) return rc;
+        double smax = -INFINITY;
+        for (int64_t t = 0; t < L; ++t) {
+            int64_t row = bh * L_max + t;
+            rc = oracle_decode_codes(k_codes + row * (d / 2), k_flags + row * (d / gs), 1, d, gs, vk);
+            if (rc) return rc;
+            double acc = 0.0;
+            for (int64_t g = 0; g < G; ++g) {
+                int64_t P = 0;
+                for (int64_t k = g * gq; k < (g + 1) * gq; ++k) P += (int64_t)vq[k] * (int64_t)vk[k];
+                acc += (double)oracle_half_to_float(q_scales[bh * G + g]) *
+                       (double)oracle_half_to_float(k_scales[row * G + g]) * (double)P;
+            }
+            score[t] = scale * acc;
+            if (score[t] > smax) smax = score[t];
+        }
+        double denom = 0.0;
+        for (int64_t t = 0; t < L; ++t) {
+            score[t] = exp(score[t] - smax);
+            denom += score[t];
+        }
+        for (int64_t k = 0; k < d; ++k) {
+            o[bh * d + k] = 0.0;
+            if (oabs) oabs[bh * d + k] = 0.0;
+        }
+        for (int64_t t = 0; t < L; ++t) {
+            int64_t row = bh * L_max + t;
+            double p = score[t] / denom;
+            rc = oracle_decode_codes(v_codes + row * (d / 2), v_flags + row * (d / gs), 1, d, gs, vk);
+            if (rc) return rc;
+            for (int64_t k = 0; k < d; ++k) {
+                double vhat = (double)oracle_half_to_float(v_scales[row * G + k / gq]) * (double)vk[k];
+                o[bh * d + k] += p * vhat;
+                if (oabs) oabs[bh * d + k] += p * fabs(vhat);
+            }
+        }
+    }
+    return ORACLE_OK;
+}

@@ -601,3 +601,75 @@ def test_encode16_truncation_bound_and_linear_exact():
     assert np.allclose(y, ref, rtol=1e-12, atol=1e-12 * np.abs(ref).max())
     P = O.group_partials(O.decode_values(a), O.decode_values(w), 64)
     assert P[0, 0, 0] == -64 * 28672 * 28672 and abs(P[0, 0, 0]) > 2 ** 31
+
+
+# --- attention decode step (Appendix D, Table 6) ----------------------------
+
+def _attn_inputs(BH, L_max, d, gs, seed):
+    q = O.encode(inputs.laplace_activations(BH, d, seed=seed, outlier_frac=0.01, outlier_scale=20.0), 64, gs)
+    k = O.encode(inputs.laplace_activations(BH * L_max, d, seed=seed + 1, outlier_frac=0.01,
+                                            outlier_scale=20.0), 64, gs)
+    v = O.encode(inputs.mixture_activations(BH * L_max, d, seed=seed + 2), 64, gs)
+    return q, k, v
+
+
+@pytest.mark.parametrize("gs", [8, 16, 32])
+def test_attention_equals_dense_softmax_of_dequantised(gs):
+    """A different route: dequantise q, K, V (binary64), then dense
+    softmax(q K^T scale) V with SciPy's softmax, per head over the first L
+    cache rows of that head.  Catches a wrong cache row, a dropped scale, a
+    transposed operand or a softmax over the wrong axis."""
+    from scipy.special import softmax
+    BH, L_max, L, d = 5, 40, 33, 128
+    q, k, v = _attn_inputs(BH, L_max, d, gs, 300 + gs)
+    scale = d ** -0.5
+    o, oabs = O.attention_decode(q, k, v, L_max, L, scale, with_abs=True)
+    qh, kh, vh = O.dequantize(q), O.dequantize(k), O.dequantize(v)
+    for bh in range(BH):
+        kk = kh[bh * L_max:bh * L_max + L]
+        vv = vh[bh * L_max:bh * L_max + L]
+        p = softmax(scale * (kk @ qh[bh]))
+        ref = p @ vv
+        assert np.allclose(o[bh], ref, rtol=1e-12, atol=1e-14)
+        assert np.allclose(oabs[bh], p @ np.abs(vv), rtol=1e-12, atol=1e-14)
+
+
+def test_attention_special_cases():
+    """L = 1 returns that token's dequantised value exactly; a zero query
+    gives equal weights (the mean of the V rows); every output lies in the
+    hull of the V rows; rows beyond L never matter; a key aligned with the
+    query and 60 nats ahead takes all the weight."""
+    BH, L_max, d = 3, 20, 128
+    q, k, v = _attn_inputs(BH, L_max, d, 16, 400)
+    vh = O.dequantize(v)
+    o1 = O.attention_decode(q, k, v, L_max, 1, 0.1)
+    assert np.array_equal(o1, vh[0::L_max][:BH])
+    qz = O.encode(np.zeros((BH, d), np.float16), 64, 16)
+    L = 13
+    oz = O.attention_decode(qz, k, v, L_max, L, 0.1)
+    for bh in range(BH):
+        rows = vh[bh * L_max:bh * L_max + L]
+        assert np.allclose(oz[bh], rows.mean(axis=0), rtol=1e-12, atol=1e-15)
+    o = O.attention_decode(q, k, v, L_max, L, 0.3)
+    for bh in range(BH):
+        rows = vh[bh * L_max:bh * L_max + L]
+        assert (o[bh] >= rows.min(axis=0) - 1e-12).all() and (o[bh] <= rows.max(axis=0) + 1e-12).all()
+    # rows beyond L ignored
+    k2, v2 = _attn_inputs(BH, L_max, d, 16, 500)[1:]
+    for dst, src in ((k, k2), (v, v2)):
+        for bh in range(BH):
+            sl = slice(bh * L_max + L, (bh + 1) * L_max)
+            dst.codes[sl], dst.flags[sl], dst.scales[sl] = src.codes[sl], src.flags[sl], src.scales[sl]
+    assert np.array_equal(O.attention_decode(q, k, v, L_max, L, 0.3), o)
+    # a dominant key: q = k_t* = ones vs all other keys 0; after Eq. 1 and
+    # LZS both decode to 112 s with s = fp16(1/127), so the gap is
+    # 128 * scale * (112 s)^2 = 46.7 nats and the rest weighs < L e^-46
+    xq = np.ones((1, d), np.float16)
+    xk = np.zeros((L_max, d), np.float16)
+    xk[7] = 1.0
+    qd, kd = O.encode(xq, 64, 16), O.encode(xk, 64, 16)
+    vd = O.encode(inputs.mixture_activations(L_max, d, seed=600), 64, 16)
+    od = O.attention_decode(qd, kd, vd, L_max, L_max, 60.0 / 128)
+    vmax = np.abs(O.dequantize(vd)).max()
+    assert np.allclose(od[0], O.dequantize(vd)[7], rtol=0, atol=L_max * np.exp(-46) * vmax)
+    assert not np.array_equal(od[0], O.dequantize(vd)[7])
