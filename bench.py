@@ -51,6 +51,9 @@ def parse():
     p.add_argument("--compare-algos", action="store_true",
                    help="also time the three GEMM algorithms (tcgen05, simt, shift) on each layer")
     p.add_argument("--layers", default="", help="comma-separated subset of layer names (profiling)")
+    p.add_argument("--attention", action="store_true",
+                   help="also time the attention decode step (Appendix D, Table 6: heads x 128, "
+                        "G_s 8/16/32) over a 4096-token encoded cache, batch 16")
     p.add_argument("--llm", action="store_true",
                    help="also time the LLM variant (Section 5: 16-bit codes straight to 4 bits, "
                         "G_s = 8) on LLaMA-2-7B block linears")
@@ -428,6 +431,7 @@ def run_ours(args):
 
     # ---- LLM variant (optional) ---------------------------------------------
     llm = run_llm_variant(args, Q, inputs, dev, n_sm, sm_mhz, peak_src, fp8_peak) if args.llm else None
+    attn = run_attention(args, Q, inputs, dev, hbm_peak, peak_src) if args.attention else None
 
     # ---- end to end through the public API with host buffers ---------------
     # Each (step, layer) unit copies its activations from pinned host memory,
@@ -520,6 +524,7 @@ def run_ours(args):
         "fused": fused,
         "gemm_algos": algos,
         "llm_variant": llm,
+        "attention": attn,
         "e2e": e2e,
         "cpu_baseline": cpu,
     }
@@ -527,6 +532,56 @@ def run_ours(args):
 
 
 LLM_GROUP_S = 8
+
+
+def run_attention(args, Q, inputs, dev, hbm_peak, peak_src):
+    """Attention decode step (one query per batch x head over an encoded
+    4096-token key / value cache) for each Table 6 setting: heads x 128 and
+    G_s in {8, 16, 32}.  Time = CUDA events around quartz_attention_decode
+    (split kernel + combine), median of the timed repetitions; roofline =
+    algorithmic cache bytes over the measured HBM copy peak."""
+    import torch
+    B, L, d = inputs.ATTN_BATCH, inputs.ATTN_CONTEXT, inputs.ATTN_DIM
+    BHmax = B * max(inputs.ATTN_HEADS)
+    xq, xk, xv = inputs.attention_inputs(BHmax, L, seed=inputs.BASE_SEED + 6000)
+    xq_d, xk_d, xv_d = (torch.from_numpy(x).to(dev) for x in (xq, xk, xv))
+    del xk, xv
+    ev = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
+    reps = max(5, min(args.steps, 50))
+    out = []
+    for heads in inputs.ATTN_HEADS:
+        BH = B * heads
+        for gs in (8, 16, 32):
+            q = Q.quantize(xq_d[:BH].contiguous(), group_s=gs)
+            k = Q.quantize(xk_d[:BH * L], group_s=gs)
+            v = Q.quantize(xv_d[:BH * L], group_s=gs)
+            o = torch.empty((BH, d), dtype=torch.float16, device=dev)
+            ws = torch.empty(Q.attention_workspace_size(BH, L), dtype=torch.uint8, device=dev)
+            for _ in range(max(3, args.warmup)):
+                Q.attention_decode(q, k, v, L, L, d ** -0.5, out=o, workspace=ws)
+            torch.cuda.synchronize()
+            times = []
+            for _ in range(reps):
+                e0, e1 = ev(), ev()
+                e0.record()
+                Q.attention_decode(q, k, v, L, L, d ** -0.5, out=o, workspace=ws)
+                e1.record()
+                times.append((e0, e1))
+            torch.cuda.synchronize()
+            assert Q.device_status() == 0
+            ms = statistics.median(a.elapsed_time(b) for a, b in times)
+            cache_bytes = 2 * BH * L * (d // 2 + d // gs + 2 * (d // GROUP_Q))
+            gbs = cache_bytes / (ms / 1e3) / 1e9
+            out.append({"heads": heads, "dim": d, "group_s": gs, "batch": B, "context": L, "us": ms * 1e3,
+                        "cache_bytes": cache_bytes, "gbs": gbs, "frac": gbs / hbm_peak,
+                        "fp16_cache_bytes": 2 * BH * L * d * 2})
+            del q, k, v, o, ws
+    return {"workload": "attention decode step over an encoded key/value cache (Table 6 settings)",
+            "kernels": "attn_decode_kernel + attn_combine_kernel", "peak_gbs": hbm_peak,
+            "peak_source": peak_src, "bound": "hbm",
+            "bytes": "2 x BH x L x (d/2 codes + d/G_s FLAG bytes + 2 fp16 scales x d/64) per step",
+            "inputs": "seeded synthetic N(0,1) q, k, v; 2% of key dims x8; caches > L2 (no flush)",
+            "settings": out}
 
 
 def run_llm_variant(args, Q, inputs, dev, n_sm, sm_mhz, peak_src, fp8_peak):

@@ -244,6 +244,48 @@ int32_t quartz_linear_f16(const void *x_f16, int64_t M, const quartz_encoded_t *
 int32_t quartz_linear_noalloc(const quartz_encoded_t *a, const quartz_encoded_t *w,
                               const void *bias_f16, void *y, int32_t y_type, void *stream);
 
+/* ---------------------------------------------------------------------------
+ * QuaRTZ attention, one decode step (Appendix D, Table 6: attention kernels
+ * for heads x 128 dimensions with LZS groups of 8 / 16 / 32).  The paper
+ * gives no formula; here the query and a key / value cache are QuaRTZ-encoded
+ * per token (Eq. 1 + Eq. 2 along the head dimension, 64-groups, symmetric
+ * 8-bit codes), and for each of BH = batch x heads rows
+ *     score_t = scale * sum_g s_q[g] s_k[t,g] P_g[t],
+ *     P_g[t] = sum_{k in g} v_q[k] v_k[t,k]  (exact integer, as in the linear)
+ *     o = sum_t softmax(score)_t s_v[t,g] v_v[t,.]
+ * over the first L tokens of the head, softmax and value sum in binary32.
+ * Cache layout: an encoded tensor of BH * L_max rows and K = 128 columns;
+ * token t of head bh is row bh * L_max + t.
+ * ------------------------------------------------------------------------- */
+
+/* Workspace bytes of quartz_attention_decode (split-L partial results);
+ * 0 for invalid sizes (BH outside [1, 65535], L outside [1, 2^30]). */
+size_t quartz_attention_workspace_size(int64_t BH, int64_t L);
+
+/* Encode new tokens into a cache: x_f16 fp16 [BH, T, K] (16-byte aligned)
+ * goes to rows bh * L_max + t0 + j (j < T) of `cache` (BH * L_max rows,
+ * K % 128 == 0, group_q 64, SYMMETRIC, 8-bit codes, any G_s and FLAG
+ * storage), with the arithmetic of quartz_quantize.  Requires
+ * 0 <= t0, t0 + T <= L_max.  T == 0 or BH == 0 is a no-op. */
+int32_t quartz_kv_append(const void *x_f16, int64_t BH, int64_t T, const quartz_encoded_t *cache, int64_t L_max,
+                         int64_t t0, void *stream);
+
+/* One decode step of attention.
+ *   q              encoded queries [BH, 128] (one per batch x head)
+ *   k_cache        encoded keys   [BH * L_max, 128]
+ *   v_cache        encoded values [BH * L_max, 128]
+ *                  (all three: group_q 64, SYMMETRIC, 8-bit codes, the same
+ *                  G_s; each may store its FLAGs in bytes or packed)
+ *   L              tokens attended per head, 1 <= L <= L_max
+ *   scale          softmax scale (finite; typically 1/sqrt(128))
+ *   o              [BH, 128] of o_type (quartz_out_t), 16-byte aligned
+ *   workspace      >= quartz_attention_workspace_size(BH, L) bytes, 16-byte
+ *                  aligned, scratch owned by the caller
+ * BH <= 65535. */
+int32_t quartz_attention_decode(const quartz_encoded_t *q, const quartz_encoded_t *k_cache,
+                                const quartz_encoded_t *v_cache, int64_t L_max, int64_t L, float scale, void *o,
+                                int32_t o_type, void *workspace, size_t workspace_bytes, void *stream);
+
 /* Synchronise `stream`, then read and clear the library's device error word.
  * Returns QUARTZ_OK, QUARTZ_ERR_TIMEOUT if a kernel gave up on a bounded
  * wait since the last call (its outputs are then invalid), or

@@ -23,6 +23,7 @@ from ._native import (ALGO_SHIFT, ALGO_SIMT, ALGO_TCGEN05, ASYMMETRIC, OUT_BF16,
 
 __all__ = ["Params", "Encoded", "quantize", "encode_weights", "dequantize", "linear",
            "linear_workspace_size", "empty_encoded", "device_status", "selftest_timeout",
+           "kv_append", "attention_decode", "attention_workspace_size",
            "SYMMETRIC", "ASYMMETRIC", "QuartzError"]
 
 
@@ -233,3 +234,39 @@ def device_status(stream=None) -> int:
 
 def selftest_timeout(limit_ns: int, stream=None) -> int:
     return int(N.load().quartz_selftest_timeout(limit_ns, _stream(stream)))
+
+
+# --- attention decode step (Appendix D, Table 6) ----------------------------
+
+def attention_workspace_size(BH: int, L: int) -> int:
+    return int(N.load().quartz_attention_workspace_size(BH, L))
+
+
+def kv_append(x, cache: Encoded, L_max: int, t0: int, stream=None) -> None:
+    """Encode fp16 x [BH, T, d] into cache rows bh * L_max + t0 + j."""
+    torch = _torch()
+    if not (x.is_cuda and x.dtype == torch.float16 and x.dim() == 3 and x.is_contiguous()):
+        raise ValueError("x must be a contiguous [BH, T, d] float16 CUDA tensor")
+    BH, T, _ = x.shape
+    cc = cache.c()
+    N.check(N.load().quartz_kv_append(x.data_ptr(), BH, T, C.byref(cc), L_max, t0, _stream(stream)),
+            "quartz_kv_append")
+
+
+def attention_decode(q: Encoded, k_cache: Encoded, v_cache: Encoded, L_max: int, L: int, scale: float,
+                     out_dtype=None, out=None, workspace=None, stream=None):
+    """o [BH, 128]: one encoded query per (batch x head) row attending over
+    the first L tokens of that head's encoded key / value cache."""
+    torch = _torch()
+    out_dtype = out_dtype or torch.float16
+    dev = q.codes.device
+    o = out if out is not None else torch.empty((q.rows, q.K), dtype=out_dtype, device=dev)
+    o_type = _OUT[str(o.dtype).replace("torch.", "")]
+    if workspace is None:
+        workspace = torch.empty(max(attention_workspace_size(q.rows, L), 16), dtype=torch.uint8, device=dev)
+    qc, kc, vc = q.c(), k_cache.c(), v_cache.c()
+    N.check(N.load().quartz_attention_decode(C.byref(qc), C.byref(kc), C.byref(vc), L_max, L, float(scale),
+                                             o.data_ptr(), o_type, workspace.data_ptr(),
+                                             workspace.numel() * workspace.element_size(), _stream(stream)),
+            "quartz_attention_decode")
+    return o

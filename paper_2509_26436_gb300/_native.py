@@ -69,6 +69,11 @@ SIGNATURES = {
                                      _I32, _P]),
     "quartz_linear_f16": (_I32, [_P, _I64, C.POINTER(QuartzEncoded), _P, _P, _I32,
                                  C.POINTER(QuartzEncoded), _P, _SZ, _P]),
+    "quartz_attention_workspace_size": (_SZ, [_I64, _I64]),
+    "quartz_kv_append": (_I32, [_P, _I64, _I64, C.POINTER(QuartzEncoded), _I64, _I64, _P]),
+    "quartz_attention_decode": (_I32, [C.POINTER(QuartzEncoded), C.POINTER(QuartzEncoded),
+                                       C.POINTER(QuartzEncoded), _I64, _I64, C.c_float, _P, _I32, _P, _SZ,
+                                       _P]),
     "quartz_device_status": (_I32, [_P]),
     "quartz_selftest_timeout": (_I32, [_I64, _P]),
 }

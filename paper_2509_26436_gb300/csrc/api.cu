@@ -96,7 +96,7 @@ const char *quartz_status_string(int32_t status)
     }
 }
 
-int32_t quartz_version(void) { return (1 << 16) | 3; }
+int32_t quartz_version(void) { return (1 << 16) | 4; }
 
 int32_t quartz_encoded_sizes(int64_t rows, int64_t K, const quartz_params_t *p, size_t out[5])
 {
@@ -264,6 +264,67 @@ int32_t quartz_linear_f16(const void *x_f16, int64_t M, const quartz_encoded_t *
     if (e == cudaSuccess)
         e = launch_gemm_tcgen05(ws, M, N, K, w->p.mode, bias_f16, y, y_type, nullptr, 0, dev_err, s);
     return map_cuda(e);
+}
+
+namespace {
+// Encoded tensors of the attention step: 128 columns (the head dimension),
+// 64-groups, symmetric 8-bit codes, the same G_s.
+int32_t check_attention_operand(const quartz_encoded_t *e, int group_s)
+{
+    const int32_t rc = check_encoded(e);
+    if (rc) return rc;
+    if (e->K != 128 || e->p.group_s != group_s) return QUARTZ_ERR_INVALID_ARG;
+    if (e->p.group_q != 64 || e->p.mode != QUARTZ_SYMMETRIC || wide_codes(e->p)) return QUARTZ_ERR_UNSUPPORTED;
+    return QUARTZ_OK;
+}
+}  // namespace
+
+size_t quartz_attention_workspace_size(int64_t BH, int64_t L)
+{
+    if (BH <= 0 || BH > 65535 || L <= 0 || L > (int64_t(1) << 30)) return 0;
+    return attention_workspace_bytes(BH, L);
+}
+
+int32_t quartz_kv_append(const void *x_f16, int64_t BH, int64_t T, const quartz_encoded_t *cache, int64_t L_max,
+                         int64_t t0, void *stream)
+{
+    if (!cache) return QUARTZ_ERR_INVALID_ARG;
+    int32_t rc = check_encoded(cache);
+    if (rc) return rc;
+    if (cache->p.mode != QUARTZ_SYMMETRIC || cache->p.group_q != 64 || wide_codes(cache->p))
+        return QUARTZ_ERR_UNSUPPORTED;
+    if (cache->K % 128 != 0) return QUARTZ_ERR_UNSUPPORTED;
+    if (BH < 0 || T < 0 || L_max <= 0 || t0 < 0 || t0 + T > L_max || cache->rows != BH * L_max)
+        return QUARTZ_ERR_INVALID_ARG;
+    if (BH == 0 || T == 0) return QUARTZ_OK;
+    if (!x_f16) return QUARTZ_ERR_INVALID_ARG;
+    if (!aligned16(x_f16)) return QUARTZ_ERR_ALIGNMENT;
+    return map_cuda(launch_kv_append(x_f16, BH, T, cache, L_max, t0, static_cast<cudaStream_t>(stream)));
+}
+
+int32_t quartz_attention_decode(const quartz_encoded_t *q, const quartz_encoded_t *k_cache,
+                                const quartz_encoded_t *v_cache, int64_t L_max, int64_t L, float scale, void *o,
+                                int32_t o_type, void *workspace, size_t workspace_bytes, void *stream)
+{
+    if (!q || !k_cache || !v_cache) return QUARTZ_ERR_INVALID_ARG;
+    int32_t rc = check_attention_operand(q, q->p.group_s);
+    if (rc) return rc;
+    if ((rc = check_attention_operand(k_cache, q->p.group_s)) != QUARTZ_OK) return rc;
+    if ((rc = check_attention_operand(v_cache, q->p.group_s)) != QUARTZ_OK) return rc;
+    const int64_t BH = q->rows;
+    if (BH > 65535 || L_max <= 0 || L <= 0 || L > L_max || L > (int64_t(1) << 30) ||
+        k_cache->rows != BH * L_max || v_cache->rows != BH * L_max)
+        return QUARTZ_ERR_INVALID_ARG;
+    if (!(scale == scale) || scale > 3.0e38f || scale < -3.0e38f) return QUARTZ_ERR_INVALID_ARG;  // finite
+    if (o_type != QUARTZ_OUT_F16 && o_type != QUARTZ_OUT_BF16 && o_type != QUARTZ_OUT_F32)
+        return QUARTZ_ERR_INVALID_ARG;
+    if (BH == 0) return QUARTZ_OK;
+    if (!o) return QUARTZ_ERR_INVALID_ARG;
+    if (!aligned16(o)) return QUARTZ_ERR_ALIGNMENT;
+    if (!workspace || workspace_bytes < attention_workspace_bytes(BH, L)) return QUARTZ_ERR_WORKSPACE;
+    if (!aligned16(workspace)) return QUARTZ_ERR_ALIGNMENT;
+    return map_cuda(launch_attention_decode(q, k_cache, v_cache, L_max, L, scale, o, o_type, workspace,
+                                            static_cast<cudaStream_t>(stream)));
 }
 
 int32_t quartz_device_status(void *stream)

@@ -1,0 +1,363 @@
+// QuaRTZ attention, one decode step (Appendix D, Table 6: attention with
+// heads x 128 dimensions on LZS-coded operands, groups of 8 / 16 / 32), for
+// sm_103a.
+//
+// One query per (batch x head) row attends over the first L tokens of that
+// head's key / value cache.  Query, keys and values are QuaRTZ-encoded per
+// token (Eq. 1 + Eq. 2, 64-wide groups along the head dimension):
+//     score_t = scale * sum_g s_q[g] s_k[t,g] P_g[t],
+//     P_g[t]  = sum_{k in g} v_q[k] v_k[t,k]            (exact integers)
+//     o       = sum_t softmax(score)_t * s_v[t,g] v_v[t,.]
+// The step is HBM-bound: per token and head it reads 2 x (64 code bytes +
+// 128/G_s FLAG bytes + 4 scale bytes) and does about 2 operations per cached
+// element, so the kernel streams the caches once, split over enough CTAs to
+// keep every SM's memory pipe busy (split-L with a combine pass):
+//
+//   attn_decode_kernel<G_s>: CTA (split, bh), 128 threads, tokens in tiles
+//     of 128.  Keys: one token per thread; the integer group sums are dp4a
+//     products of the query's decoded values (int8, |v| <= 112, computed
+//     once per CTA) with the key codes placed in the high nibble of each
+//     byte (16 c), shifted per subgroup by the key's FLAG — the paper's
+//     accumulator-shift schedule (Section 4.4) on the key side, exact.
+//     Softmax: running maximum and sum per CTA in the log2 domain.  Values:
+//     16 threads per token row (one 32-bit word of 8 codes each) x 8 token
+//     slots; each code becomes a float exactly through the 2^23 magic
+//     number, and o += p_t s_v 2^FLAG c in fp32.  The value words of a tile
+//     are loaded before the key arithmetic so that both DRAM round trips
+//     overlap.  Output per CTA: unnormalised o, running max, running sum.
+//   attn_combine_kernel: one CTA per bh merges the splits.
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+
+#include "lzs_e4m3.cuh"
+#include "quartz_internal.h"
+
+namespace quartz {
+namespace {
+
+constexpr int kD = 128;              // head dimension
+constexpr int kWords = kD / 8;       // 32-bit code words per token row
+constexpr int kTile = 128;           // tokens per tile = threads per CTA
+constexpr int kAttnThreads = 128;
+constexpr int kSlots = kAttnThreads / kWords;  // token slots of the value phase
+constexpr int kPartStride = kD + 4;  // o[128], m, l (+ pad) per split
+constexpr int kMaxSplits = 64;
+constexpr float kLog2e = 1.4426950408889634f;
+
+struct AttnArgs {
+    const uint32_t *q_codes;
+    const uint8_t *q_flags;
+    const __half *q_scales;
+    const uint32_t *k_codes;
+    const uint8_t *k_flags;
+    const __half *k_scales;
+    const uint32_t *v_codes;
+    const uint8_t *v_flags;
+    const __half *v_scales;
+    int q_packed, k_packed, v_packed;
+    int64_t L_max;
+    int L, n_split, chunk;
+    float scale_log2;  // softmax scale * log2(e)
+    float *part;       // [BH][n_split][kPartStride]
+};
+
+__device__ __forceinline__ uint32_t ldg_nc(const uint32_t *p)
+{
+    uint32_t v;
+    asm volatile("ld.global.nc.L1::no_allocate.u32 %0, [%1];" : "=r"(v) : "l"(p));
+    return v;
+}
+
+__device__ __forceinline__ uint4 ldg_nc4(const uint4 *p)
+{
+    uint4 v;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p));
+    return v;
+}
+
+// The FLAG bytes (or nibbles) of one token row: S = 128 / G_s subgroups,
+// stored at subgroup index row * S + j (one byte each, or two per byte).
+template <int GS>
+__device__ __forceinline__ void load_row_flags(const uint8_t *flags, int64_t row, bool packed, uint32_t (&f)[4])
+{
+    constexpr int S = kD / GS;
+    f[0] = f[1] = f[2] = f[3] = 0u;
+    const int bytes = packed ? S / 2 : S;
+    const uint8_t *p = flags + row * bytes;
+    if (bytes == 16) {
+        const uint4 v = *reinterpret_cast<const uint4 *>(p);
+        f[0] = v.x, f[1] = v.y, f[2] = v.z, f[3] = v.w;
+    } else if (bytes == 8) {
+        const uint2 v = *reinterpret_cast<const uint2 *>(p);
+        f[0] = v.x, f[1] = v.y;
+    } else if (bytes == 4) {
+        f[0] = *reinterpret_cast<const uint32_t *>(p);
+    } else if (bytes == 2) {
+        f[0] = *reinterpret_cast<const uint16_t *>(p);
+    } else {
+        f[0] = *p;
+    }
+}
+
+__device__ __forceinline__ int row_flag(const uint32_t (&f)[4], int j, bool packed)
+{
+    return packed ? static_cast<int>((f[j >> 3] >> (4 * (j & 7))) & 0xFu)
+                  : static_cast<int>((f[j >> 2] >> (8 * (j & 3))) & 0xFFu);
+}
+
+__device__ __forceinline__ float2 load_scales2(const __half *scales, int64_t row)
+{
+    const uint32_t w = *reinterpret_cast<const uint32_t *>(scales + 2 * row);
+    return __half22float2(*reinterpret_cast<const __half2 *>(&w));
+}
+
+// Byte permute selecting byte `b` of {hi:lo} into byte 0 (see prmt_b32).
+__device__ __forceinline__ float code_to_float(uint32_t biased_bytes, uint32_t sel)
+{
+    // biased byte = c + 8 in [0, 15]; 0x4B0000xx is the float 2^23 + xx
+    return __int_as_float(prmt_b32(biased_bytes, 0x4B000000u, sel)) - 8388616.0f;
+}
+
+template <int GS>
+__global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(const __grid_constant__ AttnArgs a)
+{
+    constexpr int S = kD / GS;            // subgroups per row
+    constexpr int kWordsPerSub = GS / 8;  // code words per subgroup
+    __shared__ float s_p[kTile];          // softmax weights of the tile
+    __shared__ float s_fv[kTile][S + 1];  // value factors s_v 2^FLAG per token and subgroup
+    __shared__ float s_red[kSlots][kD];   // final reduction over token slots
+    __shared__ float s_wmax[kAttnThreads / 32];
+    __shared__ float s_wsum[kAttnThreads / 32];
+
+    const int tid = threadIdx.x;
+    const int split = blockIdx.x;
+    const int64_t bh = blockIdx.y;
+    const int t_begin = split * a.chunk;
+    const int t_end = min(t_begin + a.chunk, a.L);
+
+    // ---- the query's decoded values, as int8 (even codes, odd codes) -------
+    uint32_t qe[kWords], qo[kWords];
+    float sq0, sq1;
+    {
+        uint32_t f[4];
+        load_row_flags<GS>(a.q_flags, bh, a.q_packed != 0, f);
+        const float2 s2 = load_scales2(a.q_scales, bh);
+        sq0 = s2.x, sq1 = s2.y;
+#pragma unroll
+        for (int w = 0; w < kWords; ++w) {
+            const uint32_t word = a.q_codes[bh * kWords + w];
+            const int F = row_flag(f, w / kWordsPerSub, a.q_packed != 0);
+            uint32_t e = 0u, o = 0u;
+#pragma unroll
+            for (int b = 0; b < 4; ++b) {
+                const int c0 = static_cast<int>(word << (28 - 8 * b)) >> 28;  // code 2b
+                const int c1 = static_cast<int>(word << (24 - 8 * b)) >> 28;  // code 2b + 1
+                e |= (static_cast<uint32_t>(c0 * (1 << F)) & 0xFFu) << (8 * b);
+                o |= (static_cast<uint32_t>(c1 * (1 << F)) & 0xFFu) << (8 * b);
+            }
+            qe[w] = e;
+            qo[w] = o;
+        }
+    }
+
+    const int vw = tid % kWords;   // value phase: code word of this thread
+    const int slot = tid / kWords; // value phase: token slot
+    const int vsub = vw / kWordsPerSub;
+    float acc[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) acc[k] = 0.f;
+    float m_run = -INFINITY;  // running maximum (log2 domain)
+    float l_thr = 0.f;        // this thread's share of the running sum
+
+    for (int tile = t_begin; tile < t_end; tile += kTile) {
+        // value words of this tile (independent of the scores): issue first
+        uint32_t vwords[kTile / kSlots];
+#pragma unroll
+        for (int i = 0; i < kTile / kSlots; ++i) {
+            const int t = tile + slot + i * kSlots;
+            vwords[i] = t < t_end ? ldg_nc(a.v_codes + (bh * a.L_max + t) * kWords + vw) : 0u;
+        }
+
+        // ---- keys: one token per thread -----------------------------------
+        const int t = tile + tid;
+        const bool valid = t < t_end;
+        float s2 = -INFINITY;
+        if (valid) {
+            const int64_t row = bh * a.L_max + t;
+            uint4 kc[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) kc[i] = ldg_nc4(reinterpret_cast<const uint4 *>(a.k_codes + row * kWords) + i);
+            uint32_t kf[4], vf[4];
+            load_row_flags<GS>(a.k_flags, row, a.k_packed != 0, kf);
+            load_row_flags<GS>(a.v_flags, row, a.v_packed != 0, vf);
+            const float2 sk = load_scales2(a.k_scales, row);
+            const float2 sv = load_scales2(a.v_scales, row);
+            const uint32_t kw[kWords] = {kc[0].x, kc[0].y, kc[0].z, kc[0].w, kc[1].x, kc[1].y, kc[1].z, kc[1].w,
+                                         kc[2].x, kc[2].y, kc[2].z, kc[2].w, kc[3].x, kc[3].y, kc[3].z, kc[3].w};
+            int P[2] = {0, 0};
+#pragma unroll
+            for (int j = 0; j < S; ++j) {
+                int dot = 0;  // 16 x the code dot product of subgroup j
+#pragma unroll
+                for (int w = j * kWordsPerSub; w < (j + 1) * kWordsPerSub; ++w) {
+                    dot = __dp4a(static_cast<int>(qe[w]), static_cast<int>((kw[w] << 4) & 0xF0F0F0F0u), dot);
+                    dot = __dp4a(static_cast<int>(qo[w]), static_cast<int>(kw[w] & 0xF0F0F0F0u), dot);
+                }
+                P[(j * GS) / 64] += (dot >> 4) * (1 << row_flag(kf, j, a.k_packed != 0));
+                s_fv[tid][j] = ldexpf((j * GS) / 64 ? sv.y : sv.x, row_flag(vf, j, a.v_packed != 0));
+            }
+            const float sc = __fmul_rn(__fmul_rn(sq0, sk.x), static_cast<float>(P[0])) +
+                             __fmul_rn(__fmul_rn(sq1, sk.y), static_cast<float>(P[1]));
+            s2 = sc * a.scale_log2;
+        } else {
+#pragma unroll
+            for (int j = 0; j < S; ++j) s_fv[tid][j] = 0.f;
+        }
+
+        // ---- softmax: tile maximum, rescale, weights ----------------------
+        float wm = s2;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) wm = fmaxf(wm, __shfl_xor_sync(0xffffffffu, wm, o));
+        if ((tid & 31) == 0) s_wmax[tid >> 5] = wm;
+        __syncthreads();
+        float tmax = s_wmax[0];
+#pragma unroll
+        for (int w = 1; w < kAttnThreads / 32; ++w) tmax = fmaxf(tmax, s_wmax[w]);
+        const float m_new = fmaxf(m_run, tmax);
+        const float alpha = exp2f(m_run - m_new);  // 0 on the first tile
+        const float p = valid ? exp2f(s2 - m_new) : 0.f;
+        l_thr = l_thr * alpha + p;
+        s_p[tid] = p;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) acc[k] *= alpha;
+        m_run = m_new;
+        __syncthreads();
+
+        // ---- values: o += p_t s_v 2^FLAG c_t -------------------------------
+#pragma unroll
+        for (int i = 0; i < kTile / kSlots; ++i) {
+            const int ti = slot + i * kSlots;
+            const float pf = s_p[ti] * s_fv[ti][vsub];  // 0 for tokens past the end
+            const uint32_t word = vwords[i];
+            const uint32_t ev = (word & 0x0F0F0F0Fu) ^ 0x08080808u;         // codes 0, 2, 4, 6 as c + 8
+            const uint32_t od = ((word >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u;  // codes 1, 3, 5, 7
+#pragma unroll
+            for (int b = 0; b < 4; ++b) {
+                acc[2 * b] = fmaf(pf, code_to_float(ev, 0x7440u | b), acc[2 * b]);
+                acc[2 * b + 1] = fmaf(pf, code_to_float(od, 0x7440u | b), acc[2 * b + 1]);
+            }
+        }
+        __syncthreads();  // s_p / s_fv are rewritten by the next tile
+    }
+
+    // ---- reduce over token slots, write this split's partial result -------
+#pragma unroll
+    for (int k = 0; k < 8; ++k) s_red[slot][vw * 8 + k] = acc[k];
+    float ws = l_thr;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) ws += __shfl_xor_sync(0xffffffffu, ws, o);
+    if ((tid & 31) == 0) s_wsum[tid >> 5] = ws;
+    __syncthreads();
+    float od = 0.f;
+#pragma unroll
+    for (int sl = 0; sl < kSlots; ++sl) od += s_red[sl][tid];
+    float *part = a.part + (bh * a.n_split + split) * kPartStride;
+    part[tid] = od;
+    if (tid == 0) {
+        float l = 0.f;
+#pragma unroll
+        for (int w = 0; w < kAttnThreads / 32; ++w) l += s_wsum[w];
+        part[kD] = m_run;
+        part[kD + 1] = l;
+    }
+}
+
+template <int OUT>
+__global__ void __launch_bounds__(kD) attn_combine_kernel(const float *__restrict__ part, int n_split, void *out)
+{
+    const int64_t bh = blockIdx.x;
+    const int d = threadIdx.x;
+    const float *p = part + bh * n_split * kPartStride;
+    float M = -INFINITY;
+    for (int s = 0; s < n_split; ++s) M = fmaxf(M, p[s * kPartStride + kD]);
+    float num = 0.f, den = 0.f;
+    for (int s = 0; s < n_split; ++s) {
+        const float w = exp2f(p[s * kPartStride + kD] - M);  // 0 for an empty split
+        num = fmaf(w, p[s * kPartStride + d], num);
+        den = fmaf(w, p[s * kPartStride + kD + 1], den);
+    }
+    const float v = num / den;
+    const int64_t off = bh * kD + d;
+    if (OUT == QUARTZ_OUT_F16) static_cast<__half *>(out)[off] = __float2half_rn(v);
+    else if (OUT == QUARTZ_OUT_BF16) static_cast<__nv_bfloat16 *>(out)[off] = __float2bfloat16_rn(v);
+    else static_cast<float *>(out)[off] = v;
+}
+
+int attn_splits(int64_t BH, int64_t L, int *chunk)
+{
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (sms <= 0) sms = 1;
+    const int64_t tiles = (L + kTile - 1) / kTile;
+    const int64_t max_split = tiles < kMaxSplits ? tiles : kMaxSplits;
+    int64_t n = (8 * static_cast<int64_t>(sms) + BH - 1) / BH;  // about 8 CTAs per SM
+    if (n < 1) n = 1;
+    if (n > max_split) n = max_split;
+    const int64_t per = (tiles + n - 1) / n;  // tiles per split
+    *chunk = static_cast<int>(per * kTile);
+    return static_cast<int>((tiles + per - 1) / per);
+}
+
+}  // namespace
+
+size_t attention_workspace_bytes(int64_t BH, int64_t L)
+{
+    const int64_t tiles = (L + kTile - 1) / kTile;
+    const int64_t splits = tiles < kMaxSplits ? tiles : kMaxSplits;
+    return static_cast<size_t>(BH * splits * kPartStride) * sizeof(float);
+}
+
+cudaError_t launch_attention_decode(const quartz_encoded_t *q, const quartz_encoded_t *k, const quartz_encoded_t *v,
+                                    int64_t L_max, int64_t L, float scale, void *o, int o_type, void *workspace,
+                                    cudaStream_t s)
+{
+    const int64_t BH = q->rows;
+    if (BH == 0) return cudaSuccess;
+    AttnArgs a;
+    a.q_codes = reinterpret_cast<const uint32_t *>(q->codes);
+    a.q_flags = q->flags;
+    a.q_scales = reinterpret_cast<const __half *>(q->scales);
+    a.k_codes = reinterpret_cast<const uint32_t *>(k->codes);
+    a.k_flags = k->flags;
+    a.k_scales = reinterpret_cast<const __half *>(k->scales);
+    a.v_codes = reinterpret_cast<const uint32_t *>(v->codes);
+    a.v_flags = v->flags;
+    a.v_scales = reinterpret_cast<const __half *>(v->scales);
+    a.q_packed = q->p.flag_bits == 4;
+    a.k_packed = k->p.flag_bits == 4;
+    a.v_packed = v->p.flag_bits == 4;
+    a.L_max = L_max;
+    a.L = static_cast<int>(L);
+    a.n_split = attn_splits(BH, L, &a.chunk);
+    a.scale_log2 = scale * kLog2e;
+    a.part = static_cast<float *>(workspace);
+    const dim3 grid(static_cast<unsigned>(a.n_split), static_cast<unsigned>(BH));
+    switch (q->p.group_s) {
+        case 8: attn_decode_kernel<8><<<grid, kAttnThreads, 0, s>>>(a); break;
+        case 16: attn_decode_kernel<16><<<grid, kAttnThreads, 0, s>>>(a); break;
+        case 32: attn_decode_kernel<32><<<grid, kAttnThreads, 0, s>>>(a); break;
+        default: attn_decode_kernel<64><<<grid, kAttnThreads, 0, s>>>(a); break;
+    }
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const unsigned cb = static_cast<unsigned>(BH);
+    if (o_type == QUARTZ_OUT_F16) attn_combine_kernel<QUARTZ_OUT_F16><<<cb, kD, 0, s>>>(a.part, a.n_split, o);
+    else if (o_type == QUARTZ_OUT_BF16) attn_combine_kernel<QUARTZ_OUT_BF16><<<cb, kD, 0, s>>>(a.part, a.n_split, o);
+    else attn_combine_kernel<QUARTZ_OUT_F32><<<cb, kD, 0, s>>>(a.part, a.n_split, o);
+    return cudaGetLastError();
+}
+
+}  // namespace quartz

@@ -509,6 +509,36 @@ __global__ void __launch_bounds__(kThreads) quantize_kernel(const uint4 *__restr
     }
 }
 
+// Cache append (attention decode step): x [BH, T, d] fp16 is encoded into
+// rows bh * L_max + t0 + j of an encoded cache, symmetric 8-bit codes.  The
+// chunk encoder is the one above; only the output chunk index is remapped
+// (d % 128 == 0 keeps every 64-group and every FLAG byte inside one row).
+template <int GS>
+__global__ void __launch_bounds__(kThreads) kv_append_kernel(const uint4 *__restrict__ x, int64_t n_chunks,
+                                                             int64_t chunks_per_row, int64_t T, int64_t L_max,
+                                                             int64_t t0, uint32_t *__restrict__ codes,
+                                                             uint8_t *__restrict__ flags,
+                                                             __half *__restrict__ scales, int packed)
+{
+    const int lane = threadIdx.x & 31;
+    const int64_t base = static_cast<int64_t>(blockIdx.x) * (kThreads * kChunksPerThread) + threadIdx.x;
+    uint4 raw[kChunksPerThread];
+#pragma unroll
+    for (int j = 0; j < kChunksPerThread; ++j) {
+        const int64_t c = base + j * kThreads;
+        raw[j] = (c < n_chunks) ? ldg_stream(x + c) : make_uint4(0, 0, 0, 0);
+    }
+#pragma unroll
+    for (int j = 0; j < kChunksPerThread; ++j) {
+        const int64_t c = base + j * kThreads;
+        const int64_t r = c / chunks_per_row;
+        const int64_t dst_row = (r / T) * L_max + t0 + (r % T);
+        const int64_t dst = dst_row * chunks_per_row + (c - r * chunks_per_row);
+        encode_chunk<GS, QUARTZ_SYMMETRIC, false>(raw[j], dst, c < n_chunks, lane, codes, flags, scales,
+                                                  nullptr, nullptr, packed != 0);
+    }
+}
+
 // x_hat = s * (v - z), v = sgn(c) (|c| << FLAG); one thread per 8 elements.
 __global__ void __launch_bounds__(kThreads) dequantize_kernel(
     const uint32_t *__restrict__ codes, const uint8_t *__restrict__ flags,
@@ -600,6 +630,27 @@ cudaError_t launch_quantize_row(const void *x, const quartz_encoded_t *e, int us
 }
 
 }  // namespace
+
+cudaError_t launch_kv_append(const void *x, int64_t BH, int64_t T, const quartz_encoded_t *cache, int64_t L_max,
+                             int64_t t0, cudaStream_t s)
+{
+    const int64_t cpr = cache->K / 8;
+    const int64_t n_chunks = BH * T * cpr;
+    if (n_chunks == 0) return cudaSuccess;
+    const int64_t per_block = kThreads * kChunksPerThread;
+    const unsigned blocks = static_cast<unsigned>((n_chunks + per_block - 1) / per_block);
+    const uint4 *xv = static_cast<const uint4 *>(x);
+    uint32_t *codes = reinterpret_cast<uint32_t *>(cache->codes);
+    __half *scales = reinterpret_cast<__half *>(cache->scales);
+    const int packed = cache->p.flag_bits == 4;
+    switch (cache->p.group_s) {
+        case 8: kv_append_kernel<8><<<blocks, kThreads, 0, s>>>(xv, n_chunks, cpr, T, L_max, t0, codes, cache->flags, scales, packed); break;
+        case 16: kv_append_kernel<16><<<blocks, kThreads, 0, s>>>(xv, n_chunks, cpr, T, L_max, t0, codes, cache->flags, scales, packed); break;
+        case 32: kv_append_kernel<32><<<blocks, kThreads, 0, s>>>(xv, n_chunks, cpr, T, L_max, t0, codes, cache->flags, scales, packed); break;
+        default: kv_append_kernel<64><<<blocks, kThreads, 0, s>>>(xv, n_chunks, cpr, T, L_max, t0, codes, cache->flags, scales, packed); break;
+    }
+    return cudaGetLastError();
+}
 
 cudaError_t launch_quantize_static(const void *x, const quartz_encoded_t *out, uint16_t s16, cudaStream_t s)
 {

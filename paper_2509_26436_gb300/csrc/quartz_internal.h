@@ -23,6 +23,15 @@ int *device_error_word();
 
 // Encoder / decoder launches (quantize.cu).  Arguments are pre-validated.
 cudaError_t launch_quantize(const void *x, const quartz_encoded_t *out, cudaStream_t s);
+// Attention decode step (attention.cu): encode x [BH, T, d] into cache rows
+// bh * L_max + t0 + j (quantize.cu), and one query per bh row over the first
+// L cached tokens of that head.
+cudaError_t launch_kv_append(const void *x, int64_t BH, int64_t T, const quartz_encoded_t *cache, int64_t L_max,
+                             int64_t t0, cudaStream_t s);
+size_t attention_workspace_bytes(int64_t BH, int64_t L);
+cudaError_t launch_attention_decode(const quartz_encoded_t *q, const quartz_encoded_t *k, const quartz_encoded_t *v,
+                                    int64_t L_max, int64_t L, float scale, void *o, int o_type, void *workspace,
+                                    cudaStream_t s);
 cudaError_t launch_dequantize(const quartz_encoded_t *e, void *y, cudaStream_t s);
 // Symmetric encoding with a static (calibrated) fp16 scale `s16` for every group.
 cudaError_t launch_quantize_static(const void *x, const quartz_encoded_t *out, uint16_t s16, cudaStream_t s);

@@ -19,6 +19,8 @@ available; these recipes stand in for them:
   1% U(-8,8);
 * UNet convolutions: SiLU(N(0,1)) feature maps with sparse x10 channels,
   lowered to a GEMM by im2col with K ordered (kh, kw, c_in), padding 1;
+* attention decode step (Appendix D, Table 6): N(0, 1) queries, keys and
+  values, 2% of the key dimensions x8;
 * LLM layers (Section 5 variant; the paper's Qwen2 / LLaMA checkpoints and
   its perplexity corpus are not available): the Laplace recipe with 0.2% of
   the channels x100, the few very large channels of LLM hidden states.
@@ -162,6 +164,30 @@ CONFIG_LLM = [
     Layer("llama2_gate_up", 2048, 22016, 4096, 5, 2, outlier_frac=0.002, outlier_scale=100.0),
     Layer("llama2_down", 2048, 4096, 11008, 5, 3, outlier_frac=0.002, outlier_scale=100.0),
 ]
+
+# Attention decode step (Appendix D, Table 6: heads x 128 dimensions, LZS
+# groups 8 / 16 / 32): batch 16, a 4096-token key / value cache per head.
+ATTN_HEADS = (32, 40, 64)
+ATTN_DIM = 128
+ATTN_BATCH = 16
+ATTN_CONTEXT = 4096
+
+
+def attention_inputs(BH: int, L: int, seed: int, outlier_frac: float = 0.02, outlier_scale: float = 8.0):
+    """q [BH, 128], k and v [BH * L, 128] fp16 (head bh's tokens in rows
+    bh * L ..): N(0, 1) entries, the keys with a seeded `outlier_frac` of the
+    head dimensions scaled by `outlier_scale` (the outlier channels of LLM
+    keys), the queries and values plain."""
+    rng = np.random.default_rng(seed)
+    d = ATTN_DIM
+    q = rng.normal(0.0, 1.0, size=(BH, d)).astype(np.float32)
+    k = rng.normal(0.0, 1.0, size=(BH * L, d)).astype(np.float32)
+    ch = _outlier_channels(rng, d, outlier_frac)
+    if ch.size:
+        k[:, ch] *= np.float32(outlier_scale)
+    v = rng.normal(0.0, 1.0, size=(BH * L, d)).astype(np.float32)
+    return q.astype(np.float16), k.astype(np.float16), v.astype(np.float16)
+
 
 # Encode sweep sizes: 1M, 16M and 128M fp16 elements as [rows, 4096].
 ENCODE_SWEEP = [(2 ** 20 // 4096, 4096), (4096, 4096), (32768, 4096)]

@@ -166,6 +166,39 @@ def test_code_bits_validation(lib):
                                  None) == N.QUARTZ_ERR_UNSUPPORTED
 
 
+def test_attention_validation(lib):
+    """Host checks of the attention decode step and the cache append."""
+    def enc(rows, K=128, gs=16, mode=0, gq=64, bits=8):
+        return N.QuartzEncoded(0x1000, 0x1000, 0x1000, 0x1000, 0x1000, rows, K, N.QuartzParams(gq, gs, mode, 8, bits))
+
+    assert lib.quartz_attention_workspace_size(4, 1000) > 0
+    assert lib.quartz_attention_workspace_size(0, 1000) == 0
+    assert lib.quartz_attention_workspace_size(4, 0) == 0
+    A = lib.quartz_attention_decode
+
+    def att(q, k, v, L_max=50, L=40, o=0x2000, t=0, ws=0x3000, wsb=1 << 20, scale=0.1):
+        return A(C.byref(q), C.byref(k), C.byref(v), L_max, L, scale, o, t, ws, wsb, None)
+
+    q, k, v = enc(4), enc(200), enc(200)
+    assert att(enc(4, K=256), enc(200, K=256), enc(200, K=256)) == N.QUARTZ_ERR_INVALID_ARG  # d != 128
+    assert att(q, enc(200, gs=32), v) == N.QUARTZ_ERR_INVALID_ARG          # G_s mismatch
+    assert att(q, enc(199), v) == N.QUARTZ_ERR_INVALID_ARG                 # rows != BH * L_max
+    assert att(q, k, v, L=51) == N.QUARTZ_ERR_INVALID_ARG                  # L > L_max
+    assert att(q, k, v, L=0) == N.QUARTZ_ERR_INVALID_ARG
+    assert att(q, k, v, t=3) == N.QUARTZ_ERR_INVALID_ARG
+    assert att(q, k, v, scale=float("nan")) == N.QUARTZ_ERR_INVALID_ARG
+    assert att(q, k, v, o=0x2004) == N.QUARTZ_ERR_ALIGNMENT
+    assert att(q, k, v, wsb=16) == N.QUARTZ_ERR_WORKSPACE
+    assert att(enc(4, mode=1), enc(200, mode=1), enc(200, mode=1)) == N.QUARTZ_ERR_UNSUPPORTED
+    assert att(enc(4, bits=16), enc(200, bits=16), enc(200, bits=16)) == N.QUARTZ_ERR_UNSUPPORTED
+    K = lib.quartz_kv_append
+    assert K(0x1000, 4, 3, C.byref(enc(200)), 50, 48, None) == N.QUARTZ_ERR_INVALID_ARG   # t0 + T > L_max
+    assert K(0x1000, 4, 3, C.byref(enc(199)), 50, 0, None) == N.QUARTZ_ERR_INVALID_ARG    # rows
+    assert K(0x1000, 4, 3, C.byref(enc(200, K=64)), 50, 0, None) == N.QUARTZ_ERR_UNSUPPORTED
+    assert K(0x1008, 4, 3, C.byref(enc(200)), 50, 0, None) == N.QUARTZ_ERR_ALIGNMENT
+    assert K(None, 4, 0, C.byref(enc(200)), 50, 0, None) == N.QUARTZ_OK                   # T == 0
+
+
 def test_linear_f16_validation(lib):
     """Host checks of the fused activation path: nothing is launched on error."""
     L = lib.quartz_linear_f16
