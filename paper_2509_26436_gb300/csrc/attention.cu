@@ -19,12 +19,19 @@
 //     once per CTA) with the key codes placed in the high nibble of each
 //     byte (16 c), shifted per subgroup by the key's FLAG — the paper's
 //     accumulator-shift schedule (Section 4.4) on the key side, exact.
-//     Softmax: running maximum and sum per CTA in the log2 domain.  Values:
-//     16 threads per token row (one 32-bit word of 8 codes each) x 8 token
-//     slots; each code becomes a float exactly through the 2^23 magic
-//     number, and o += p_t s_v 2^FLAG c in fp32.  The value words of a tile
-//     are loaded before the key arithmetic so that both DRAM round trips
-//     overlap.  Output per CTA: unnormalised o, running max, running sum.
+//     Softmax: running maximum and sum per CTA in the log2 domain; each key
+//     thread then writes p_t s_v 2^FLAG for its token's value subgroups
+//     (the FLAG added to the scale's exponent field).  Values: 16 threads
+//     per token row (one 32-bit word of 8 codes each) x 8 token slots; each
+//     code becomes a float exactly through the 2^23 magic number, and
+//     o += p_t s_v 2^FLAG c with paired f32x2 subtract and fused
+//     multiply-add (two instructions per two codes).  The code tiles of
+//     both caches (8 KB each per 128 tokens) stream through a 2-stage
+//     shared-memory ring filled by cp.async (chunks XOR-swizzled against
+//     bank conflicts) one tile ahead (more stages measured slower: fewer
+//     CTAs fit an SM); FLAGs and scales of the next tile are prefetched
+//     into registers.  Output per CTA: unnormalised o, running
+//     max, running sum.
 //   attn_combine_kernel: one CTA per bh merges the splits.
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
@@ -60,22 +67,6 @@ struct AttnArgs {
     float scale_log2;  // softmax scale * log2(e)
     float *part;       // [BH][n_split][kPartStride]
 };
-
-__device__ __forceinline__ uint32_t ldg_nc(const uint32_t *p)
-{
-    uint32_t v;
-    asm volatile("ld.global.nc.L1::no_allocate.u32 %0, [%1];" : "=r"(v) : "l"(p));
-    return v;
-}
-
-__device__ __forceinline__ uint4 ldg_nc4(const uint4 *p)
-{
-    uint4 v;
-    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
-                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-                 : "l"(p));
-    return v;
-}
 
 // The FLAG bytes (or nibbles) of one token row: S = 128 / G_s subgroups,
 // stored at subgroup index row * S + j (one byte each, or two per byte).
@@ -113,21 +104,99 @@ __device__ __forceinline__ float2 load_scales2(const __half *scales, int64_t row
     return __half22float2(*reinterpret_cast<const __half2 *>(&w));
 }
 
-// Byte permute selecting byte `b` of {hi:lo} into byte 0 (see prmt_b32).
-__device__ __forceinline__ float code_to_float(uint32_t biased_bytes, uint32_t sel)
+// The float 2^23 + (c + 8) for the biased code byte selected by `sel` (byte
+// b of `biased_bytes` into byte 0, 0x4B above it: 0x4B0000xx = 2^23 + xx).
+__device__ __forceinline__ float magic_float(uint32_t biased_bytes, uint32_t sel)
 {
-    // biased byte = c + 8 in [0, 15]; 0x4B0000xx is the float 2^23 + xx
-    return __int_as_float(prmt_b32(biased_bytes, 0x4B000000u, sel)) - 8388616.0f;
+    return __int_as_float(prmt_b32(biased_bytes, 0x4B000000u, sel));
 }
+
+__device__ __forceinline__ uint4 lds_u4(uint32_t addr)
+{
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr));
+    return v;
+}
+
+__device__ __forceinline__ uint32_t lds_u32(uint32_t addr)
+{
+    uint32_t v;
+    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(addr));
+    return v;
+}
+
+// s v 2^F for a float s that is 0 or normal: the exponent field grows by F
+// (exact; for s = 0 the result is a tiny normal, only ever multiplied by 0).
+__device__ __forceinline__ float scale_pow2(float s, int F)
+{
+    return __int_as_float(__float_as_int(s) + (F << 23));
+}
+
+// (acc0, acc1) += p * (c0, c1), where c = f - (2^23 + 8) for the magic floats
+// f: one paired subtraction and one paired fused multiply-add.
+__device__ __forceinline__ void fma_codes2(float &acc0, float &acc1, float p, float f0, float f1)
+{
+    asm("{\n\t.reg .b64 f, m, c, pp, acc;\n\t"
+        "mov.b64 f, {%2, %3};\n\t"
+        "mov.b64 m, {%5, %5};\n\t"
+        "add.rn.f32x2 c, f, m;\n\t"
+        "mov.b64 pp, {%4, %4};\n\t"
+        "mov.b64 acc, {%0, %1};\n\t"
+        "fma.rn.f32x2 acc, pp, c, acc;\n\t"
+        "mov.b64 {%0, %1}, acc;\n\t}"
+        : "+f"(acc0), "+f"(acc1)
+        : "f"(f0), "f"(f1), "f"(p), "f"(-8388616.0f));
+}
+
+// Asynchronous 16-byte global -> shared copies (cp.async, completion tracked
+// per thread in commit groups; the wait is the hardware's own).
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src)
+{
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+// Shared-memory offset of 16-byte chunk c (0..3) of token row r in a code
+// tile: rows of 64 bytes, chunks XOR-swizzled by (r / 2) % 4 so that eight
+// consecutive rows reading the same chunk hit eight different bank groups.
+__device__ __forceinline__ uint32_t tile_off(int r, int c) { return r * 64 + ((c ^ ((r >> 1) & 3)) << 4); }
+
+// The FLAGs and scales of one token row of the key and value caches.
+struct RowSide {
+    uint32_t kf[4], vf[4];
+    float2 sk, sv;
+};
+
+template <int GS>
+__device__ __forceinline__ void load_side(const AttnArgs &a, int64_t row, bool valid, RowSide &r)
+{
+    if (valid) {
+        load_row_flags<GS>(a.k_flags, row, a.k_packed != 0, r.kf);
+        load_row_flags<GS>(a.v_flags, row, a.v_packed != 0, r.vf);
+        r.sk = load_scales2(a.k_scales, row);
+        r.sv = load_scales2(a.v_scales, row);
+    } else {
+        r.kf[0] = r.kf[1] = r.kf[2] = r.kf[3] = 0u;
+        r.vf[0] = r.vf[1] = r.vf[2] = r.vf[3] = 0u;
+        r.sk = r.sv = make_float2(0.f, 0.f);
+    }
+}
+
+constexpr int kStages = 2;                     // code tiles in flight per CTA
+constexpr int kTileBytes = kTile * kD / 2;     // 8 KB of codes per tile and cache
+constexpr int kAttnDynSmem = kStages * 2 * kTileBytes;
 
 template <int GS>
 __global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(const __grid_constant__ AttnArgs a)
 {
     constexpr int S = kD / GS;            // subgroups per row
     constexpr int kWordsPerSub = GS / 8;  // code words per subgroup
-    __shared__ float s_p[kTile];          // softmax weights of the tile
-    __shared__ float s_fv[kTile][S + 1];  // value factors s_v 2^FLAG per token and subgroup
+    extern __shared__ __align__(128) uint8_t s_ring[];  // [kStages][K, V][kTileBytes]
+    __shared__ float s_pf[kTile][S + 1];  // p_t s_v 2^FLAG per token and subgroup
     __shared__ float s_red[kSlots][kD];   // final reduction over token slots
+    __shared__ uint32_t s_q[2 * kWords];  // the query's decoded values (even, odd codes)
     __shared__ float s_wmax[kAttnThreads / 32];
     __shared__ float s_wsum[kAttnThreads / 32];
 
@@ -136,30 +205,61 @@ __global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(const __grid_
     const int64_t bh = blockIdx.y;
     const int t_begin = split * a.chunk;
     const int t_end = min(t_begin + a.chunk, a.L);
+    const int n_tiles = (t_end - t_begin + kTile - 1) / kTile;
+    const uint32_t ring = static_cast<uint32_t>(__cvta_generic_to_shared(s_ring));
+    const uint8_t *kbytes = reinterpret_cast<const uint8_t *>(a.k_codes);
+    const uint8_t *vbytes = reinterpret_cast<const uint8_t *>(a.v_codes);
+
+    // Copies of tile `it` (both caches) into stage it % kStages; every thread
+    // commits one group per call, empty past the last tile.
+    auto issue = [&](int it) {
+        if (it < n_tiles) {
+            const int tile = t_begin + it * kTile;
+            const uint32_t kdst = ring + (it % kStages) * 2 * kTileBytes;
+            const uint32_t vdst = kdst + kTileBytes;
+#pragma unroll
+            for (int k = 0; k < kTileBytes / 16 / kAttnThreads; ++k) {
+                const int ci = tid + k * kAttnThreads;
+                const int r = ci >> 2, c = ci & 3;
+                if (tile + r < t_end) {
+                    const int64_t src = (bh * a.L_max + tile + r) * (kD / 2) + c * 16;
+                    cp_async16(kdst + tile_off(r, c), kbytes + src);
+                    cp_async16(vdst + tile_off(r, c), vbytes + src);
+                }
+            }
+        }
+        cp_async_commit();
+    };
+#pragma unroll
+    for (int it = 0; it < kStages - 1; ++it) issue(it);
 
     // ---- the query's decoded values, as int8 (even codes, odd codes) -------
-    uint32_t qe[kWords], qo[kWords];
-    float sq0, sq1;
-    {
+    // decoded once per CTA by the first 16 threads (one code word each)
+    if (tid < kWords) {
         uint32_t f[4];
         load_row_flags<GS>(a.q_flags, bh, a.q_packed != 0, f);
-        const float2 s2 = load_scales2(a.q_scales, bh);
-        sq0 = s2.x, sq1 = s2.y;
+        const uint32_t word = a.q_codes[bh * kWords + tid];
+        const int F = row_flag(f, tid / kWordsPerSub, a.q_packed != 0);
+        uint32_t e = 0u, o = 0u;
 #pragma unroll
-        for (int w = 0; w < kWords; ++w) {
-            const uint32_t word = a.q_codes[bh * kWords + w];
-            const int F = row_flag(f, w / kWordsPerSub, a.q_packed != 0);
-            uint32_t e = 0u, o = 0u;
-#pragma unroll
-            for (int b = 0; b < 4; ++b) {
-                const int c0 = static_cast<int>(word << (28 - 8 * b)) >> 28;  // code 2b
-                const int c1 = static_cast<int>(word << (24 - 8 * b)) >> 28;  // code 2b + 1
-                e |= (static_cast<uint32_t>(c0 * (1 << F)) & 0xFFu) << (8 * b);
-                o |= (static_cast<uint32_t>(c1 * (1 << F)) & 0xFFu) << (8 * b);
-            }
-            qe[w] = e;
-            qo[w] = o;
+        for (int b = 0; b < 4; ++b) {
+            const int c0 = static_cast<int>(word << (28 - 8 * b)) >> 28;  // code 2b
+            const int c1 = static_cast<int>(word << (24 - 8 * b)) >> 28;  // code 2b + 1
+            e |= (static_cast<uint32_t>(c0 * (1 << F)) & 0xFFu) << (8 * b);
+            o |= (static_cast<uint32_t>(c1 * (1 << F)) & 0xFFu) << (8 * b);
         }
+        s_q[tid] = e;
+        s_q[kWords + tid] = o;
+    }
+    const float2 sq = load_scales2(a.q_scales, bh);
+    RowSide cur;
+    load_side<GS>(a, bh * a.L_max + t_begin + tid, t_begin + tid < t_end, cur);
+    __syncthreads();
+    uint32_t qe[kWords], qo[kWords];
+#pragma unroll
+    for (int w = 0; w < kWords; ++w) {
+        qe[w] = s_q[w];
+        qo[w] = s_q[kWords + w];
     }
 
     const int vw = tid % kWords;   // value phase: code word of this thread
@@ -171,31 +271,27 @@ __global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(const __grid_
     float m_run = -INFINITY;  // running maximum (log2 domain)
     float l_thr = 0.f;        // this thread's share of the running sum
 
-    for (int tile = t_begin; tile < t_end; tile += kTile) {
-        // value words of this tile (independent of the scores): issue first
-        uint32_t vwords[kTile / kSlots];
-#pragma unroll
-        for (int i = 0; i < kTile / kSlots; ++i) {
-            const int t = tile + slot + i * kSlots;
-            vwords[i] = t < t_end ? ldg_nc(a.v_codes + (bh * a.L_max + t) * kWords + vw) : 0u;
-        }
+    for (int it = 0; it < n_tiles; ++it) {
+        const int tile = t_begin + it * kTile;
+        issue(it + kStages - 1);     // into the stage tile it - 1 used
+        cp_async_wait<kStages - 1>();  // this thread's copies of tile `it` have landed
+        __syncthreads();     // ... and everyone else's
+        const uint32_t kst = ring + (it % kStages) * 2 * kTileBytes;
+        const uint32_t vst = kst + kTileBytes;
+        // FLAGs and scales of the next tile, while this one is processed
+        RowSide nxt;
+        load_side<GS>(a, bh * a.L_max + tile + kTile + tid, tile + kTile + tid < t_end, nxt);
 
         // ---- keys: one token per thread -----------------------------------
-        const int t = tile + tid;
-        const bool valid = t < t_end;
+        const bool valid = tile + tid < t_end;
         float s2 = -INFINITY;
         if (valid) {
-            const int64_t row = bh * a.L_max + t;
-            uint4 kc[4];
+            uint32_t kw[kWords];
 #pragma unroll
-            for (int i = 0; i < 4; ++i) kc[i] = ldg_nc4(reinterpret_cast<const uint4 *>(a.k_codes + row * kWords) + i);
-            uint32_t kf[4], vf[4];
-            load_row_flags<GS>(a.k_flags, row, a.k_packed != 0, kf);
-            load_row_flags<GS>(a.v_flags, row, a.v_packed != 0, vf);
-            const float2 sk = load_scales2(a.k_scales, row);
-            const float2 sv = load_scales2(a.v_scales, row);
-            const uint32_t kw[kWords] = {kc[0].x, kc[0].y, kc[0].z, kc[0].w, kc[1].x, kc[1].y, kc[1].z, kc[1].w,
-                                         kc[2].x, kc[2].y, kc[2].z, kc[2].w, kc[3].x, kc[3].y, kc[3].z, kc[3].w};
+            for (int c = 0; c < 4; ++c) {
+                const uint4 v = lds_u4(kst + tile_off(tid, c));
+                kw[4 * c] = v.x, kw[4 * c + 1] = v.y, kw[4 * c + 2] = v.z, kw[4 * c + 3] = v.w;
+            }
             int P[2] = {0, 0};
 #pragma unroll
             for (int j = 0; j < S; ++j) {
@@ -205,15 +301,11 @@ __global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(const __grid_
                     dot = __dp4a(static_cast<int>(qe[w]), static_cast<int>((kw[w] << 4) & 0xF0F0F0F0u), dot);
                     dot = __dp4a(static_cast<int>(qo[w]), static_cast<int>(kw[w] & 0xF0F0F0F0u), dot);
                 }
-                P[(j * GS) / 64] += (dot >> 4) * (1 << row_flag(kf, j, a.k_packed != 0));
-                s_fv[tid][j] = ldexpf((j * GS) / 64 ? sv.y : sv.x, row_flag(vf, j, a.v_packed != 0));
+                P[(j * GS) / 64] += (dot >> 4) * (1 << row_flag(cur.kf, j, a.k_packed != 0));
             }
-            const float sc = __fmul_rn(__fmul_rn(sq0, sk.x), static_cast<float>(P[0])) +
-                             __fmul_rn(__fmul_rn(sq1, sk.y), static_cast<float>(P[1]));
+            const float sc = __fmul_rn(__fmul_rn(sq.x, cur.sk.x), static_cast<float>(P[0])) +
+                             __fmul_rn(__fmul_rn(sq.y, cur.sk.y), static_cast<float>(P[1]));
             s2 = sc * a.scale_log2;
-        } else {
-#pragma unroll
-            for (int j = 0; j < S; ++j) s_fv[tid][j] = 0.f;
         }
 
         // ---- softmax: tile maximum, rescale, weights ----------------------
@@ -229,7 +321,9 @@ __global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(const __grid_
         const float alpha = exp2f(m_run - m_new);  // 0 on the first tile
         const float p = valid ? exp2f(s2 - m_new) : 0.f;
         l_thr = l_thr * alpha + p;
-        s_p[tid] = p;
+#pragma unroll
+        for (int j = 0; j < S; ++j)  // p_t s_v 2^FLAG of every value subgroup (0 past the end)
+            s_pf[tid][j] = p * scale_pow2((j * GS) / 64 ? cur.sv.y : cur.sv.x, row_flag(cur.vf, j, a.v_packed != 0));
 #pragma unroll
         for (int k = 0; k < 8; ++k) acc[k] *= alpha;
         m_run = m_new;
@@ -239,18 +333,18 @@ __global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(const __grid_
 #pragma unroll
         for (int i = 0; i < kTile / kSlots; ++i) {
             const int ti = slot + i * kSlots;
-            const float pf = s_p[ti] * s_fv[ti][vsub];  // 0 for tokens past the end
-            const uint32_t word = vwords[i];
+            const float pf = s_pf[ti][vsub];  // 0 for tokens past the end
+            const uint32_t word = lds_u32(vst + tile_off(ti, vw >> 2) + 4 * (vw & 3));
             const uint32_t ev = (word & 0x0F0F0F0Fu) ^ 0x08080808u;         // codes 0, 2, 4, 6 as c + 8
             const uint32_t od = ((word >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u;  // codes 1, 3, 5, 7
 #pragma unroll
-            for (int b = 0; b < 4; ++b) {
-                acc[2 * b] = fmaf(pf, code_to_float(ev, 0x7440u | b), acc[2 * b]);
-                acc[2 * b + 1] = fmaf(pf, code_to_float(od, 0x7440u | b), acc[2 * b + 1]);
-            }
+            for (int b = 0; b < 4; ++b)
+                fma_codes2(acc[2 * b], acc[2 * b + 1], pf, magic_float(ev, 0x7440u | b), magic_float(od, 0x7440u | b));
         }
-        __syncthreads();  // s_p / s_fv are rewritten by the next tile
+        cur = nxt;
+        __syncthreads();  // s_pf and this stage are rewritten later
     }
+    cp_async_wait<0>();
 
     // ---- reduce over token slots, write this split's partial result -------
 #pragma unroll
@@ -293,6 +387,16 @@ __global__ void __launch_bounds__(kD) attn_combine_kernel(const float *__restric
     if (OUT == QUARTZ_OUT_F16) static_cast<__half *>(out)[off] = __float2half_rn(v);
     else if (OUT == QUARTZ_OUT_BF16) static_cast<__nv_bfloat16 *>(out)[off] = __float2bfloat16_rn(v);
     else static_cast<float *>(out)[off] = v;
+}
+
+template <int GS>
+cudaError_t launch_decode(dim3 grid, const AttnArgs &a, cudaStream_t s)
+{
+    cudaError_t e = cudaFuncSetAttribute(attn_decode_kernel<GS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         kAttnDynSmem);
+    if (e != cudaSuccess) return e;
+    attn_decode_kernel<GS><<<grid, kAttnThreads, kAttnDynSmem, s>>>(a);
+    return cudaGetLastError();
 }
 
 int attn_splits(int64_t BH, int64_t L, int *chunk)
@@ -345,13 +449,13 @@ cudaError_t launch_attention_decode(const quartz_encoded_t *q, const quartz_enco
     a.scale_log2 = scale * kLog2e;
     a.part = static_cast<float *>(workspace);
     const dim3 grid(static_cast<unsigned>(a.n_split), static_cast<unsigned>(BH));
+    cudaError_t e;
     switch (q->p.group_s) {
-        case 8: attn_decode_kernel<8><<<grid, kAttnThreads, 0, s>>>(a); break;
-        case 16: attn_decode_kernel<16><<<grid, kAttnThreads, 0, s>>>(a); break;
-        case 32: attn_decode_kernel<32><<<grid, kAttnThreads, 0, s>>>(a); break;
-        default: attn_decode_kernel<64><<<grid, kAttnThreads, 0, s>>>(a); break;
+        case 8: e = launch_decode<8>(grid, a, s); break;
+        case 16: e = launch_decode<16>(grid, a, s); break;
+        case 32: e = launch_decode<32>(grid, a, s); break;
+        default: e = launch_decode<64>(grid, a, s); break;
     }
-    cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     const unsigned cb = static_cast<unsigned>(BH);
     if (o_type == QUARTZ_OUT_F16) attn_combine_kernel<QUARTZ_OUT_F16><<<cb, kD, 0, s>>>(a.part, a.n_split, o);
