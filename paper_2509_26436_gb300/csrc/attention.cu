@@ -21,8 +21,8 @@
 //     accumulator-shift schedule (Section 4.4) on the key side, exact.
 //     Softmax: running maximum and sum per CTA in the log2 domain; each key
 //     thread then writes p_t s_v 2^FLAG for its token's value subgroups
-//     (the FLAG added to the scale's exponent field).  Values: 16 threads
-//     per token row (one 32-bit word of 8 codes each) x 8 token slots; each
+//     (the FLAG added to the scale's exponent field).  Values: 4 threads per
+//     token row (one 16-byte chunk of 32 codes each) x 32 token slots; each
 //     code becomes a float exactly through the 2^23 magic number, and
 //     o += p_t s_v 2^FLAG c with paired f32x2 subtract and fused
 //     multiply-add (two instructions per two codes).  The code tiles of
@@ -46,7 +46,9 @@ constexpr int kD = 128;              // head dimension
 constexpr int kWords = kD / 8;       // 32-bit code words per token row
 constexpr int kTile = 128;           // tokens per tile = threads per CTA
 constexpr int kAttnThreads = 128;
-constexpr int kSlots = kAttnThreads / kWords;  // token slots of the value phase
+constexpr int kChunksPerRow = 4;               // 16-byte code chunks (32 codes) per token row
+constexpr int kSlots = kAttnThreads / kChunksPerRow;  // token slots of the value phase
+constexpr int kPfStride = kTile + 2;           // s_pf row stride: conflict-free reads and writes
 constexpr int kPartStride = kD + 4;  // o[128], m, l (+ pad) per split
 constexpr int kMaxSplits = 64;
 constexpr float kLog2e = 1.4426950408889634f;
@@ -118,13 +120,6 @@ __device__ __forceinline__ uint4 lds_u4(uint32_t addr)
     return v;
 }
 
-__device__ __forceinline__ uint32_t lds_u32(uint32_t addr)
-{
-    uint32_t v;
-    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(addr));
-    return v;
-}
-
 // s v 2^F for a float s that is 0 or normal: the exponent field grows by F
 // (exact; for s = 0 the result is a tiny normal, only ever multiplied by 0).
 __device__ __forceinline__ float scale_pow2(float s, int F)
@@ -187,6 +182,7 @@ __device__ __forceinline__ void load_side(const AttnArgs &a, int64_t row, bool v
 constexpr int kStages = 2;                     // code tiles in flight per CTA
 constexpr int kTileBytes = kTile * kD / 2;     // 8 KB of codes per tile and cache
 constexpr int kAttnDynSmem = kStages * 2 * kTileBytes;
+static_assert(kAttnThreads * 33 * 4 <= kAttnDynSmem, "slot reduction fits the code ring");
 
 template <int GS>
 __global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(const __grid_constant__ AttnArgs a)
@@ -194,9 +190,8 @@ __global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(const __grid_
     constexpr int S = kD / GS;            // subgroups per row
     constexpr int kWordsPerSub = GS / 8;  // code words per subgroup
     extern __shared__ __align__(128) uint8_t s_ring[];  // [kStages][K, V][kTileBytes]
-    __shared__ float s_pf[kTile][S + 1];  // p_t s_v 2^FLAG per token and subgroup
-    __shared__ float s_red[kSlots][kD];   // final reduction over token slots
-    __shared__ uint32_t s_q[2 * kWords];  // the query's decoded values (even, odd codes)
+    __shared__ float s_pf[S][kPfStride];  // p_t s_v 2^FLAG per value subgroup and token
+    __shared__ __align__(16) uint32_t s_q[2 * kWords];  // the query's decoded values (even, odd codes)
     __shared__ float s_wmax[kAttnThreads / 32];
     __shared__ float s_wsum[kAttnThreads / 32];
 
@@ -255,19 +250,13 @@ __global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(const __grid_
     RowSide cur;
     load_side<GS>(a, bh * a.L_max + t_begin + tid, t_begin + tid < t_end, cur);
     __syncthreads();
-    uint32_t qe[kWords], qo[kWords];
-#pragma unroll
-    for (int w = 0; w < kWords; ++w) {
-        qe[w] = s_q[w];
-        qo[w] = s_q[kWords + w];
-    }
+    const uint32_t sq_addr = static_cast<uint32_t>(__cvta_generic_to_shared(s_q));
 
-    const int vw = tid % kWords;   // value phase: code word of this thread
-    const int slot = tid / kWords; // value phase: token slot
-    const int vsub = vw / kWordsPerSub;
-    float acc[8];
+    const int vc = tid % kChunksPerRow;  // value phase: 16-byte code chunk (dims 32 vc ..)
+    const int slot = tid / kChunksPerRow; // value phase: token slot
+    float acc[32];
 #pragma unroll
-    for (int k = 0; k < 8; ++k) acc[k] = 0.f;
+    for (int k = 0; k < 32; ++k) acc[k] = 0.f;
     float m_run = -INFINITY;  // running maximum (log2 domain)
     float l_thr = 0.f;        // this thread's share of the running sum
 
@@ -286,11 +275,15 @@ __global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(const __grid_
         const bool valid = tile + tid < t_end;
         float s2 = -INFINITY;
         if (valid) {
-            uint32_t kw[kWords];
+            uint32_t kw[kWords], qe[kWords], qo[kWords];  // the query words: broadcast shared loads
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
                 const uint4 v = lds_u4(kst + tile_off(tid, c));
                 kw[4 * c] = v.x, kw[4 * c + 1] = v.y, kw[4 * c + 2] = v.z, kw[4 * c + 3] = v.w;
+                const uint4 e = lds_u4(sq_addr + 16 * c);
+                qe[4 * c] = e.x, qe[4 * c + 1] = e.y, qe[4 * c + 2] = e.z, qe[4 * c + 3] = e.w;
+                const uint4 o = lds_u4(sq_addr + 4 * kWords + 16 * c);
+                qo[4 * c] = o.x, qo[4 * c + 1] = o.y, qo[4 * c + 2] = o.z, qo[4 * c + 3] = o.w;
             }
             int P[2] = {0, 0};
 #pragma unroll
@@ -323,9 +316,9 @@ __global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(const __grid_
         l_thr = l_thr * alpha + p;
 #pragma unroll
         for (int j = 0; j < S; ++j)  // p_t s_v 2^FLAG of every value subgroup (0 past the end)
-            s_pf[tid][j] = p * scale_pow2((j * GS) / 64 ? cur.sv.y : cur.sv.x, row_flag(cur.vf, j, a.v_packed != 0));
+            s_pf[j][tid] = p * scale_pow2((j * GS) / 64 ? cur.sv.y : cur.sv.x, row_flag(cur.vf, j, a.v_packed != 0));
 #pragma unroll
-        for (int k = 0; k < 8; ++k) acc[k] *= alpha;
+        for (int k = 0; k < 32; ++k) acc[k] *= alpha;
         m_run = m_new;
         __syncthreads();
 
@@ -333,13 +326,20 @@ __global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(const __grid_
 #pragma unroll
         for (int i = 0; i < kTile / kSlots; ++i) {
             const int ti = slot + i * kSlots;
-            const float pf = s_pf[ti][vsub];  // 0 for tokens past the end
-            const uint32_t word = lds_u32(vst + tile_off(ti, vw >> 2) + 4 * (vw & 3));
-            const uint32_t ev = (word & 0x0F0F0F0Fu) ^ 0x08080808u;         // codes 0, 2, 4, 6 as c + 8
-            const uint32_t od = ((word >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u;  // codes 1, 3, 5, 7
+            const uint4 ch = lds_u4(vst + tile_off(ti, vc));
+            const uint32_t words[4] = {ch.x, ch.y, ch.z, ch.w};
 #pragma unroll
-            for (int b = 0; b < 4; ++b)
-                fma_codes2(acc[2 * b], acc[2 * b + 1], pf, magic_float(ev, 0x7440u | b), magic_float(od, 0x7440u | b));
+            for (int w = 0; w < 4; ++w) {
+                // word 4 vc + w of the row; its subgroup's factor (0 past the end)
+                const int sub = (4 * vc + w) / kWordsPerSub;
+                const float pf = s_pf[sub][ti];
+                const uint32_t ev = (words[w] & 0x0F0F0F0Fu) ^ 0x08080808u;         // codes 0, 2, 4, 6 as c + 8
+                const uint32_t od = ((words[w] >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u;  // codes 1, 3, 5, 7
+#pragma unroll
+                for (int b = 0; b < 4; ++b)
+                    fma_codes2(acc[8 * w + 2 * b], acc[8 * w + 2 * b + 1], pf, magic_float(ev, 0x7440u | b),
+                               magic_float(od, 0x7440u | b));
+            }
         }
         cur = nxt;
         __syncthreads();  // s_pf and this stage are rewritten later
@@ -347,16 +347,21 @@ __global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(const __grid_
     cp_async_wait<0>();
 
     // ---- reduce over token slots, write this split's partial result -------
+    // (the code ring is free now: thread (slot, vc) stores its 32 sums at
+    // (4 slot + vc) * 33, which keeps both the stores and the column reads
+    // below free of bank conflicts)
+    __syncthreads();
+    float *s_red = reinterpret_cast<float *>(s_ring);
 #pragma unroll
-    for (int k = 0; k < 8; ++k) s_red[slot][vw * 8 + k] = acc[k];
+    for (int k = 0; k < 32; ++k) s_red[(slot * kChunksPerRow + vc) * 33 + k] = acc[k];
     float ws = l_thr;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) ws += __shfl_xor_sync(0xffffffffu, ws, o);
     if ((tid & 31) == 0) s_wsum[tid >> 5] = ws;
     __syncthreads();
     float od = 0.f;
-#pragma unroll
-    for (int sl = 0; sl < kSlots; ++sl) od += s_red[sl][tid];
+#pragma unroll 8
+    for (int sl = 0; sl < kSlots; ++sl) od += s_red[(sl * kChunksPerRow + tid / 32) * 33 + (tid & 31)];
     float *part = a.part + (bh * a.n_split + split) * kPartStride;
     part[tid] = od;
     if (tid == 0) {
@@ -389,30 +394,47 @@ __global__ void __launch_bounds__(kD) attn_combine_kernel(const float *__restric
     else static_cast<float *>(out)[off] = v;
 }
 
-template <int GS>
-cudaError_t launch_decode(dim3 grid, const AttnArgs &a, cudaStream_t s)
+// Splits of the L axis per head.  Every CTA streams ceil(tiles / n) tiles
+// plus about one tile's worth of fixed cost; with `per_wave` CTAs resident at
+// once the step takes ceil(BH n / per_wave) waves of that, which this picks
+// the smallest of (ties: fewer CTAs).
+int attn_splits(int64_t BH, int64_t L, int64_t per_wave, int *chunk)
 {
+    const int64_t tiles = (L + kTile - 1) / kTile;
+    const int64_t max_split = tiles < kMaxSplits ? tiles : kMaxSplits;
+    int64_t best_n = 1, best_cost = -1;
+    for (int64_t n = 1; n <= max_split; ++n) {
+        const int64_t per = (tiles + n - 1) / n;
+        if ((tiles + per - 1) / per != n) continue;  // some split would get no tile
+        const int64_t waves = (BH * n + per_wave - 1) / per_wave;
+        const int64_t cost = waves * (per + 1);
+        if (best_cost < 0 || cost < best_cost) best_cost = cost, best_n = n;
+    }
+    *chunk = static_cast<int>(((tiles + best_n - 1) / best_n) * kTile);
+    return static_cast<int>(best_n);
+}
+
+template <int GS>
+cudaError_t launch_decode(int64_t BH, AttnArgs &a, cudaStream_t s)
+{
+    static int occ = 0;  // resident CTAs per SM of this instance
     cudaError_t e = cudaFuncSetAttribute(attn_decode_kernel<GS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          kAttnDynSmem);
     if (e != cudaSuccess) return e;
-    attn_decode_kernel<GS><<<grid, kAttnThreads, kAttnDynSmem, s>>>(a);
-    return cudaGetLastError();
-}
-
-int attn_splits(int64_t BH, int64_t L, int *chunk)
-{
+    if (occ == 0) {
+        int n = 0;
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attn_decode_kernel<GS>, kAttnThreads, kAttnDynSmem);
+        if (e != cudaSuccess) return e;
+        occ = n > 0 ? n : 1;
+    }
     int dev = 0, sms = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (sms <= 0) sms = 1;
-    const int64_t tiles = (L + kTile - 1) / kTile;
-    const int64_t max_split = tiles < kMaxSplits ? tiles : kMaxSplits;
-    int64_t n = (8 * static_cast<int64_t>(sms) + BH - 1) / BH;  // about 8 CTAs per SM
-    if (n < 1) n = 1;
-    if (n > max_split) n = max_split;
-    const int64_t per = (tiles + n - 1) / n;  // tiles per split
-    *chunk = static_cast<int>(per * kTile);
-    return static_cast<int>((tiles + per - 1) / per);
+    a.n_split = attn_splits(BH, a.L, static_cast<int64_t>(sms) * occ, &a.chunk);
+    const dim3 grid(static_cast<unsigned>(a.n_split), static_cast<unsigned>(BH));
+    attn_decode_kernel<GS><<<grid, kAttnThreads, kAttnDynSmem, s>>>(a);
+    return cudaGetLastError();
 }
 
 }  // namespace
@@ -445,16 +467,14 @@ cudaError_t launch_attention_decode(const quartz_encoded_t *q, const quartz_enco
     a.v_packed = v->p.flag_bits == 4;
     a.L_max = L_max;
     a.L = static_cast<int>(L);
-    a.n_split = attn_splits(BH, L, &a.chunk);
     a.scale_log2 = scale * kLog2e;
     a.part = static_cast<float *>(workspace);
-    const dim3 grid(static_cast<unsigned>(a.n_split), static_cast<unsigned>(BH));
     cudaError_t e;
     switch (q->p.group_s) {
-        case 8: e = launch_decode<8>(grid, a, s); break;
-        case 16: e = launch_decode<16>(grid, a, s); break;
-        case 32: e = launch_decode<32>(grid, a, s); break;
-        default: e = launch_decode<64>(grid, a, s); break;
+        case 8: e = launch_decode<8>(BH, a, s); break;
+        case 16: e = launch_decode<16>(BH, a, s); break;
+        case 32: e = launch_decode<32>(BH, a, s); break;
+        default: e = launch_decode<64>(BH, a, s); break;
     }
     if (e != cudaSuccess) return e;
     const unsigned cb = static_cast<unsigned>(BH);
