@@ -51,12 +51,12 @@ def parse():
     p.add_argument("--compare-algos", action="store_true",
                    help="also time the three GEMM algorithms (tcgen05, simt, shift) on each layer")
     p.add_argument("--layers", default="", help="comma-separated subset of layer names (profiling)")
-    p.add_argument("--attention", action="store_true",
-                   help="also time the attention decode step (Appendix D, Table 6: heads x 128, "
-                        "G_s 8/16/32) over a 4096-token encoded cache, batch 16")
-    p.add_argument("--llm", action="store_true",
-                   help="also time the LLM variant (Section 5: 16-bit codes straight to 4 bits, "
-                        "G_s = 8) on LLaMA-2-7B block linears")
+    p.add_argument("--no-attention", dest="attention", action="store_false",
+                   help="skip the attention decode step leg (Appendix D, Table 6: heads x 128, "
+                        "G_s 8/16/32, a 4096-token encoded cache, batch 16)")
+    p.add_argument("--no-llm", dest="llm", action="store_false",
+                   help="skip the LLM-variant leg (Section 5: 16-bit codes straight to 4 bits, "
+                        "G_s = 8, LLaMA-2-7B block linears)")
     return p.parse_args()
 
 
