@@ -108,6 +108,17 @@ def gemm_traffic():
     return float(kv["dram_bytes_per_launch"])
 
 
+def max_over_ranks(t, world, device=None):
+    """The slowest rank's time: the whole job finishes when its last rank does."""
+    if world <= 1:
+        return t
+    import torch
+    import torch.distributed as dist
+    x = torch.tensor([t], dtype=torch.float64, device=device)
+    dist.all_reduce(x, op=dist.ReduceOp.MAX)
+    return float(x.item())
+
+
 def dist_env():
     return (int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)),
             int(os.environ.get("LOCAL_RANK", 0)))
@@ -336,11 +347,7 @@ def run_ours(args):
     status = Q.device_status()
     assert status == 0, f"device status {status}"
     t_step = t0.elapsed_time(t1) / 1e3 / args.steps
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([t_step], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        t_step = float(t.item())
+    t_step = max_over_ranks(t_step, world, dev)
 
     ops_step = sum(l.ops for l in layers)
     value = world * ops_step / t_step / 1e12
@@ -402,11 +409,7 @@ def run_ours(args):
         barrier()
         assert Q.device_status() == 0
         tf = f0.elapsed_time(f1) / 1e3 / args.steps
-        if world > 1:
-            import torch.distributed as dist
-            t = torch.tensor([tf], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            tf = float(t.item())
+        tf = max_over_ranks(tf, world, dev)
         fused = {"value": world * ops_step / tf / 1e12, "unit": "TOPS", "ms_per_step": tf * 1e3,
                  "path": "quartz_linear_f16 per layer (activations encoded straight into the GEMM "
                          "operand; bit-identical to quantize + linear)"}
@@ -485,11 +488,7 @@ def run_ours(args):
         torch.cuda.synchronize()
         barrier()
         te = a0.elapsed_time(a1) / 1e3 / e_steps
-        if world > 1:
-            import torch.distributed as dist
-            t = torch.tensor([te], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            te = float(t.item())
+        te = max_over_ranks(te, world, dev)
         e2e = {"value": world * ops_step / te / 1e12, "unit": "TOPS",
                "h2d_bytes_per_step": sum(x.numel() * 2 for x in x_host),
                "d2h_bytes_per_step": sum(l.M * l.N * 2 for l in layers), "steps": e_steps,
