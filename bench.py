@@ -119,6 +119,33 @@ def max_over_ranks(t, world, device=None):
     return float(x.item())
 
 
+def host_link_gbs(torch, dev, mib=256, reps=3):
+    """Pinned host <-> device copy rates (GB/s): H2D alone, D2H alone and the
+    two directions at once on two streams; best of `reps`."""
+    n = mib << 20
+    h_in = torch.empty(n, dtype=torch.uint8).pin_memory()
+    h_out = torch.empty(n, dtype=torch.uint8).pin_memory()
+    d_in = torch.empty(n, dtype=torch.uint8, device=dev)
+    d_out = torch.zeros(n, dtype=torch.uint8, device=dev)
+    s1, s2 = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+    best = {"h2d": 0.0, "d2h": 0.0, "both": 0.0}
+    for _ in range(reps):
+        for key in best:
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            if key in ("h2d", "both"):
+                with torch.cuda.stream(s1):
+                    d_in.copy_(h_in, non_blocking=True)
+            if key in ("d2h", "both"):
+                with torch.cuda.stream(s2):
+                    h_out.copy_(d_out, non_blocking=True)
+            torch.cuda.synchronize()
+            dt = time.perf_counter() - t0
+            moved = n * (2 if key == "both" else 1)
+            best[key] = max(best[key], moved / dt / 1e9)
+    return best
+
+
 def dist_env():
     return (int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)),
             int(os.environ.get("LOCAL_RANK", 0)))
@@ -489,11 +516,18 @@ def run_ours(args):
         barrier()
         te = a0.elapsed_time(a1) / 1e3 / e_steps
         te = max_over_ranks(te, world, dev)
+        h2d = sum(x.numel() * 2 for x in x_host)
+        d2h = sum(l.M * l.N * 2 for l in layers)
+        link = host_link_gbs(torch, dev)
+        floor = max(h2d / (link["h2d"] * 1e9), d2h / (link["d2h"] * 1e9), (h2d + d2h) / (link["both"] * 1e9))
         e2e = {"value": world * ops_step / te / 1e12, "unit": "TOPS",
-               "h2d_bytes_per_step": sum(x.numel() * 2 for x in x_host),
-               "d2h_bytes_per_step": sum(l.M * l.N * 2 for l in layers), "steps": e_steps,
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": e_steps,
                "ms_per_step": te * 1e3,
-               "overlap": "H2D / compute / D2H on three streams, double-buffered"}
+               "overlap": "H2D / compute / D2H on three streams, double-buffered",
+               "roofline": {"bound": "host link", "link_gbs_measured": link,
+                            "floor_ms": floor * 1e3, "frac": floor / te,
+                            "work": "the step's H2D and D2H bytes at the link rates measured here "
+                                    "(pinned 256 MiB copies, each direction alone and both at once)"}}
 
     # ---- CPU oracle baseline (rank 0 only, N = 1) ---------------------------
     cpu = None

@@ -313,6 +313,7 @@ int32_t quartz_attention_decode(const quartz_encoded_t *q, const quartz_encoded_
     if ((rc = check_attention_operand(v_cache, q->p.group_s)) != QUARTZ_OK) return rc;
     const int64_t BH = q->rows;
     if (BH > 65535 || L_max <= 0 || L <= 0 || L > L_max || L > (int64_t(1) << 30) ||
+        BH * ((L + 127) / 128) > (int64_t(1) << 31) ||
         k_cache->rows != BH * L_max || v_cache->rows != BH * L_max)
         return QUARTZ_ERR_INVALID_ARG;
     if (!(scale == scale) || scale > 3.0e38f || scale < -3.0e38f) return QUARTZ_ERR_INVALID_ARG;  // finite
