@@ -5,8 +5,9 @@ One step = the whole hot path over one batch: for each of the four MM-DiT
 block linears (QKV 3072->9216, proj 3072->3072, MLP 3072->12288 and
 12288->3072, M = (4096 + 512) tokens x batch 4 = 18432), quantize + LZS-encode
 the fp16 activations (Eq. 1, Eq. 2), expand the codes and run the tcgen05
-GEMM with its dequant epilogue (Section 4.4).  Weights are encoded once,
-offline, outside the timed region (as the paper's PTQ does).
+GEMM with its dequant epilogue (Section 4.4).  Weights are encoded, and
+their tensor-core operand prepared, once, offline, outside the timed region
+(as the paper's PTQ does).
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
@@ -320,6 +321,8 @@ def run_ours(args):
     per_row = args.scales == "per-row"
     gq = [l.K if per_row else GROUP_Q for l in layers]
     enc_w = [Q.encode_weights(torch.from_numpy(w).to(dev), group_s=GROUP_S, group_q=g) for w, g in zip(ws, gq)]
+    # weights are encoded and their tensor-core operand prepared once, offline
+    prep_w = [Q.prepare_weights(w) for w in enc_w]
     enc_a = [Q.empty_encoded(l.M, l.K, Q.Params(g, GROUP_S), dev) for l, g in zip(layers, gq)]
     y_dev = [torch.empty((l.M, l.N), dtype=torch.float16, device=dev) for l in layers]
     ws_bytes = max(Q.linear_workspace_size(l.M, l.N, l.K) for l in layers)
@@ -338,7 +341,7 @@ def run_ours(args):
             Q.quantize(x_dev[i], out=enc_a[i], group_s=GROUP_S, group_q=gq[i])
             if rec is not None:
                 rec["q"][i][1].record(stream)
-            Q.linear(enc_a[i], enc_w[i], out=y_dev[i], workspace=workspace,
+            Q.linear(enc_a[i], enc_w[i], out=y_dev[i], workspace=workspace, w_prepared=prep_w[i],
                      gemm_events=None if rec is None else rec["g"][i])
 
     def barrier():
@@ -397,7 +400,7 @@ def run_ours(args):
     elems = sum(l.M * l.K for l in layers)
     enc_bytes = sum(l.M * l.K * encode_bytes_per_elem(GROUP_S, g) for l, g in zip(layers, gq))
     enc_gbs = enc_bytes / (sum(quant_ms) / 1e3) / 1e9
-    launches_per_step = nl * 3   # quantize; prepare (both operands); GEMM
+    launches_per_step = nl * 3   # quantize; prepare (activations); GEMM
 
     alu_view = {"achieved": gemm_alu, "unit": "Top/s", "peak": alu_peak, "frac": gemm_alu / alu_peak,
                 "peak_source": f"derived: {n_sm} SMs x {FP32_LANES_PER_SM} fp32 lanes x "
@@ -494,7 +497,7 @@ def run_ours(args):
                 consumed[u].record(stream)
                 if u >= 2:
                     stream.wait_event(drained[u - 2])
-                Q.linear(enc_a[i], enc_w[i], out=y_buf[p][i], workspace=workspace)
+                Q.linear(enc_a[i], enc_w[i], out=y_buf[p][i], workspace=workspace, w_prepared=prep_w[i])
                 computed[u] = torch.cuda.Event()
                 computed[u].record(stream)
                 with torch.cuda.stream(s_out):
@@ -627,6 +630,7 @@ def run_llm_variant(args, Q, inputs, dev, n_sm, sm_mhz, peak_src, fp8_peak):
     x_dev = [torch.from_numpy(l.activations()).to(dev) for l in layers]
     enc_w = [Q.encode_weights(torch.from_numpy(l.weights()).to(dev), group_s=LLM_GROUP_S, code_bits=16)
              for l in layers]
+    prep_w = [Q.prepare_weights(w) for w in enc_w]
     enc_a = [Q.empty_encoded(l.M, l.K, Q.Params(GROUP_Q, LLM_GROUP_S, code_bits=16), dev) for l in layers]
     y_dev = [torch.empty((l.M, l.N), dtype=torch.float16, device=dev) for l in layers]
     workspace = torch.empty(max(Q.linear_workspace_size(l.M, l.N, l.K, enc_a[0].params) for l in layers),
@@ -645,7 +649,7 @@ def run_llm_variant(args, Q, inputs, dev, n_sm, sm_mhz, peak_src, fp8_peak):
                 Q.quantize(x_dev[i], out=enc_a[i], group_s=LLM_GROUP_S, code_bits=16)
                 if rec is not None:
                     rec[i][1].record(stream)
-                Q.linear(enc_a[i], enc_w[i], out=y_dev[i], workspace=workspace, algo=algo,
+                Q.linear(enc_a[i], enc_w[i], out=y_dev[i], workspace=workspace, algo=algo, w_prepared=prep_w[i],
                          gemm_events=None if rec is None else rec[i][2:])
 
         for _ in range(max(3, args.warmup)):

@@ -188,6 +188,7 @@ int32_t quartz_linear(const quartz_encoded_t *a, const quartz_encoded_t *w, cons
  *                     (8-bit codes only: QUARTZ_ERR_UNSUPPORTED with 16-bit
  *                     codes, whose partials need 64 bits)
  *   algo              quartz_algo_t: which GEMM kernel runs
+ *   w_prepared        NULL, or prepared weights (below)
  *   gemm_event_begin  NULL, or a cudaEvent_t recorded on `stream` right before
  *   gemm_event_end    / right after the GEMM kernel (after operand expansion),
  *                     so a caller can time the GEMM kernel alone */
@@ -197,7 +198,23 @@ typedef struct {
     int32_t algo;
     void *gemm_event_begin;
     void *gemm_event_end;
+    const void *w_prepared;  /* NULL, or the weights prepared by quartz_prepare_weights
+                              * from the same encoded `w`: the call then prepares the
+                              * activations only (same results) */
 } quartz_linear_opts_t;
+
+/* Bytes of a prepared weight operand for quartz_prepare_weights; 0 for
+ * invalid arguments (the shape rules of quartz_linear's weights). */
+size_t quartz_prepared_weights_size(int64_t N, int64_t K, const quartz_params_t *p);
+
+/* Prepare encoded weights [N, K] once (offline, like their encoding): their
+ * tensor-core operand (the decoded values, E4M3, or E5M2 for 16-bit codes)
+ * and transposed group scales, written to `prepared` (device memory owned by
+ * the caller, >= quartz_prepared_weights_size bytes, 16-byte aligned).  A
+ * later quartz_linear_ex with opts->w_prepared = prepared and the same `w`
+ * skips that work on every call; the buffer is only valid for that `w`
+ * (its codes, FLAGs, scales and params) and becomes stale if `w` changes. */
+int32_t quartz_prepare_weights(const quartz_encoded_t *w, void *prepared, size_t prepared_bytes, void *stream);
 
 /* quartz_linear with the controls above (opts may be NULL = defaults). */
 int32_t quartz_linear_ex(const quartz_encoded_t *a, const quartz_encoded_t *w,

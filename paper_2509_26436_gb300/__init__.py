@@ -23,7 +23,7 @@ from ._native import (ALGO_SHIFT, ALGO_SIMT, ALGO_TCGEN05, ASYMMETRIC, OUT_BF16,
 
 __all__ = ["Params", "Encoded", "quantize", "encode_weights", "dequantize", "linear",
            "linear_workspace_size", "empty_encoded", "device_status", "selftest_timeout",
-           "kv_append", "attention_decode", "attention_workspace_size",
+           "kv_append", "attention_decode", "attention_workspace_size", "prepare_weights",
            "SYMMETRIC", "ASYMMETRIC", "QuartzError"]
 
 
@@ -155,9 +155,24 @@ def linear_workspace_size(M: int, N_: int, K: int, params: Params = Params()) ->
 _OUT = {"float16": OUT_F16, "bfloat16": OUT_BF16, "float32": OUT_F32}
 
 
+def prepare_weights(w: Encoded, stream=None):
+    """The weights' tensor-core operand and scale side values, prepared once
+    (offline, like the encoding) for linear(..., w_prepared=...)."""
+    torch = _torch()
+    p = w.params.c()
+    n = int(N.load().quartz_prepared_weights_size(w.rows, w.K, C.byref(p)))
+    if n == 0:
+        raise ValueError("invalid weight shape for preparation")
+    buf = torch.empty(n, dtype=torch.uint8, device=w.codes.device)
+    wc = w.c()
+    N.check(N.load().quartz_prepare_weights(C.byref(wc), buf.data_ptr(), n, _stream(stream)),
+            "quartz_prepare_weights")
+    return buf
+
+
 def linear(a: Encoded, w: Encoded, bias=None, out_dtype=None, out=None, workspace=None,
            partials_group: int | None = None, algo: int = ALGO_TCGEN05, stream=None,
-           gemm_events=None):
+           gemm_events=None, w_prepared=None):
     """W4A4 QuaRTZ linear: y = dequant(a) @ dequant(w)^T (+ bias), computed as
     exact integer group partials scaled by the 16-bit group scales.
 
@@ -191,7 +206,8 @@ def linear(a: Encoded, w: Encoded, bias=None, out_dtype=None, out=None, workspac
     opts = N.QuartzLinearOpts(None if part is None else part.data_ptr(),
                               0 if partials_group is None else partials_group, algo,
                               None if gemm_events is None else gemm_events[0].cuda_event,
-                              None if gemm_events is None else gemm_events[1].cuda_event)
+                              None if gemm_events is None else gemm_events[1].cuda_event,
+                              None if w_prepared is None else w_prepared.data_ptr())
     rc = N.load().quartz_linear_ex(
         C.byref(ac), C.byref(wc), None if bias is None else bias.data_ptr(), y.data_ptr(), y_type,
         workspace.data_ptr(), workspace.numel() * workspace.element_size(), C.byref(opts),

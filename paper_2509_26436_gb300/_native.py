@@ -49,7 +49,7 @@ class QuartzEncoded(C.Structure):
 
 class QuartzLinearOpts(C.Structure):
     _fields_ = [("partials", _P), ("partials_group", C.c_int32), ("algo", C.c_int32),
-                ("gemm_event_begin", _P), ("gemm_event_end", _P)]
+                ("gemm_event_begin", _P), ("gemm_event_end", _P), ("w_prepared", _P)]
 
 
 SIGNATURES = {
@@ -69,6 +69,8 @@ SIGNATURES = {
                                      _I32, _P]),
     "quartz_linear_f16": (_I32, [_P, _I64, C.POINTER(QuartzEncoded), _P, _P, _I32,
                                  C.POINTER(QuartzEncoded), _P, _SZ, _P]),
+    "quartz_prepared_weights_size": (_SZ, [_I64, _I64, C.POINTER(QuartzParams)]),
+    "quartz_prepare_weights": (_I32, [C.POINTER(QuartzEncoded), _P, _SZ, _P]),
     "quartz_attention_workspace_size": (_SZ, [_I64, _I64]),
     "quartz_kv_append": (_I32, [_P, _I64, _I64, C.POINTER(QuartzEncoded), _I64, _I64, _P]),
     "quartz_attention_decode": (_I32, [C.POINTER(QuartzEncoded), C.POINTER(QuartzEncoded),

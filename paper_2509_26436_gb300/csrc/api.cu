@@ -197,13 +197,15 @@ int32_t quartz_linear_ex(const quartz_encoded_t *a, const quartz_encoded_t *w,
     const size_t need = linear_workspace_bytes(M, N, K, a->p.mode);
     if (!workspace || workspace_bytes < need) return QUARTZ_ERR_WORKSPACE;
     if (!aligned16(workspace)) return QUARTZ_ERR_ALIGNMENT;
+    if (o.w_prepared && !aligned16(o.w_prepared)) return QUARTZ_ERR_ALIGNMENT;
     int *dev_err = device_error_word();
     if (!dev_err) return QUARTZ_ERR_CUDA;
 
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     LinearWorkspace ws;
     linear_workspace_carve(workspace, M, N, K, a->p.mode, &ws);
-    cudaError_t e = launch_prepare(a, w, ws, s, algo != QUARTZ_ALGO_SHIFT);
+    if (o.w_prepared) prepared_weights_carve(o.w_prepared, N, K, a->p.mode, &ws);
+    cudaError_t e = launch_prepare(a, w, ws, s, algo != QUARTZ_ALGO_SHIFT, o.w_prepared != nullptr);
     if (e != cudaSuccess) return QUARTZ_ERR_CUDA;
     if (o.gemm_event_begin && cudaEventRecord(static_cast<cudaEvent_t>(o.gemm_event_begin), s) != cudaSuccess)
         return QUARTZ_ERR_CUDA;
@@ -217,6 +219,25 @@ int32_t quartz_linear_ex(const quartz_encoded_t *a, const quartz_encoded_t *w,
     if (e == cudaSuccess && o.gemm_event_end)
         e = cudaEventRecord(static_cast<cudaEvent_t>(o.gemm_event_end), s);
     return map_cuda(e);
+}
+
+size_t quartz_prepared_weights_size(int64_t N, int64_t K, const quartz_params_t *p)
+{
+    if (check_shape(N, K, p) != QUARTZ_OK || N <= 0 || N % 8 != 0 || N > (int64_t(1) << 24)) return 0;
+    return prepared_weights_bytes(N, K, p->mode);
+}
+
+int32_t quartz_prepare_weights(const quartz_encoded_t *w, void *prepared, size_t prepared_bytes, void *stream)
+{
+    int32_t rc = check_encoded(w);
+    if (rc) return rc;
+    const int64_t N = w->rows, K = w->K;
+    if (N <= 0 || N % 8 != 0 || N > (int64_t(1) << 24)) return QUARTZ_ERR_INVALID_ARG;
+    if (!prepared || prepared_bytes < prepared_weights_bytes(N, K, w->p.mode)) return QUARTZ_ERR_WORKSPACE;
+    if (!aligned16(prepared)) return QUARTZ_ERR_ALIGNMENT;
+    LinearWorkspace ws{};
+    prepared_weights_carve(prepared, N, K, w->p.mode, &ws);
+    return map_cuda(launch_prepare(nullptr, w, ws, static_cast<cudaStream_t>(stream)));
 }
 
 int32_t quartz_linear(const quartz_encoded_t *a, const quartz_encoded_t *w, const void *bias_f16,

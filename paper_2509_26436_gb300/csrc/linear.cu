@@ -1185,8 +1185,24 @@ void linear_workspace_carve(void *base, int64_t M, int64_t N, int64_t K, int mod
     ws->w_side = reinterpret_cast<float *>(p);
 }
 
+size_t prepared_weights_bytes(int64_t N, int64_t K, int mode)
+{
+    const int nside = mode == QUARTZ_ASYMMETRIC ? 3 : 1;
+    const int64_t G = K / kGroupQ;
+    return align256(static_cast<size_t>(round_up(N, 16)) * K) + align256(static_cast<size_t>(nside) * G * round_up(N, BN) * 4);
+}
+
+void prepared_weights_carve(const void *base, int64_t N, int64_t K, int mode, LinearWorkspace *ws)
+{
+    uint8_t *p = static_cast<uint8_t *>(const_cast<void *>(base));
+    ws->w_op = p;
+    ws->w_side = reinterpret_cast<float *>(p + align256(static_cast<size_t>(round_up(N, 16)) * K));
+    ws->n_pad = round_up(N, BN);
+    ws->nside = mode == QUARTZ_ASYMMETRIC ? 3 : 1;
+}
+
 cudaError_t launch_prepare(const quartz_encoded_t *a, const quartz_encoded_t *w, const LinearWorkspace &ws,
-                           cudaStream_t s, bool expand)
+                           cudaStream_t s, bool expand, bool w_ready)
 {
     const int64_t K = w->K;
     const int64_t upr = K / 16;
@@ -1203,8 +1219,8 @@ cudaError_t launch_prepare(const quartz_encoded_t *a, const quartz_encoded_t *w,
         p.sd_a = {reinterpret_cast<const __half *>(a->scales), a->zeros, a->gsum, ws.a_side, a->rows, ws.m_pad, 1};
     p.sd_w = {reinterpret_cast<const __half *>(w->scales), w->zeros, w->gsum, ws.w_side, w->rows, ws.n_pad, 0};
     const int64_t side_chunks = (p.G + kSideGroupsPerThread - 1) / kSideGroupsPerThread;
-    const int64_t threads[4] = {expand ? p.ex_a.units_pad : 0, expand ? p.ex_w.units_pad : 0,
-                                a ? ws.m_pad * side_chunks : 0, ws.n_pad * side_chunks};
+    const int64_t threads[4] = {expand ? p.ex_a.units_pad : 0, expand && !w_ready ? p.ex_w.units_pad : 0,
+                                a ? ws.m_pad * side_chunks : 0, w_ready ? 0 : ws.n_pad * side_chunks};
     int64_t acc = 0;
     for (int i = 0; i < 4; ++i) {
         acc += (threads[i] + kPrepThreads - 1) / kPrepThreads;

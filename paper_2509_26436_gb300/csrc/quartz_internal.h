@@ -60,8 +60,15 @@ void linear_workspace_carve(void *base, int64_t M, int64_t N, int64_t K, int mod
 // workspace (one launch).  `a` may be NULL: then only the weight operand is
 // prepared (the fused encoder below has written the activation side).  With
 // `expand` false only the scales are transposed (accumulator-shift GEMM).
+// With `w_ready` the weight operand and its side values are already in
+// ws.w_op / ws.w_side (prepared once, quartz_prepare_weights) and only the
+// activation jobs run.
 cudaError_t launch_prepare(const quartz_encoded_t *a, const quartz_encoded_t *w, const LinearWorkspace &ws,
-                           cudaStream_t s, bool expand = true);
+                           cudaStream_t s, bool expand = true, bool w_ready = false);
+// Layout of a prepared weight operand: the expanded operand [round_up(N, 16),
+// K] bytes, then the side values [nside][K/64][round_up(N, 256)] fp32.
+size_t prepared_weights_bytes(int64_t N, int64_t K, int mode);
+void prepared_weights_carve(const void *base, int64_t N, int64_t K, int mode, LinearWorkspace *ws);
 // The paper's accumulator-shift schedule on CUDA cores, from the packed codes;
 // `wide`: 16-bit stage-1 codes (FLAGs up to 12, 64-bit group sums).
 cudaError_t launch_gemm_shift(const LinearWorkspace &ws, const quartz_encoded_t *a, const quartz_encoded_t *w,

@@ -199,6 +199,23 @@ def test_attention_validation(lib):
     assert K(None, 4, 0, C.byref(enc(200)), 50, 0, None) == N.QUARTZ_OK                   # T == 0
 
 
+def test_prepared_weights_validation(lib):
+    p = N.QuartzParams(64, 16, 0)
+    assert lib.quartz_prepared_weights_size(24, 128, C.byref(p)) >= 24 * 128
+    assert lib.quartz_prepared_weights_size(20, 128, C.byref(p)) == 0          # N % 8
+    assert lib.quartz_prepared_weights_size(24, 100, C.byref(p)) == 0          # K % 64
+    P = lib.quartz_prepare_weights
+    w = _enc(24, 128)
+    need = lib.quartz_prepared_weights_size(24, 128, C.byref(p))
+    assert P(C.byref(w), 0x4000, need - 1, None) == N.QUARTZ_ERR_WORKSPACE
+    assert P(C.byref(w), None, need, None) == N.QUARTZ_ERR_WORKSPACE
+    assert P(C.byref(w), 0x4008, need, None) == N.QUARTZ_ERR_ALIGNMENT
+    assert P(C.byref(_enc(20, 128)), 0x4000, need, None) == N.QUARTZ_ERR_INVALID_ARG
+    o = N.QuartzLinearOpts(None, 0, 0, None, None, 0x5008)                   # misaligned prepared weights
+    assert lib.quartz_linear_ex(C.byref(_enc(16, 128)), C.byref(w), None, 0x2000, 0, 0x3000, 1 << 30,
+                                C.byref(o), None) == N.QUARTZ_ERR_ALIGNMENT
+
+
 def test_linear_f16_validation(lib):
     """Host checks of the fused activation path: nothing is launched on error."""
     L = lib.quartz_linear_f16

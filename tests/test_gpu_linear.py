@@ -368,3 +368,47 @@ def test_linear_f16_packed_flag_output(Q):
     a = Q.quantize(x, flag_bits=4)
     assert torch.equal(a_out.flags, a.flags) and torch.equal(a_out.codes, a.codes)
     assert torch.equal(y, Q.linear(a, w))
+
+
+@pytest.mark.parametrize("algo", list(ALGOS))
+@pytest.mark.parametrize("mode", [O.SYMMETRIC, O.ASYMMETRIC])
+def test_prepared_weights_identical(Q, algo, mode):
+    """Weights prepared once give the same bits as preparing them per call."""
+    xa = inputs.laplace_activations(200, 640, seed=8100)
+    xw = inputs.gaussian_weights(264, 640, seed=8101)
+    bias = np.random.default_rng(3).normal(0, 0.1, 264).astype(np.float16)
+    a = Q.quantize(torch.from_numpy(xa).cuda(), group_s=16, mode=mode)
+    w = Q.encode_weights(torch.from_numpy(xw).cuda(), group_s=16, mode=mode)
+    b = torch.from_numpy(bias).cuda()
+    prep = Q.prepare_weights(w)
+    y0 = Q.linear(a, w, b, algo=ALGOS[algo])
+    y1 = Q.linear(a, w, b, algo=ALGOS[algo], w_prepared=prep)
+    y2 = Q.linear(a, w, b, algo=ALGOS[algo], w_prepared=prep)   # reusable
+    assert Q.device_status() == 0
+    assert torch.equal(y0, y1) and torch.equal(y0, y2)
+
+
+@pytest.mark.parametrize("kind", ["per_row", "wide", "packed"])
+def test_prepared_weights_other_formats(Q, kind):
+    xa = inputs.laplace_activations(130, 1152, seed=8200)
+    xw = inputs.gaussian_weights(136, 1152, seed=8201)
+    kw = {"per_row": dict(group_q=1152), "wide": dict(group_s=8, code_bits=16),
+          "packed": dict(flag_bits=4)}[kind]
+    gs = kw.pop("group_s", 16)
+    a = Q.quantize(torch.from_numpy(xa).cuda(), group_s=gs, **kw)
+    w = Q.encode_weights(torch.from_numpy(xw).cuda(), group_s=gs, **kw)
+    prep = Q.prepare_weights(w)
+    y0 = Q.linear(a, w)
+    y1 = Q.linear(a, w, w_prepared=prep)
+    assert Q.device_status() == 0
+    assert torch.equal(y0, y1)
+
+
+def test_prepared_weights_flux_fc1(Q):
+    layer = inputs.CONFIG4[2]
+    a = Q.quantize(torch.from_numpy(layer.activations()).cuda(), group_s=16)
+    w = Q.encode_weights(torch.from_numpy(layer.weights()).cuda(), group_s=16)
+    y0 = Q.linear(a, w)
+    y1 = Q.linear(a, w, w_prepared=Q.prepare_weights(w))
+    assert Q.device_status() == 0
+    assert torch.equal(y0, y1)
