@@ -239,6 +239,13 @@ int32_t quartz_linear_f16(const void *x_f16, int64_t M, const quartz_encoded_t *
                           void *y, int32_t y_type, const quartz_encoded_t *a_out, void *workspace,
                           size_t workspace_bytes, void *stream);
 
+/* quartz_linear_f16 with the weights prepared once by quartz_prepare_weights
+ * (`w_prepared`, from the same `w`; NULL = quartz_linear_f16): the call is
+ * then one encoder launch and the GEMM. */
+int32_t quartz_linear_f16_ex(const void *x_f16, int64_t M, const quartz_encoded_t *w, const void *w_prepared,
+                             const void *bias_f16, void *y, int32_t y_type, const quartz_encoded_t *a_out,
+                             void *workspace, size_t workspace_bytes, void *stream);
+
 /* Scratch-free variant of quartz_linear, for callers that cannot allocate
  * device memory (for example a plugin inside a host framework that owns all
  * device memory through its own pool and forbids side allocations, or code on

@@ -217,10 +217,11 @@ def linear(a: Encoded, w: Encoded, bias=None, out_dtype=None, out=None, workspac
 
 
 def linear_f16(x, w: Encoded, bias=None, out_dtype=None, out=None, workspace=None,
-               a_out: Encoded | None = None, stream=None):
+               a_out: Encoded | None = None, stream=None, w_prepared=None):
     """Fused activation path: y = linear(quantize(x), w) from fp16 x [M, K]
     in one pass over x (the activations are encoded straight into the GEMM
-    operand; symmetric mode).  `a_out` optionally receives the encoding."""
+    operand; symmetric mode).  `a_out` optionally receives the encoding;
+    `w_prepared` = prepare_weights(w) skips the per-call weight preparation."""
     torch = _torch()
     _check_f16(x, "x")
     out_dtype = out_dtype or torch.float16
@@ -235,11 +236,12 @@ def linear_f16(x, w: Encoded, bias=None, out_dtype=None, out=None, workspace=Non
         raise ValueError("bias must be a float16 CUDA tensor of N elements")
     wc = w.c()
     ac = a_out.c() if a_out is not None else None
-    rc = N.load().quartz_linear_f16(
-        x.data_ptr(), M, C.byref(wc), None if bias is None else bias.data_ptr(), y.data_ptr(), y_type,
+    rc = N.load().quartz_linear_f16_ex(
+        x.data_ptr(), M, C.byref(wc), None if w_prepared is None else w_prepared.data_ptr(),
+        None if bias is None else bias.data_ptr(), y.data_ptr(), y_type,
         None if ac is None else C.byref(ac), workspace.data_ptr(),
         workspace.numel() * workspace.element_size(), _stream(stream))
-    N.check(rc, "quartz_linear_f16")
+    N.check(rc, "quartz_linear_f16_ex")
     return y
 
 

@@ -69,6 +69,8 @@ SIGNATURES = {
                                      _I32, _P]),
     "quartz_linear_f16": (_I32, [_P, _I64, C.POINTER(QuartzEncoded), _P, _P, _I32,
                                  C.POINTER(QuartzEncoded), _P, _SZ, _P]),
+    "quartz_linear_f16_ex": (_I32, [_P, _I64, C.POINTER(QuartzEncoded), _P, _P, _P, _I32,
+                                    C.POINTER(QuartzEncoded), _P, _SZ, _P]),
     "quartz_prepared_weights_size": (_SZ, [_I64, _I64, C.POINTER(QuartzParams)]),
     "quartz_prepare_weights": (_I32, [C.POINTER(QuartzEncoded), _P, _SZ, _P]),
     "quartz_attention_workspace_size": (_SZ, [_I64, _I64]),

@@ -251,6 +251,14 @@ int32_t quartz_linear_f16(const void *x_f16, int64_t M, const quartz_encoded_t *
                           void *y, int32_t y_type, const quartz_encoded_t *a_out, void *workspace,
                           size_t workspace_bytes, void *stream)
 {
+    return quartz_linear_f16_ex(x_f16, M, w, nullptr, bias_f16, y, y_type, a_out, workspace, workspace_bytes,
+                                stream);
+}
+
+int32_t quartz_linear_f16_ex(const void *x_f16, int64_t M, const quartz_encoded_t *w, const void *w_prepared,
+                             const void *bias_f16, void *y, int32_t y_type, const quartz_encoded_t *a_out,
+                             void *workspace, size_t workspace_bytes, void *stream)
+{
     int32_t rc = check_encoded(w);
     if (rc) return rc;
     if (w->p.mode != QUARTZ_SYMMETRIC || w->p.group_q != 64 || wide_codes(w->p)) return QUARTZ_ERR_UNSUPPORTED;
@@ -270,7 +278,9 @@ int32_t quartz_linear_f16(const void *x_f16, int64_t M, const quartz_encoded_t *
     if (M * N >= (int64_t(1) << 40)) return QUARTZ_ERR_UNSUPPORTED;
     if (M == 0) return QUARTZ_OK;
     if (!x_f16 || !y) return QUARTZ_ERR_INVALID_ARG;
-    if (!aligned16(x_f16) || !aligned16(y) || (bias_f16 && !aligned16(bias_f16))) return QUARTZ_ERR_ALIGNMENT;
+    if (!aligned16(x_f16) || !aligned16(y) || (bias_f16 && !aligned16(bias_f16)) ||
+        (w_prepared && !aligned16(w_prepared)))
+        return QUARTZ_ERR_ALIGNMENT;
     const size_t need = linear_workspace_bytes(M, N, K, w->p.mode);
     if (!workspace || workspace_bytes < need) return QUARTZ_ERR_WORKSPACE;
     if (!aligned16(workspace)) return QUARTZ_ERR_ALIGNMENT;
@@ -280,8 +290,9 @@ int32_t quartz_linear_f16(const void *x_f16, int64_t M, const quartz_encoded_t *
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     LinearWorkspace ws;
     linear_workspace_carve(workspace, M, N, K, w->p.mode, &ws);
+    if (w_prepared) prepared_weights_carve(w_prepared, N, K, w->p.mode, &ws);
     cudaError_t e = launch_encode_operand(x_f16, M, K, &w->p, ws, a_out, s);
-    if (e == cudaSuccess) e = launch_prepare(nullptr, w, ws, s);
+    if (e == cudaSuccess && !w_prepared) e = launch_prepare(nullptr, w, ws, s);
     if (e == cudaSuccess)
         e = launch_gemm_tcgen05(ws, M, N, K, w->p.mode, bias_f16, y, y_type, nullptr, 0, dev_err, s);
     return map_cuda(e);

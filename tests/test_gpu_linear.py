@@ -412,3 +412,15 @@ def test_prepared_weights_flux_fc1(Q):
     y1 = Q.linear(a, w, w_prepared=Q.prepare_weights(w))
     assert Q.device_status() == 0
     assert torch.equal(y0, y1)
+
+
+def test_linear_f16_prepared_weights_identical(Q):
+    xa = inputs.laplace_activations(300, 1216, seed=8300)
+    xw = inputs.gaussian_weights(520, 1216, seed=8301)
+    x = torch.from_numpy(xa).cuda()
+    w = Q.encode_weights(torch.from_numpy(xw).cuda(), group_s=16)
+    y0 = Q.linear_f16(x, w)
+    y1 = Q.linear_f16(x, w, w_prepared=Q.prepare_weights(w))
+    y2 = Q.linear(Q.quantize(x, group_s=16), w)
+    assert Q.device_status() == 0
+    assert torch.equal(y0, y1) and torch.equal(y0, y2)
