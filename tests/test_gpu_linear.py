@@ -381,11 +381,11 @@ def test_prepared_weights_identical(Q, algo, mode):
     w = Q.encode_weights(torch.from_numpy(xw).cuda(), group_s=16, mode=mode)
     b = torch.from_numpy(bias).cuda()
     prep = Q.prepare_weights(w)
-    y0 = Q.linear(a, w, b, algo=ALGOS[algo])
-    y1 = Q.linear(a, w, b, algo=ALGOS[algo], w_prepared=prep)
+    y0, p0 = Q.linear(a, w, b, algo=ALGOS[algo], partials_group=3)
+    y1, p1 = Q.linear(a, w, b, algo=ALGOS[algo], w_prepared=prep, partials_group=3)
     y2 = Q.linear(a, w, b, algo=ALGOS[algo], w_prepared=prep)   # reusable
     assert Q.device_status() == 0
-    assert torch.equal(y0, y1) and torch.equal(y0, y2)
+    assert torch.equal(y0, y1) and torch.equal(y0, y2) and torch.equal(p0, p1)
 
 
 @pytest.mark.parametrize("kind", ["per_row", "wide", "packed"])
@@ -420,7 +420,11 @@ def test_linear_f16_prepared_weights_identical(Q):
     x = torch.from_numpy(xa).cuda()
     w = Q.encode_weights(torch.from_numpy(xw).cuda(), group_s=16)
     y0 = Q.linear_f16(x, w)
-    y1 = Q.linear_f16(x, w, w_prepared=Q.prepare_weights(w))
-    y2 = Q.linear(Q.quantize(x, group_s=16), w)
+    a_out = Q.empty_encoded(300, 1216, Q.Params(64, 16), "cuda")
+    y1 = Q.linear_f16(x, w, w_prepared=Q.prepare_weights(w), a_out=a_out)
+    a = Q.quantize(x, group_s=16)
+    y2 = Q.linear(a, w)
     assert Q.device_status() == 0
     assert torch.equal(y0, y1) and torch.equal(y0, y2)
+    assert torch.equal(a_out.codes, a.codes) and torch.equal(a_out.flags, a.flags)
+    assert torch.equal(a_out.scales, a.scales)
