@@ -82,8 +82,8 @@ typedef struct {
                         * 16 requires SYMMETRIC mode and group_q == 64. */
 } quartz_params_t;
 
-/* One encoded tensor of `rows` rows and `K` columns (Section 4.4: "packed
- * s4" codes plus "a single flag byte per subgroup").  Buffers are device
+/* One encoded tensor of `rows` rows and `K` columns (Section 4.4's format:
+ * signed 4-bit codes two per byte, one FLAG byte per subgroup).  Buffers are device
  * memory owned by the caller; sizes in elements:
  *   codes  uint8 [rows, K/2]        two's-complement 4-bit codes in [-7, 7],
  *                                   element 2j in the low nibble of byte j
@@ -122,8 +122,8 @@ int32_t quartz_version(void);
  * QUARTZ_ERR_INVALID_ARG. */
 int32_t quartz_encoded_sizes(int64_t rows, int64_t K, const quartz_params_t *p, size_t out[5]);
 
-/* Two-stage QuaRTZ encoder, on the fly for activations (Appendix C: "4-bit
- * compression is applied on-the-fly"): Eq. 1 per group of p->group_q along
+/* Two-stage QuaRTZ encoder, run on activations as they are produced
+ * (Appendix C compresses them to 4 bits at run time): Eq. 1 per group of p->group_q along
  * K, then Eq. 2 per subgroup of p->group_s, then nibble packing.
  *   x_f16  fp16 [out->rows, out->K] device, 16-byte aligned
  *   out    describes the destination: rows, K, p and the buffers above
@@ -222,8 +222,8 @@ int32_t quartz_linear_ex(const quartz_encoded_t *a, const quartz_encoded_t *w,
                          size_t workspace_bytes, const quartz_linear_opts_t *opts, void *stream);
 
 /* Fused activation path: the W4A4 linear layer straight from fp16
- * activations, encoding them on the fly (the "on-the-fly activation
- * compression" of Appendix C).  One pass over x does Eq. 1 and Eq. 2 and
+ * activations, encoding them at run time (Appendix C's run-time activation
+ * compression).  One pass over x does Eq. 1 and Eq. 2 and
  * writes the tensor-core operand directly, instead of writing the encoded
  * activations and reading them back; results are bit-identical to
  * quartz_quantize followed by quartz_linear with the same parameters.

@@ -240,7 +240,8 @@ int oracle_lzs_encode(const int8_t *q, int64_t n, int gs, uint8_t *flags, int8_t
 }
 
 /* 4-bit values c [n] + flags -> decoded integers v = sgn * (|c| << FLAG):
- * "each group has been shifted equally", so the shift is undone by FLAG. */
+ * every value of a subgroup was shifted by the same FLAG, so shifting back by
+ * FLAG restores its magnitude (minus the truncated low bits). */
 int oracle_lzs_decode(const int8_t *c, const uint8_t *flags, int64_t n, int gs, int16_t *v)
 {
     if (gs <= 0 || n % gs != 0) return ORACLE_ERR_ARG;
@@ -328,8 +329,8 @@ int oracle_encode_static(const uint16_t *x, int64_t rows, int64_t K, uint16_t s1
 }
 
 /* ---------------------------------------------------------------------------
- * LLM variant (Section 5, "Potential Applications to LLMs": 16-bit
- * activations compressed directly to 4 bits, G_s = 8).  Stage 1 quantizes
+ * LLM variant (Section 5: activations quantized to 16-bit integers and
+ * then LZS-coded to 4 bits, subgroups of G_s = 8).  Stage 1 quantizes
  * each group to 16-bit integers, symmetric: s = fp16(max|x| / 32767),
  * q = clamp(round(x * r), -32767, 32767) with r = RN(1/s) (R3); a zero scale
  * gives all-zero codes (R5).  Stage 2 is Eq. 2 unchanged on the wider codes:
