@@ -61,7 +61,8 @@ typedef enum { QUARTZ_OUT_F16 = 0, QUARTZ_OUT_BF16 = 1, QUARTZ_OUT_F32 = 2 } qua
  * on-device path; SHIFT is the paper's own schedule (Section 4.4): integer
  * dot products of the packed 4-bit codes per subgroup, each shifted by the
  * two operands' FLAGs, with no decoded operand (CUDA cores, dp4a).  All three
- * give the same exact group partials P_g. */
+ * give the same exact group partials P_g (8-bit codes; see quartz_linear for
+ * 16-bit codes). */
 typedef enum { QUARTZ_ALGO_TCGEN05 = 0, QUARTZ_ALGO_SIMT = 1, QUARTZ_ALGO_SHIFT = 2 } quartz_algo_t;
 
 typedef struct {
@@ -71,8 +72,9 @@ typedef struct {
     int32_t group_s; /* LZS subgroup G_s along K: 8, 16, 32 or 64 (Section 3, Table 1) */
     int32_t mode;    /* quartz_mode_t */
     int32_t flag_bits; /* FLAG storage: 0 or 8 = one byte per subgroup (Section
-                        * 4.4); 4 = two FLAGs per byte (values 0..4 fit in 4
-                        * bits), 4 + 4/G_s + 16/group_q bits per element */
+                        * 4.4); 4 = two FLAGs per byte (values 0..4, or 0..12
+                        * with 16-bit codes, fit in 4 bits), 4 + 4/G_s +
+                        * 16/group_q bits per element */
     int32_t code_bits; /* width of the stage-1 codes: 0 or 8 = Eq. 1's 8-bit
                         * codes; 16 = the LLM variant of Section 5 (16-bit
                         * activations compressed straight to 4 bits; the

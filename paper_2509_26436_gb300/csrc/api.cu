@@ -96,7 +96,7 @@ const char *quartz_status_string(int32_t status)
     }
 }
 
-int32_t quartz_version(void) { return (1 << 16) | 4; }
+int32_t quartz_version(void) { return (1 << 16) | 5; }
 
 int32_t quartz_encoded_sizes(int64_t rows, int64_t K, const quartz_params_t *p, size_t out[5])
 {
