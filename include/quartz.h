@@ -150,15 +150,27 @@ int32_t quartz_quantize_static(const void *x_f16, uint16_t scale_f16, const quar
 int32_t quartz_encode_weights(const void *w_f16, const quartz_encoded_t *out, void *stream);
 
 /* Dequantise an encoded tensor: x_hat = s * (v - z) with the decoded LZS
- * value v = sgn(c)(|c| << FLAG) (Section 3: "each group has been shifted
- * equally"), computed in binary32 and rounded once to fp16.
+ * value v = sgn(c)(|c| << FLAG) (Section 3: one FLAG shift for every value
+ * of a subgroup), computed in binary32 and rounded once to fp16.
  *   x_hat_f16  fp16 [e->rows, e->K] device output. */
 int32_t quartz_dequantize(const quartz_encoded_t *e, void *x_hat_f16, void *stream);
 
 /* Workspace bytes quartz_linear needs for an [M, K] x [N, K]^T product
- * (the operands expanded to the tensor-core input format plus transposed
- * group scales).  Returns 0 for invalid arguments. */
+ * (the operands expanded to the tensor-core input format, transposed group
+ * scales and, where the symmetric tcgen05 GEMM splits its last wave of
+ * tiles along K, the fp32 partial tiles of that wave).  The last part
+ * depends on the current device's SM count: query it on the device that
+ * will run the call.  Returns 0 for invalid arguments. */
 size_t quartz_linear_workspace_size(int64_t M, int64_t N, int64_t K, const quartz_params_t *p);
+
+/* Kernels one quartz_linear_ex call with these sizes, algorithm and
+ * partials setting launches on the current device: operand preparation,
+ * the GEMM and, when the symmetric group-64 tcgen05 GEMM (no partials)
+ * splits its last wave of tiles along K, the kernel that adds the parts in
+ * a fixed order and writes those tiles.  Returns 0 for invalid arguments
+ * or M = 0 (no launch). */
+int32_t quartz_linear_launch_count(int64_t M, int64_t N, int64_t K, const quartz_params_t *p, int32_t algo,
+                                   int32_t with_partials);
 
 /* W4A4 QuaRTZ linear (Section 4.4 with Appendix C's group scales):
  *   y[m, n] = sum_g s_a[m,g] s_w[n,g] (P_g[m,n] - z_w[n,g] A_g[m] - z_a[m,g] W_g[n]

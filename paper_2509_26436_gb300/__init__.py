@@ -152,6 +152,14 @@ def linear_workspace_size(M: int, N_: int, K: int, params: Params = Params()) ->
     return int(N.load().quartz_linear_workspace_size(M, N_, K, C.byref(p)))
 
 
+def linear_launch_count(M: int, N_: int, K: int, params: Params = Params(), algo: int = ALGO_TCGEN05,
+                        partials: bool = False) -> int:
+    """Kernels one linear() call with these sizes launches on the current
+    device (0: invalid arguments or M = 0)."""
+    p = params.c()
+    return int(N.load().quartz_linear_launch_count(M, N_, K, C.byref(p), algo, 1 if partials else 0))
+
+
 _OUT = {"float16": OUT_F16, "bfloat16": OUT_BF16, "float32": OUT_F32}
 
 

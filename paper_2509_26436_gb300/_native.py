@@ -61,6 +61,7 @@ SIGNATURES = {
     "quartz_encode_weights": (_I32, [_P, C.POINTER(QuartzEncoded), _P]),
     "quartz_dequantize": (_I32, [C.POINTER(QuartzEncoded), _P, _P]),
     "quartz_linear_workspace_size": (_SZ, [_I64, _I64, _I64, C.POINTER(QuartzParams)]),
+    "quartz_linear_launch_count": (_I32, [_I64, _I64, _I64, C.POINTER(QuartzParams), _I32, _I32]),
     "quartz_linear": (_I32, [C.POINTER(QuartzEncoded), C.POINTER(QuartzEncoded), _P, _P, _I32,
                              _P, _SZ, _P]),
     "quartz_linear_ex": (_I32, [C.POINTER(QuartzEncoded), C.POINTER(QuartzEncoded), _P, _P, _I32,

@@ -96,7 +96,7 @@ const char *quartz_status_string(int32_t status)
     }
 }
 
-int32_t quartz_version(void) { return (1 << 16) | 5; }
+int32_t quartz_version(void) { return (1 << 16) | 6; }
 
 int32_t quartz_encoded_sizes(int64_t rows, int64_t K, const quartz_params_t *p, size_t out[5])
 {
@@ -156,6 +156,17 @@ size_t quartz_linear_workspace_size(int64_t M, int64_t N, int64_t K, const quart
 {
     if (check_shape(M, K, p) != QUARTZ_OK || N <= 0 || N % 8 != 0) return 0;
     return linear_workspace_bytes(M, N, K, p->mode);
+}
+
+int32_t quartz_linear_launch_count(int64_t M, int64_t N, int64_t K, const quartz_params_t *p, int32_t algo,
+                                   int32_t with_partials)
+{
+    if (check_shape(M, K, p) != QUARTZ_OK || N <= 0 || N % 8 != 0) return 0;
+    if (algo != QUARTZ_ALGO_TCGEN05 && algo != QUARTZ_ALGO_SIMT && algo != QUARTZ_ALGO_SHIFT) return 0;
+    if (M == 0) return 0;
+    const bool split = algo == QUARTZ_ALGO_TCGEN05 && p->mode == QUARTZ_SYMMETRIC && !with_partials &&
+                       p->group_q == 64 && linear_tail_parts(M, N, K, p->mode) > 1;
+    return split ? 3 : 2;
 }
 
 int32_t quartz_linear_ex(const quartz_encoded_t *a, const quartz_encoded_t *w,

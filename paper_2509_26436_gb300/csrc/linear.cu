@@ -223,6 +223,13 @@ struct GemmArgs {
     int *dev_err;
     int per_row;          // scales per row (group_q = K) rather than per 64-group
     int wide;             // E5M2 operands (16-bit stage-1 codes) instead of E4M3
+    // Split last wave: the first full_tiles tiles go round robin over the CTAs
+    // (the same count each); each of the remaining tail_tiles is cut along K
+    // into `split` group ranges taken by CTAs 0 .. tail_tiles * split - 1,
+    // which leave fp32 partial tiles in tail_part; tail_combine_kernel adds
+    // them in part order and writes the outputs.
+    int full_tiles, tail_tiles, split;
+    float *tail_part;     // [tail_tiles][split][16][kEpiWarps * 32] float4 (fp32 pairs)
 };
 
 // Shared memory: the operand stages, then a ring of side-value slots (one
@@ -256,6 +263,45 @@ __device__ __forceinline__ void tile_coords(int tile, const GemmArgs &a, int &mt
     nt = r / gm;
 }
 
+// This CTA's work: whole tiles, then (split last wave) one part of a tail tile.
+struct WorkItem {
+    int tile, g0, g1;  // tile index and group range [g0, g1)
+    int part, tail;    // part of tail tile `tail` (part = -1: a whole tile)
+};
+
+__device__ __forceinline__ int work_items(const GemmArgs &a)
+{
+    const int c = blockIdx.x, P = gridDim.x;
+    if (a.split <= 1) return (a.num_tiles - c + P - 1) / P;
+    return a.full_tiles / P + (c < a.tail_tiles * a.split ? 1 : 0);
+}
+
+__device__ __forceinline__ WorkItem work_item(const GemmArgs &a, int k)
+{
+    WorkItem w;
+    const int c = blockIdx.x, P = gridDim.x;
+    if (a.split <= 1 || k < a.full_tiles / P) {
+        w.tile = c + k * P;
+        w.g0 = 0;
+        w.g1 = a.G;
+        w.part = -1;
+        w.tail = 0;
+    } else {
+        w.tail = c / a.split;
+        w.part = c - w.tail * a.split;
+        w.tile = a.full_tiles + w.tail;
+        w.g0 = w.part * a.G / a.split;
+        w.g1 = (w.part + 1) * a.G / a.split;
+    }
+    return w;
+}
+
+// (a.x, a.y) += (b.x, b.y) on a packed fp32 pair.
+__device__ __forceinline__ void add2_rn(uint64_t &a, uint64_t b)
+{
+    asm("add.rn.f32x2 %0, %0, %1;" : "+l"(a) : "l"(b));
+}
+
 template <int OUT>
 __device__ __forceinline__ void store_quad(void *y, int64_t off, float4 v)
 {
@@ -270,6 +316,52 @@ __device__ __forceinline__ void store_quad(void *y, int64_t off, float4 v)
     } else {
         *reinterpret_cast<float4 *>(static_cast<float *>(y) + off) = v;
     }
+}
+
+// v + bias[n .. n + 3] in fp32 (no bias: v).
+__device__ __forceinline__ float4 add_bias4(const GemmArgs &args, int64_t n, float4 v)
+{
+    if (args.bias) {
+        const uint2 braw = __ldg(reinterpret_cast<const uint2 *>(args.bias + n));
+        const float2 b0 = __half22float2(*reinterpret_cast<const __half2 *>(&braw.x));
+        const float2 b1 = __half22float2(*reinterpret_cast<const __half2 *>(&braw.y));
+        v.x = __fadd_rn(v.x, b0.x);
+        v.y = __fadd_rn(v.y, b0.y);
+        v.z = __fadd_rn(v.z, b1.x);
+        v.w = __fadd_rn(v.w, b1.y);
+    }
+    return v;
+}
+
+// Output of one 128 x 256 tile from the symmetric epilogue's registers:
+// acc[c][4h + i] holds output column 16c + tq + i of this warp's slice, rows
+// trow + 16h (low half) and trow + 16h + 8 (high half) of its quarter; the
+// bias is added in fp32, then one rounding to the output type.
+template <int OUT>
+__device__ __forceinline__ void store_tile_sym(const GemmArgs &args, int tile, int quarter, int slot, int trow,
+                                               int tq, const uint64_t (&acc)[4][8])
+{
+    int mt, nt;
+    tile_coords(tile, args, mt, nt);
+#pragma unroll
+    for (int h = 0; h < 2; ++h)
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+            const int64_t m = static_cast<int64_t>(mt) * BM + quarter * 32 + 16 * h + 8 * e + trow;
+            if (m >= args.M) continue;
+#pragma unroll
+            for (int chunk = 0; chunk < 4; ++chunk) {
+                const int64_t n = static_cast<int64_t>(nt) * BN + slot * kColsPerWarp + 16 * chunk + tq;
+                if (n >= args.N) continue;
+                float vv[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const uint64_t q = acc[chunk][4 * h + i];
+                    vv[i] = __uint_as_float(static_cast<uint32_t>(e ? (q >> 32) : q));
+                }
+                store_quad<OUT>(args.y, m * args.N + n, add_bias4(args, n, make_float4(vv[0], vv[1], vv[2], vv[3])));
+            }
+        }
 }
 
 // Half of one 16-column chunk: one 16x128b.x4 TMEM load (16 lanes), then
@@ -428,10 +520,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) {
             int it = 0;  // groups whose operand copies were issued
             bool ok = true;
-            for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
+            const int n_items = work_items(args);
+            for (int k = 0; k < n_items && ok; ++k) {
+                const WorkItem wi = work_item(args, k);
                 int mt, nt;
-                tile_coords(tile, args, mt, nt);
-                for (int g = 0; g < G; ++g, ++it) {
+                tile_coords(wi.tile, args, mt, nt);
+                for (int g = wi.g0; g < wi.g1; ++g, ++it) {
                     const int s = it % kStages;
                     if (it >= kStages &&
                         !mbar_wait_bounded(empty_bar(s), ((it / kStages) - 1) & 1, abort_flag,
@@ -466,10 +560,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int64_t w_plane = args.n_pad * G;
             int it = 0;  // groups whose side-value copies were issued
             bool ok = true;
-            for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
+            const int n_items = work_items(args);
+            for (int k = 0; k < n_items && ok; ++k) {
+                const WorkItem wi = work_item(args, k);
                 int mt, nt;
-                tile_coords(tile, args, mt, nt);
-                for (int g = 0; g < G; ++g, ++it) {
+                tile_coords(wi.tile, args, mt, nt);
+                for (int g = wi.g0; g < wi.g1; ++g, ++it) {
                     const int ss = it % S;
                     if (it >= S && !mbar_wait_bounded(side_empty_bar(ss), ((it / S) - 1) & 1, abort_flag,
                                                       args.dev_err, kWaitLimitNs)) {
@@ -506,8 +602,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             bool ok = true;
             constexpr int CH = PERROW ? kPerRowChunk : 1;  // stages per TMEM accumulator
             int ic = 0;                                    // accumulators handed to the epilogue
-            for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
-                for (int g = 0; g < G; ++g, ++it) {
+            const int n_items = work_items(args);
+            for (int k = 0; k < n_items && ok; ++k) {
+                const WorkItem wi = work_item(args, k);
+                for (int g = wi.g0; g < wi.g1; ++g, ++it) {
                     const int s = it % kStages;
                     const int b = ic & 1;
                     const bool first = (g % CH) == 0;
@@ -647,12 +745,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint64_t acc64[4][8];
             int it = 0;
             bool ok = true;
-            for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
+            const int n_items = work_items(args);
+            for (int k = 0; k < n_items && ok; ++k) {
+                const WorkItem wi = work_item(args, k);
 #pragma unroll
                 for (int c = 0; c < 4; ++c)
 #pragma unroll
                     for (int j = 0; j < 8; ++j) acc64[c][j] = 0ull;
-                for (int g = 0; g < G; ++g, ++it) {
+                for (int g = wi.g0; g < wi.g1; ++g, ++it) {
                     const int b = it & 1;
                     const int ss = it % S;
                     if (!mbar_wait_bounded(side_full_bar(ss), (it / S) & 1, abort_flag, args.dev_err,
@@ -687,38 +787,23 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 }
                 if (!ok) break;
-                int mt, nt;
-                tile_coords(tile, args, mt, nt);
+                if (wi.part >= 0) {
+                    // split last wave: leave this part's fp32 partial tile for
+                    // tail_combine_kernel: slot tail * split + part holds 16
+                    // planes of one uint4 per epilogue thread (coalesced)
+                    uint4 *dst = reinterpret_cast<uint4 *>(args.tail_part) +
+                                 ((wi.tail * args.split + wi.part) * 16 * (kEpiWarps * 32) + warp * 32 + lane);
 #pragma unroll
-                for (int h = 0; h < 2; ++h)
+                    for (int c = 0; c < 4; ++c)
 #pragma unroll
-                    for (int e = 0; e < 2; ++e) {
-                        const int64_t m = static_cast<int64_t>(mt) * BM + quarter * 32 + 16 * h + 8 * e + trow;
-                        if (m >= args.M) continue;
-#pragma unroll
-                        for (int chunk = 0; chunk < 4; ++chunk) {
-                            const int64_t n = static_cast<int64_t>(nt) * BN + slot * kColsPerWarp + 16 * chunk + tq;
-                            if (n >= args.N) continue;
-                            float4 v;
-                            float vv[4];
-#pragma unroll
-                            for (int i = 0; i < 4; ++i) {
-                                const uint64_t q = acc64[chunk][4 * h + i];
-                                vv[i] = __uint_as_float(static_cast<uint32_t>(e ? (q >> 32) : q));
-                            }
-                            v = make_float4(vv[0], vv[1], vv[2], vv[3]);
-                            if (args.bias) {
-                                const uint2 braw = __ldg(reinterpret_cast<const uint2 *>(args.bias + n));
-                                const float2 b0 = __half22float2(*reinterpret_cast<const __half2 *>(&braw.x));
-                                const float2 b1 = __half22float2(*reinterpret_cast<const __half2 *>(&braw.y));
-                                v.x = __fadd_rn(v.x, b0.x);
-                                v.y = __fadd_rn(v.y, b0.y);
-                                v.z = __fadd_rn(v.z, b1.x);
-                                v.w = __fadd_rn(v.w, b1.y);
-                            }
-                            store_quad<OUT>(args.y, m * args.N + n, v);
-                        }
-                    }
+                        for (int j = 0; j < 4; ++j)
+                            dst[(4 * c + j) * (kEpiWarps * 32)] = make_uint4(static_cast<uint32_t>(acc64[c][2 * j]),
+                                                        static_cast<uint32_t>(acc64[c][2 * j] >> 32),
+                                                        static_cast<uint32_t>(acc64[c][2 * j + 1]),
+                                                        static_cast<uint32_t>(acc64[c][2 * j + 1] >> 32));
+                    continue;
+                }
+                store_tile_sym<OUT>(args, wi.tile, quarter, slot, trow, tq, acc64);
             }
         } else {
             float2 acc[2][16];
@@ -847,6 +932,53 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after();
         tmem_dealloc(tmem_base, kTmemCols);
     }
+}
+
+// Split last wave (see GemmArgs): adds each tail tile's `split` fp32
+// partial tiles in part order, then stores the sum as the epilogue would
+// have.  Grid: (tail tile, 16-column chunk c of every warp's slice); block:
+// one thread per epilogue thread, which owns the chunk's 8 column pairs.
+template <int OUT>
+__global__ void __launch_bounds__(kEpiWarps * 32) tail_combine_kernel(const __grid_constant__ GemmArgs args)
+{
+    constexpr int T = kEpiWarps * 32;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int tail = blockIdx.x >> 2, c = blockIdx.x & 3;
+    const uint4 *src = reinterpret_cast<const uint4 *>(args.tail_part) +
+                       static_cast<int64_t>(tail) * args.split * 16 * T + 4 * c * T + threadIdx.x;
+    uint64_t acc[8];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        const uint4 v = __ldcg(src + j * T);
+        acc[2 * j] = (static_cast<uint64_t>(v.y) << 32) | v.x;
+        acc[2 * j + 1] = (static_cast<uint64_t>(v.w) << 32) | v.z;
+    }
+    for (int p = 1; p < args.split; ++p) {
+        const uint4 *sp = src + static_cast<int64_t>(p) * 16 * T;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const uint4 v = __ldcg(sp + j * T);
+            add2_rn(acc[2 * j], (static_cast<uint64_t>(v.y) << 32) | v.x);
+            add2_rn(acc[2 * j + 1], (static_cast<uint64_t>(v.w) << 32) | v.z);
+        }
+    }
+    int mt, nt;
+    tile_coords(args.full_tiles + tail, args, mt, nt);
+    const int quarter = warp & 3, slot = warp >> 2, trow = lane >> 2, tq = 4 * (lane & 3);
+    const int64_t n = static_cast<int64_t>(nt) * BN + slot * kColsPerWarp + 16 * c + tq;
+    if (n >= args.N) return;
+#pragma unroll
+    for (int h = 0; h < 2; ++h)
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+            const int64_t m = static_cast<int64_t>(mt) * BM + quarter * 32 + 16 * h + 8 * e + trow;
+            if (m >= args.M) continue;
+            float vv[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+                vv[i] = __uint_as_float(static_cast<uint32_t>(e ? (acc[4 * h + i] >> 32) : acc[4 * h + i]));
+            store_quad<OUT>(args.y, m * args.N + n, add_bias4(args, n, make_float4(vv[0], vv[1], vv[2], vv[3])));
+        }
 }
 
 // ---------------------------------------------------------------------------
@@ -1069,11 +1201,22 @@ bool make_operand_map(CUtensorMap *m, const void *base, int64_t rows, int64_t K,
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// SM count of the current device (0 if there is none), looked up once per device.
+int device_sms_or_zero()
+{
+    constexpr int kMaxDevices = 64;
+    static int cached[kMaxDevices];  // 0: not looked up yet
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+    if (dev >= 0 && dev < kMaxDevices && cached[dev] > 0) return cached[dev];
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) return 0;
+    if (dev >= 0 && dev < kMaxDevices) cached[dev] = n;
+    return n;
+}
+
 int num_sms()
 {
-    int dev = 0, n = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    const int n = device_sms_or_zero();
     return n > 0 ? n : 1;
 }
 
@@ -1109,6 +1252,17 @@ cudaError_t launch_tc_out(const CUtensorMap &ta, const CUtensorMap &tw, const Ge
     }
 }
 
+cudaError_t launch_tail_combine(const GemmArgs &args, int y_type, cudaStream_t s)
+{
+    const unsigned grid = static_cast<unsigned>(args.tail_tiles) * 4;
+    switch (y_type) {
+        case QUARTZ_OUT_F16: tail_combine_kernel<QUARTZ_OUT_F16><<<grid, kEpiWarps * 32, 0, s>>>(args); break;
+        case QUARTZ_OUT_BF16: tail_combine_kernel<QUARTZ_OUT_BF16><<<grid, kEpiWarps * 32, 0, s>>>(args); break;
+        default: tail_combine_kernel<QUARTZ_OUT_F32><<<grid, kEpiWarps * 32, 0, s>>>(args); break;
+    }
+    return cudaGetLastError();
+}
+
 template <int MODE, int OUT>
 cudaError_t launch_simt(const LinearWorkspace &ws, const GemmArgs &args, int K, cudaStream_t s)
 {
@@ -1135,6 +1289,9 @@ GemmArgs make_args(const LinearWorkspace &ws, int64_t M, int64_t N, int64_t K, c
     GemmArgs a;
     a.per_row = 0;
     a.wide = 0;
+    a.split = 1;
+    a.tail_tiles = 0;
+    a.tail_part = ws.tail_part;
     a.a_side = ws.a_side;
     a.w_side = ws.w_side;
     a.m_pad = ws.m_pad;
@@ -1145,6 +1302,7 @@ GemmArgs make_args(const LinearWorkspace &ws, int64_t M, int64_t N, int64_t K, c
     a.tiles_n = static_cast<int>((N + BN - 1) / BN);
     a.tiles_m = static_cast<int>((M + BM - 1) / BM);
     a.num_tiles = a.tiles_m * a.tiles_n;
+    a.full_tiles = a.num_tiles;
     a.bias = static_cast<const __half *>(bias);
     a.y = y;
     a.y_type = y_type;
@@ -1156,6 +1314,39 @@ GemmArgs make_args(const LinearWorkspace &ws, int64_t M, int64_t N, int64_t K, c
 
 }  // namespace
 
+// Split of the GEMM's last wave on this device (symmetric, group-64 fast
+// path): when the tiles left after whole waves fill at most half of one,
+// each of them is cut along K into `split` group ranges (at most
+// kMaxTailSplit, at least two groups each) for otherwise idle CTAs.
+constexpr int kMaxTailSplit = 4;
+
+void tail_split(int64_t M, int64_t N, int64_t K, int mode, int *tail, int *split)
+{
+    *tail = 0;
+    *split = 1;
+    const int sms = device_sms_or_zero();
+    if (mode != QUARTZ_SYMMETRIC || sms <= 0 || M <= 0) return;
+    const int64_t T = ((M + BM - 1) / BM) * ((N + BN - 1) / BN);
+    const int64_t P = T < sms ? T : sms;
+    const int64_t W = T / P, R = T % P, G = K / kGroupQ;
+    if (W < 1 || R == 0 || 2 * R > P) return;
+    int64_t S = P / R;
+    if (S > kMaxTailSplit) S = kMaxTailSplit;
+    if (S > G / 2) S = G / 2;
+    if (S < 2) return;
+    *tail = static_cast<int>(R);
+    *split = static_cast<int>(S);
+}
+
+int linear_tail_parts(int64_t M, int64_t N, int64_t K, int mode)
+{
+    int tail = 0, split = 1;
+    tail_split(M, N, K, mode, &tail, &split);
+    return split;
+}
+
+size_t tail_part_bytes(int tail, int split) { return static_cast<size_t>(tail) * split * kEpiWarps * 32 * 64 * 4; }
+
 size_t linear_workspace_bytes(int64_t M, int64_t N, int64_t K, int mode)
 {
     const int nside = mode == QUARTZ_ASYMMETRIC ? 3 : 1;
@@ -1164,6 +1355,9 @@ size_t linear_workspace_bytes(int64_t M, int64_t N, int64_t K, int mode)
     b += align256(static_cast<size_t>(round_up(N, 16)) * K);
     b += align256(static_cast<size_t>(nside) * G * round_up(M > 0 ? M : 1, BM) * 4);
     b += align256(static_cast<size_t>(nside) * G * round_up(N, BN) * 4);
+    int tail = 0, split = 1;
+    tail_split(M, N, K, mode, &tail, &split);
+    if (split > 1) b += align256(tail_part_bytes(tail, split));
     return b;
 }
 
@@ -1183,6 +1377,9 @@ void linear_workspace_carve(void *base, int64_t M, int64_t N, int64_t K, int mod
     ws->a_side = reinterpret_cast<float *>(p);
     p += align256(static_cast<size_t>(nside) * G * ws->m_pad * 4);
     ws->w_side = reinterpret_cast<float *>(p);
+    p += align256(static_cast<size_t>(nside) * G * ws->n_pad * 4);
+    tail_split(M, N, K, mode, &ws->tail_tiles, &ws->tail_split);
+    ws->tail_part = ws->tail_split > 1 ? reinterpret_cast<float *>(p) : nullptr;
 }
 
 size_t prepared_weights_bytes(int64_t N, int64_t K, int mode)
@@ -1258,6 +1455,17 @@ cudaError_t launch_gemm_tcgen05(const LinearWorkspace &ws, int64_t M, int64_t N,
     GemmArgs args = make_args(ws, M, N, K, bias, y, y_type, partials, partials_group, dev_err);
     args.per_row = per_row ? 1 : 0;
     args.wide = wide ? 1 : 0;
+    int tail = 0, split = 1;  // the workspace's split must still match this device's grid
+    if (mode == QUARTZ_SYMMETRIC && !partials && !per_row && ws.tail_split > 1 && ws.tail_part)
+        tail_split(M, N, K, mode, &tail, &split);
+    if (split > 1 && split == ws.tail_split && tail == ws.tail_tiles) {
+        args.split = ws.tail_split;
+        args.tail_tiles = ws.tail_tiles;
+        args.full_tiles = args.num_tiles - ws.tail_tiles;
+        cudaError_t e = launch_tc_out<QUARTZ_SYMMETRIC>(ta, tw, args, y_type, s);
+        if (e != cudaSuccess) return e;
+        return launch_tail_combine(args, y_type, s);
+    }
     if (per_row) return launch_tc_out<QUARTZ_SYMMETRIC>(ta, tw, args, y_type, s);
     return mode == QUARTZ_ASYMMETRIC ? launch_tc_out<QUARTZ_ASYMMETRIC>(ta, tw, args, y_type, s)
                                      : launch_tc_out<QUARTZ_SYMMETRIC>(ta, tw, args, y_type, s);

@@ -50,10 +50,15 @@ struct LinearWorkspace {
     void *w_op;      // E4M3 [round_up(N, 16), K]  decoded weights, rows transposed 4x4 inside 16-row blocks
     float *a_side;   // fp32 [nside][G][Mpad]  scale (and z, gsum when asymmetric)
     float *w_side;   // fp32 [nside][G][Npad]
+    float *tail_part;  // fp32 partial tiles of the split last wave (may be NULL)
     int64_t m_pad, n_pad;
     int nside;
+    int tail_tiles, tail_split;  // tiles of the split last wave and parts per tile (1 = no split)
 };
 size_t linear_workspace_bytes(int64_t M, int64_t N, int64_t K, int mode);
+// Parts each tile of the symmetric tcgen05 GEMM's split last wave is cut
+// into on the current device (1: no split).
+int linear_tail_parts(int64_t M, int64_t N, int64_t K, int mode);
 void linear_workspace_carve(void *base, int64_t M, int64_t N, int64_t K, int mode,
                             LinearWorkspace *ws);
 // Expands the operands to E4M3 and transposes their scales into the

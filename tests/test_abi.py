@@ -134,6 +134,24 @@ def test_linear_validation(lib):
     assert lib.quartz_selftest_timeout(10, None) == N.QUARTZ_ERR_INVALID_ARG
 
 
+def test_linear_launch_count(lib):
+    """Preparation + GEMM, plus the combine kernel only where a device splits
+    the last wave (never for one tile, with partials, asymmetric or on the
+    SIMT / shift GEMMs); 0 for invalid sizes or M = 0."""
+    cnt = lib.quartz_linear_launch_count
+    p = N.QuartzParams(64, 16, 0)
+    pa = N.QuartzParams(64, 16, 1)
+    for algo in (N.ALGO_TCGEN05, N.ALGO_SIMT, N.ALGO_SHIFT):
+        assert cnt(16, 24, 128, C.byref(p), algo, 0) == 2        # one tile: no split
+        assert cnt(18432, 9216, 3072, C.byref(pa), algo, 0) == 2  # asymmetric: no split
+        assert cnt(18432, 9216, 3072, C.byref(p), algo, 1) == 2   # with partials: no split
+    assert cnt(18432, 9216, 3072, C.byref(p), N.ALGO_TCGEN05, 0) in (2, 3)
+    assert cnt(0, 24, 128, C.byref(p), 0, 0) == 0
+    assert cnt(16, 20, 128, C.byref(p), 0, 0) == 0     # N % 8 != 0
+    assert cnt(16, 24, 100, C.byref(p), 0, 0) == 0     # K not a multiple of group_q
+    assert cnt(16, 24, 128, C.byref(p), 9, 0) == 0     # algorithm
+
+
 def test_code_bits_validation(lib):
     """16-bit stage-1 codes (Section 5 LLM variant): symmetric groups of 64;
     no SIMT GEMM and no int32 partials for them."""

@@ -150,6 +150,36 @@ def test_linear_full_size_sampled(Q, layer):
     va = O.decode_values(ea)[:, g * 64:(g + 1) * 64]
     vw = O.decode_values(ew)[:, g * 64:(g + 1) * 64]
     assert np.array_equal(part[rows_t].cpu().numpy().astype(np.int64), O.group_partials(va, vw, 64)[0])
+    # without group partials the symmetric launch may split its last wave of
+    # tiles along K (sums in another order, same bound)
+    y2 = Q.linear(a, w)
+    assert Q.device_status() == 0
+    _tol_check(y2[rows_t].float().cpu().numpy(), ref, rabs, G, "float16")
+
+
+# Shapes whose last wave of 128 x 256 tiles, on a 152-SM GB300, is cut along K:
+# 9 x 18 tiles = 152 + 10 (4 parts of 2-3 groups), 13 x 15 = 152 + 43
+# (3 parts), 12 x 18 = 152 + 64 with 4 groups (2 parts of 2), and 4 x 39 =
+# 152 + 4 with 5 groups (2 parts of 2 and 3).  Every m-tile is sampled.
+SPLIT_SHAPES = [(1100, 4400, 640), (1614, 3816, 640), (1472, 4408, 256), (449, 9904, 320)]
+
+
+@pytest.mark.parametrize("out_dtype", ["float16", "bfloat16", "float32"])
+@pytest.mark.parametrize("M,N,K", SPLIT_SHAPES)
+def test_linear_split_last_wave(Q, M, N, K, out_dtype):
+    xa = inputs.laplace_activations(M, K, seed=9100 + M)
+    xw = inputs.gaussian_weights(N, K, seed=9101 + N)
+    bias = np.random.default_rng(N).normal(0, 0.1, N).astype(np.float16)
+    a = Q.quantize(torch.from_numpy(xa).cuda(), group_s=16)
+    w = Q.encode_weights(torch.from_numpy(xw).cuda(), group_s=16)
+    b = torch.from_numpy(bias).cuda()
+    y = Q.linear(a, w, b, out_dtype=getattr(torch, out_dtype))
+    y_again = Q.linear(a, w, b, out_dtype=getattr(torch, out_dtype), w_prepared=Q.prepare_weights(w))
+    assert Q.device_status() == 0
+    assert torch.equal(y, y_again)
+    rows = np.unique(np.concatenate([np.arange(0, M, 5), [M - 1]]))
+    ref, rabs = O.linear(O.encode(xa[rows], 64, 16), O.encode(xw, 64, 16), bias, with_abs=True)
+    _tol_check(y[torch.from_numpy(rows).cuda()].float().cpu().numpy(), ref, rabs, K // 64, out_dtype)
 
 
 def test_bounded_wait_reports_timeout(Q):
