@@ -242,9 +242,13 @@ int32_t quartz_linear_ex(const quartz_encoded_t *a, const quartz_encoded_t *w,
  * activations and reading them back; results are bit-identical to
  * quartz_quantize followed by quartz_linear with the same parameters.
  *   x_f16      fp16 [M, K] device, 16-byte aligned
- *   w          encoded weights [N, K]; its params (group_s, mode) are used
- *              for the activations; SYMMETRIC mode, group_q == 64 and 8-bit
- *              codes only (else QUARTZ_ERR_UNSUPPORTED)
+ *   w          encoded weights [N, K]; its params (group_s, mode, code_bits)
+ *              are used for the activations; SYMMETRIC mode and
+ *              group_q == 64 only (else QUARTZ_ERR_UNSUPPORTED).  With
+ *              16-bit codes (Section 5 LLM variant) the activations are
+ *              encoded with 32767 levels and FLAGs 0..12 and written as the
+ *              E5M2 operand, bit-identical to quartz_quantize followed by
+ *              quartz_linear with QUARTZ_ALGO_TCGEN05
  *   bias_f16, y, y_type, workspace, workspace_bytes: as quartz_linear
  *              (quartz_linear_workspace_size(M, N, K, &w->p) bytes)
  *   a_out      NULL, or an encoded [M, K] tensor with w's params that also
@@ -255,7 +259,8 @@ int32_t quartz_linear_f16(const void *x_f16, int64_t M, const quartz_encoded_t *
 
 /* quartz_linear_f16 with the weights prepared once by quartz_prepare_weights
  * (`w_prepared`, from the same `w`; NULL = quartz_linear_f16): the call is
- * then one encoder launch and the GEMM. */
+ * then one encoder launch and the GEMM (plus the tail combine where
+ * quartz_linear_launch_count counts one). */
 int32_t quartz_linear_f16_ex(const void *x_f16, int64_t M, const quartz_encoded_t *w, const void *w_prepared,
                              const void *bias_f16, void *y, int32_t y_type, const quartz_encoded_t *a_out,
                              void *workspace, size_t workspace_bytes, void *stream);

@@ -228,7 +228,8 @@ def linear_f16(x, w: Encoded, bias=None, out_dtype=None, out=None, workspace=Non
                a_out: Encoded | None = None, stream=None, w_prepared=None):
     """Fused activation path: y = linear(quantize(x), w) from fp16 x [M, K]
     in one pass over x (the activations are encoded straight into the GEMM
-    operand; symmetric mode).  `a_out` optionally receives the encoding;
+    operand; symmetric mode, 8- or 16-bit codes as in w.params).  `a_out`
+    optionally receives the encoding;
     `w_prepared` = prepare_weights(w) skips the per-call weight preparation."""
     torch = _torch()
     _check_f16(x, "x")

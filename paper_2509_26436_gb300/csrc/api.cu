@@ -272,7 +272,8 @@ int32_t quartz_linear_f16_ex(const void *x_f16, int64_t M, const quartz_encoded_
 {
     int32_t rc = check_encoded(w);
     if (rc) return rc;
-    if (w->p.mode != QUARTZ_SYMMETRIC || w->p.group_q != 64 || wide_codes(w->p)) return QUARTZ_ERR_UNSUPPORTED;
+    if (w->p.mode != QUARTZ_SYMMETRIC || w->p.group_q != 64) return QUARTZ_ERR_UNSUPPORTED;
+    const bool wide = wide_codes(w->p);  // 16-bit stage-1 codes: E5M2 operands
     const int64_t N = w->rows, K = w->K;
     rc = check_shape(M, K, &w->p);
     if (rc) return rc;
@@ -283,7 +284,7 @@ int32_t quartz_linear_f16_ex(const void *x_f16, int64_t M, const quartz_encoded_
         rc = check_encoded(a_out);
         if (rc) return rc;
         if (a_out->rows != M || a_out->K != K || a_out->p.group_q != w->p.group_q ||
-            a_out->p.group_s != w->p.group_s || a_out->p.mode != w->p.mode)
+            a_out->p.group_s != w->p.group_s || a_out->p.mode != w->p.mode || wide_codes(a_out->p) != wide)
             return QUARTZ_ERR_INVALID_ARG;
     }
     if (M * N >= (int64_t(1) << 40)) return QUARTZ_ERR_UNSUPPORTED;
@@ -305,7 +306,7 @@ int32_t quartz_linear_f16_ex(const void *x_f16, int64_t M, const quartz_encoded_
     cudaError_t e = launch_encode_operand(x_f16, M, K, &w->p, ws, a_out, s);
     if (e == cudaSuccess && !w_prepared) e = launch_prepare(nullptr, w, ws, s);
     if (e == cudaSuccess)
-        e = launch_gemm_tcgen05(ws, M, N, K, w->p.mode, bias_f16, y, y_type, nullptr, 0, dev_err, s);
+        e = launch_gemm_tcgen05(ws, M, N, K, w->p.mode, bias_f16, y, y_type, nullptr, 0, dev_err, s, false, wide);
     return map_cuda(e);
 }
 

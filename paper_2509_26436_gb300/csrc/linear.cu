@@ -34,6 +34,7 @@
 // accumulator-shift GEMM below is the exact path for those operands.
 #include <cuda.h>
 #include <cuda_fp16.h>
+#include <atomic>
 #include <type_traits>
 #include <cuda_bf16.h>
 #include <cuda_fp8.h>
@@ -1205,12 +1206,13 @@ bool make_operand_map(CUtensorMap *m, const void *base, int64_t rows, int64_t K,
 int device_sms_or_zero()
 {
     constexpr int kMaxDevices = 64;
-    static int cached[kMaxDevices];  // 0: not looked up yet
+    static std::atomic<int> cached[kMaxDevices];  // 0: not looked up yet
     int dev = 0, n = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return 0;
-    if (dev >= 0 && dev < kMaxDevices && cached[dev] > 0) return cached[dev];
+    const bool slot = dev >= 0 && dev < kMaxDevices;
+    if (slot && (n = cached[dev].load(std::memory_order_relaxed)) > 0) return n;
     if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) return 0;
-    if (dev >= 0 && dev < kMaxDevices) cached[dev] = n;
+    if (slot) cached[dev].store(n, std::memory_order_relaxed);
     return n;
 }
 

@@ -219,6 +219,68 @@ __device__ __forceinline__ UnitCodes encode_unit_sym_scaled(const uint4 lo, cons
     return u;
 }
 
+// The LLM variant of Section 5 on one unit (symmetric): Eq. 1 with 32767
+// levels (16-bit codes), then Eq. 2 straight to 4 bits with FLAG =
+// max(29 - clz(m), 0) in 0..12, m the OR of the subgroup's |q|.  The same
+// binary32 operations as the per-chunk encoder, so the codes, FLAGs and
+// scales are bit-identical to quartz_quantize's.  All 32 lanes call it
+// together (4 lanes per group).
+template <int GS>
+__device__ __forceinline__ UnitCodes encode_unit_wide(const uint4 lo, const uint4 hi)
+{
+    const uint32_t w[8] = {lo.x, lo.y, lo.z, lo.w, hi.x, hi.y, hi.z, hi.w};
+    float x[16];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        const float2 f = __half22float2(*reinterpret_cast<const __half2 *>(&w[i]));
+        x[2 * i] = f.x;
+        x[2 * i + 1] = f.y;
+    }
+    float amax = 0.f;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) amax = fmaxf(amax, fabsf(x[i]));
+    amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, 1));
+    amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, 2));
+    UnitCodes u;
+    u.s16 = __float2half_rn(__fdiv_rn(amax, 32767.0f));
+    const float s = __half2float(u.s16);
+    const float r = (s > 0.f) ? __frcp_rn(s) : 0.f;
+
+    int q[16];
+    uint32_t m0 = 0, m1 = 0;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+        const float t = fminf(fmaxf(__fmul_rn(x[i], r), -65536.0f), 65536.0f);
+        q[i] = min(max(__float2int_rn(t), -32767), 32767);
+        if (i < 8)
+            m0 |= static_cast<uint32_t>(abs(q[i]));
+        else
+            m1 |= static_cast<uint32_t>(abs(q[i]));
+    }
+    if (GS >= 16) {
+        m0 |= m1;
+        if (GS >= 32) m0 |= __shfl_xor_sync(0xffffffffu, m0, 1);
+        if (GS >= 64) m0 |= __shfl_xor_sync(0xffffffffu, m0, 2);
+        m1 = m0;
+    }
+    u.flag0 = max(29 - __clz(static_cast<int>(m0)), 0);
+    u.flag1 = max(29 - __clz(static_cast<int>(m1)), 0);
+    u.c0 = u.c1 = 0;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+        const int f = i < 8 ? u.flag0 : u.flag1;
+        const int mag = abs(q[i]) >> f;  // truncation toward zero
+        const uint32_t c = static_cast<uint32_t>(q[i] < 0 ? -mag : mag) & 0xFu;
+        if (i < 8)
+            u.c0 |= c << (4 * i);
+        else
+            u.c1 |= c << (4 * (i - 8));
+    }
+    u.flag_next = 0;
+    if (GS >= 16) u.flag_next = __shfl_down_sync(0xffffffffu, u.flag0, kUnitsPerSub<GS>());
+    return u;
+}
+
 // Store one unit's FLAGs: one byte per subgroup, or (packed) two per byte,
 // subgroup 2j in the low nibble of byte j; a packed byte is written by the
 // lane holding its first subgroup.
@@ -339,7 +401,7 @@ __global__ void __launch_bounds__(kThreads) quantize_row_sym_kernel(const uint4 
 // scale side values (fp32, [G][m_pad], rows at perm32(r)); units of the
 // padding rows [M, m_pad) write zero scales.  When `codes` is not NULL the
 // encoded tensor is stored as well.
-template <int GS>
+template <int GS, bool WIDE>
 __global__ void __launch_bounds__(kThreads) encode_operand_kernel(
     const uint4 *__restrict__ x, int64_t n_units, int64_t n_units_pad, int64_t units_per_row, int64_t m_pad,
     uint4 *__restrict__ a_op, float *__restrict__ a_side, uint2 *__restrict__ codes,
@@ -358,7 +420,7 @@ __global__ void __launch_bounds__(kThreads) encode_operand_kernel(
 #pragma unroll
     for (int j = 0; j < kUnitsPerThread; ++j) {
         const int64_t u = base + j * kThreads;
-        const UnitCodes c = encode_unit_sym<GS>(raw[j][0], raw[j][1]);
+        const UnitCodes c = WIDE ? encode_unit_wide<GS>(raw[j][0], raw[j][1]) : encode_unit_sym<GS>(raw[j][0], raw[j][1]);
         if (u >= n_units_pad) continue;
         const int64_t row = u / units_per_row;
         if ((lane & 3) == 0) {
@@ -367,8 +429,13 @@ __global__ void __launch_bounds__(kThreads) encode_operand_kernel(
         }
         if (u >= n_units) continue;
         uint4 o;
-        e4m3_from_codes8(c.c0, c.flag0, o.x, o.y);
-        e4m3_from_codes8(c.c1, c.flag1, o.z, o.w);
+        if (WIDE) {
+            e5m2_from_codes8(c.c0, c.flag0, o.x, o.y);
+            e5m2_from_codes8(c.c1, c.flag1, o.z, o.w);
+        } else {
+            e4m3_from_codes8(c.c0, c.flag0, o.x, o.y);
+            e4m3_from_codes8(c.c1, c.flag1, o.z, o.w);
+        }
         a_op[u] = o;
         if (codes) store_unit_sym<GS>(c, u, lane, codes, flags, scales, packed != 0);
     }
@@ -682,11 +749,20 @@ cudaError_t launch_encode_operand(const void *x, int64_t M, int64_t K, const qua
     uint8_t *flags = enc ? enc->flags : nullptr;
     __half *scales = enc ? reinterpret_cast<__half *>(enc->scales) : nullptr;
     const int packed = enc && enc->p.flag_bits == 4;
+    if (p->code_bits == 16) {  // Section 5 LLM variant: E5M2 operand
+        switch (p->group_s) {
+            case 8: encode_operand_kernel<8, true><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
+            case 16: encode_operand_kernel<16, true><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
+            case 32: encode_operand_kernel<32, true><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
+            default: encode_operand_kernel<64, true><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
+        }
+        return cudaGetLastError();
+    }
     switch (p->group_s) {
-        case 8: encode_operand_kernel<8><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
-        case 16: encode_operand_kernel<16><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
-        case 32: encode_operand_kernel<32><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
-        default: encode_operand_kernel<64><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
+        case 8: encode_operand_kernel<8, false><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
+        case 16: encode_operand_kernel<16, false><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
+        case 32: encode_operand_kernel<32, false><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
+        default: encode_operand_kernel<64, false><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
     }
     return cudaGetLastError();
 }

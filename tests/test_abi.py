@@ -180,8 +180,11 @@ def test_code_bits_validation(lib):
     assert lin(a, w, N.ALGO_SHIFT, part=0x4000) == N.QUARTZ_ERR_UNSUPPORTED
     assert lin(a, w, N.ALGO_TCGEN05, part=0x4000) == N.QUARTZ_ERR_UNSUPPORTED
     assert lin(a, enc(24, 128, bits=8), N.ALGO_SHIFT) == N.QUARTZ_ERR_INVALID_ARG  # mixed widths
-    assert lib.quartz_linear_f16(0x1000, 16, C.byref(w), None, 0x2000, 0, None, 0x3000, 1 << 30,
-                                 None) == N.QUARTZ_ERR_UNSUPPORTED
+    # the fused path takes 16-bit codes; an a_out of the other code width is rejected
+    assert lib.quartz_linear_f16(0x1000, 16, C.byref(w), None, 0x2000, 0, C.byref(enc(16, 128, bits=8)),
+                                 0x3000, 1 << 30, None) == N.QUARTZ_ERR_INVALID_ARG
+    assert lib.quartz_linear_f16(0x1000, 16, C.byref(enc(24, 128, mode=1)), None, 0x2000, 0, None,
+                                 0x3000, 1 << 30, None) == N.QUARTZ_ERR_UNSUPPORTED
 
 
 def test_attention_validation(lib):

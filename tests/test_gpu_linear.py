@@ -182,6 +182,25 @@ def test_linear_split_last_wave(Q, M, N, K, out_dtype):
     _tol_check(y[torch.from_numpy(rows).cuda()].float().cpu().numpy(), ref, rabs, K // 64, out_dtype)
 
 
+def test_split_last_wave_launch_count(Q):
+    """The host takes the split exactly when the tiles after whole waves
+    fill at most half a wave and each part keeps at least two groups; the
+    launch count and the workspace report it."""
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    for M, N, K in SPLIT_SHAPES + [(2048, 4096, 4096), (1100, 4400, 128), (128, 256, 640)]:
+        T = -(-M // 128) * -(-N // 256)
+        P = min(T, sms)
+        W, R = divmod(T, P)
+        split = W >= 1 and 0 < R <= P // 2 and min(P // R, 4, K // 128) >= 2
+        if sms == 152 and (M, N, K) in SPLIT_SHAPES:
+            assert split
+        assert Q.linear_launch_count(M, N, K) == (3 if split else 2)
+        assert Q.linear_launch_count(M, N, K, partials=True) == 2
+        assert Q.linear_launch_count(M, N, K, algo=Q.ALGO_SIMT) == 2
+        parts = min(P // R, 4, K // 128) if split else 0
+        assert Q.linear_workspace_size(M, N, K) >= R * parts * 128 * 256 * 4
+
+
 def test_bounded_wait_reports_timeout(Q):
     """Failure detection without a fault: a kernel waits on an mbarrier that
     nothing arrives at, gives up after 1 ms and the host reads the status;

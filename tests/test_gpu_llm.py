@@ -252,3 +252,44 @@ def test_linear16_tcgen05_llama_layers_sampled(Q, layer):
     rt = torch.from_numpy(rows).cuda()
     _tc_tol_check(y[rt].float().cpu().numpy(), O.encode16(xa[rows], 64, 8), O.encode16(xw, 64, 8), None,
                   layer.K // 64, "float16")
+
+
+# --- fused activation path with 16-bit codes ---------------------------------
+
+@pytest.mark.parametrize("flag_bits", [8, 4])
+@pytest.mark.parametrize("gs", [8, 16, 32, 64])
+@pytest.mark.parametrize("M,N,K", [(1, 8, 64), (200, 264, 640), (129, 520, 1216)])
+def test_linear16_f16_fused_identical(Q, M, N, K, gs, flag_bits):
+    """quartz_linear_f16 on 16-bit codes: the activations' encoding written
+    beside the E5M2 operand equals quartz_quantize's bit for bit, and so does
+    y against quantize + the tcgen05 linear; y also within tolerance of the
+    oracle."""
+    xa = inputs.laplace_activations(M, K, seed=6100 + M + gs, outlier_frac=0.002, outlier_scale=100.0)
+    xw = inputs.gaussian_weights(N, K, seed=6101 + N + gs)
+    xa[0, :64] = 0.0                                        # an all-zero group
+    bias = torch.from_numpy(np.random.default_rng(N).normal(0, 0.1, N).astype(np.float16)).cuda()
+    x = torch.from_numpy(xa).cuda()
+    w = Q.encode_weights(torch.from_numpy(xw).cuda(), group_s=gs, code_bits=16, flag_bits=flag_bits)
+    a = Q.quantize(x, group_s=gs, code_bits=16, flag_bits=flag_bits)
+    ref = Q.linear(a, w, bias, out_dtype=torch.float32, algo=Q.ALGO_TCGEN05)
+    a_out = Q.empty_encoded(M, K, w.params, x.device)
+    y = Q.linear_f16(x, w, bias, out_dtype=torch.float32, a_out=a_out)
+    y_prep = Q.linear_f16(x, w, bias, out_dtype=torch.float32, w_prepared=Q.prepare_weights(w))
+    assert Q.device_status() == 0
+    assert torch.equal(a_out.codes, a.codes) and torch.equal(a_out.flags, a.flags)
+    assert torch.equal(a_out.scales.view(torch.int16), a.scales.view(torch.int16))
+    assert torch.equal(y, ref) and torch.equal(y_prep, ref)
+    ea, ew = O.encode16(xa, 64, gs), O.encode16(xw, 64, gs)
+    _tc_tol_check(y.cpu().numpy(), ea, ew, bias.cpu().numpy(), K // 64, "float32")
+
+
+def test_linear16_f16_fused_llama_qkv(Q):
+    """Full-size LLaMA-2-7B qkv (its last wave split along K) through the
+    fused path: identical to quantize + linear."""
+    layer = [l for l in inputs.CONFIG_LLM if l.name == "llama2_qkv"][0]
+    x = torch.from_numpy(layer.activations()).cuda()
+    w = Q.encode_weights(torch.from_numpy(layer.weights()).cuda(), group_s=8, code_bits=16)
+    ref = Q.linear(Q.quantize(x, group_s=8, code_bits=16), w, algo=Q.ALGO_TCGEN05)
+    y = Q.linear_f16(x, w, w_prepared=Q.prepare_weights(w))
+    assert Q.device_status() == 0
+    assert torch.equal(y, ref)
