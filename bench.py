@@ -725,7 +725,7 @@ def run_llm_variant(args, Q, inputs, dev, n_sm, sm_mhz, peak_src, fp8_peak):
                                    "work": "2 dp4a + 1 shift + 1 add per output per 8-wide subgroup"}},
             "peak_source": f"alu: {n_sm} SMs x {FP32_LANES_PER_SM} lanes x {sm_mhz:.0f} MHz ({peak_src} "
                            f"max SM clock); tensor: {peak_src} bf16 burst x {FP8_OVER_BF16}",
-            "encode": {"kernel": "quantize_kernel<8, sym, wide>", "per_layer_ms": quant_ms,
+            "encode": {"kernel": "quantize_sym_kernel<8, wide>", "per_layer_ms": quant_ms,
                        "gbs": enc_bytes / (sum(quant_ms) / 1e3) / 1e9},
             "inputs": "seeded synthetic Laplace(0,0.05), 0.2% channels x100; weights N(0,0.02)"}
 

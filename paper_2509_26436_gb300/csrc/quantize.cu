@@ -312,7 +312,7 @@ __device__ __forceinline__ void store_unit_sym(const UnitCodes &u, int64_t unit,
     if ((lane & 3) == 0) scales[unit >> 2] = u.s16;
 }
 
-template <int GS>
+template <int GS, bool WIDE>
 __global__ void __launch_bounds__(kThreads) quantize_sym_kernel(const uint4 *__restrict__ x, int64_t n_units,
                                                                 uint2 *__restrict__ codes,
                                                                 uint8_t *__restrict__ flags,
@@ -331,7 +331,7 @@ __global__ void __launch_bounds__(kThreads) quantize_sym_kernel(const uint4 *__r
 #pragma unroll
     for (int j = 0; j < kUnitsPerThread; ++j) {
         const int64_t u = base + j * kThreads;
-        const UnitCodes c = encode_unit_sym<GS>(raw[j][0], raw[j][1]);
+        const UnitCodes c = WIDE ? encode_unit_wide<GS>(raw[j][0], raw[j][1]) : encode_unit_sym<GS>(raw[j][0], raw[j][1]);
         if (u < n_units) store_unit_sym<GS>(c, u, lane, codes, flags, scales, packed != 0);
     }
 }
@@ -454,10 +454,8 @@ __device__ __forceinline__ void unpack8(const uint4 &raw, float (&x)[8])
 
 // Encode the 8 elements of one chunk.  All 32 lanes must call this together
 // (the group and subgroup reductions are warp shuffles); `valid` only gates
-// the stores.  WIDE selects the LLM variant of Section 5 (symmetric only):
-// stage 1 quantizes to 16-bit codes (32767 levels) and Eq. 2 compresses them
-// straight to 4 bits, FLAG = max(29 - clz(m), 0) in 0..12.
-template <int GS, int MODE, bool WIDE>
+// the stores.  (16-bit codes, symmetric: encode_unit_wide.)
+template <int GS, int MODE>
 __device__ __forceinline__ void encode_chunk(const uint4 raw, int64_t chunk, bool valid, int lane,
                                              uint32_t *__restrict__ codes,
                                              uint8_t *__restrict__ flags,
@@ -477,7 +475,7 @@ __device__ __forceinline__ void encode_chunk(const uint4 raw, int64_t chunk, boo
         amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, 1));
         amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, 2));
         amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, 4));
-        s32 = __fdiv_rn(amax, WIDE ? 32767.0f : 127.0f);
+        s32 = __fdiv_rn(amax, 127.0f);
     } else {
         float hi = 0.f;  // the range always contains 0
 #pragma unroll
@@ -502,8 +500,8 @@ __device__ __forceinline__ void encode_chunk(const uint4 raw, int64_t chunk, boo
     uint32_t m = 0;
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
-        constexpr float kT = WIDE ? 65536.0f : 1024.0f;  // beyond the cap, below int overflow
-        constexpr int kQ = WIDE ? 32767 : 127;
+        constexpr float kT = 1024.0f;  // beyond the cap, below int overflow
+        constexpr int kQ = 127;
         const float t = fminf(fmaxf(__fmul_rn(x[i], r), -kT), kT);
         q[i] = min(max(__float2int_rn(t) + z, -kQ), kQ);
         m |= static_cast<uint32_t>(abs(q[i]));
@@ -551,7 +549,7 @@ __device__ __forceinline__ void encode_chunk(const uint4 raw, int64_t chunk, boo
     }
 }
 
-template <int GS, int MODE, bool WIDE>
+template <int GS, int MODE>
 __global__ void __launch_bounds__(kThreads) quantize_kernel(const uint4 *__restrict__ x,
                                                             int64_t n_chunks,
                                                             uint32_t *__restrict__ codes,
@@ -571,7 +569,7 @@ __global__ void __launch_bounds__(kThreads) quantize_kernel(const uint4 *__restr
 #pragma unroll
     for (int j = 0; j < kChunksPerThread; ++j) {
         const int64_t c = base + j * kThreads;
-        encode_chunk<GS, MODE, WIDE>(raw[j], c, c < n_chunks, lane, codes, flags, scales, zeros, gsum,
+        encode_chunk<GS, MODE>(raw[j], c, c < n_chunks, lane, codes, flags, scales, zeros, gsum,
                                      packed != 0);
     }
 }
@@ -601,7 +599,7 @@ __global__ void __launch_bounds__(kThreads) kv_append_kernel(const uint4 *__rest
         const int64_t r = c / chunks_per_row;
         const int64_t dst_row = (r / T) * L_max + t0 + (r % T);
         const int64_t dst = dst_row * chunks_per_row + (c - r * chunks_per_row);
-        encode_chunk<GS, QUARTZ_SYMMETRIC, false>(raw[j], dst, c < n_chunks, lane, codes, flags, scales,
+        encode_chunk<GS, QUARTZ_SYMMETRIC>(raw[j], dst, c < n_chunks, lane, codes, flags, scales,
                                                   nullptr, nullptr, packed != 0);
     }
 }
@@ -635,11 +633,11 @@ __global__ void __launch_bounds__(kThreads) dequantize_kernel(
 template <int GS, int MODE, bool WIDE = false>
 cudaError_t launch_q(const void *x, const quartz_encoded_t *e, cudaStream_t s)
 {
-    if constexpr (MODE == QUARTZ_SYMMETRIC && !WIDE) {
+    if constexpr (MODE == QUARTZ_SYMMETRIC) {
         const int64_t n_units = e->rows * e->K / 16;
         const int64_t per_block = kThreads * kUnitsPerThread;
         const int64_t blocks = (n_units + per_block - 1) / per_block;
-        quantize_sym_kernel<GS><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(
+        quantize_sym_kernel<GS, WIDE><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(
             static_cast<const uint4 *>(x), n_units, reinterpret_cast<uint2 *>(e->codes), e->flags,
             reinterpret_cast<__half *>(e->scales), e->p.flag_bits == 4);
         return cudaGetLastError();
@@ -647,7 +645,7 @@ cudaError_t launch_q(const void *x, const quartz_encoded_t *e, cudaStream_t s)
         const int64_t n_chunks = e->rows * e->K / 8;
         const int64_t per_block = kThreads * kChunksPerThread;
         const int64_t blocks = (n_chunks + per_block - 1) / per_block;
-        quantize_kernel<GS, MODE, WIDE><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(
+        quantize_kernel<GS, MODE><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(
             static_cast<const uint4 *>(x), n_chunks, reinterpret_cast<uint32_t *>(e->codes), e->flags,
             reinterpret_cast<__half *>(e->scales), e->zeros, e->gsum, e->p.flag_bits == 4);
         return cudaGetLastError();
