@@ -528,7 +528,7 @@ int oracle_linear(const uint8_t *a_codes, const uint8_t *a_flags, const uint16_t
 /* ---------------------------------------------------------------------------
  * QuaRTZ attention, one decode step (Appendix D, Table 6: QuaRTZ kernels for
  * attention with heads x 128 dimensions and LZS groups of 8 / 16 / 32).  The
- * paper gives no formula; the reading used here (R18): the query and the
+ * paper gives no formula; the reading used here: the query and the
  * key / value caches are encoded with Eq. 1 + Eq. 2 per token, groups of
  * `gq` along the head dimension d, and for each of the BH (batch x head)
  * rows
