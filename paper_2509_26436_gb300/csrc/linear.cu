@@ -228,8 +228,12 @@ struct GemmArgs {
     // (the same count each); each of the remaining tail_tiles is cut along K
     // into `split` group ranges taken by CTAs 0 .. tail_tiles * split - 1,
     // which leave fp32 partial tiles in tail_part; tail_combine_kernel adds
-    // them in part order and writes the outputs.
+    // them in part order and writes the outputs.  Two-wave form (ls > 0):
+    // the last tail_tiles tiles' tail_tiles * G group iterations are cut into
+    // one contiguous range of ls per CTA; a tile met by two ranges leaves
+    // parts 0 (groups from 0) and 1 (groups to G), the others are stored whole.
     int full_tiles, tail_tiles, split;
+    int ls;
     float *tail_part;     // [tail_tiles][split][16][kEpiWarps * 32] float4 (fp32 pairs)
 };
 
@@ -274,6 +278,12 @@ __device__ __forceinline__ int work_items(const GemmArgs &a)
 {
     const int c = blockIdx.x, P = gridDim.x;
     if (a.split <= 1) return (a.num_tiles - c + P - 1) / P;
+    if (a.ls > 0) {  // (tail_tiles * G < 2^30: checked on the host)
+        const int nf = a.full_tiles / P;
+        const int U = a.tail_tiles * a.G, b = c * a.ls, e = min(b + a.ls, U);
+        if (b >= e) return nf;
+        return nf + (e - 1) / a.G - b / a.G + 1;
+    }
     return a.full_tiles / P + (c < a.tail_tiles * a.split ? 1 : 0);
 }
 
@@ -281,6 +291,22 @@ __device__ __forceinline__ WorkItem work_item(const GemmArgs &a, int k)
 {
     WorkItem w;
     const int c = blockIdx.x, P = gridDim.x;
+    if (a.ls > 0 && k >= a.full_tiles / P) {
+        const int U = a.tail_tiles * a.G, b = c * a.ls, e = min(b + a.ls, U);
+        const int t = b / a.G + (k - a.full_tiles / P);
+        const int t0 = t * a.G;
+        w.tile = a.full_tiles + t;
+        w.g0 = max(b - t0, 0);
+        w.g1 = min(e - t0, a.G);
+        if (w.g0 == 0 && w.g1 == a.G) {
+            w.part = -1;
+            w.tail = 0;
+        } else {
+            w.part = w.g0 == 0 ? 0 : 1;
+            w.tail = t;
+        }
+        return w;
+    }
     if (a.split <= 1 || k < a.full_tiles / P) {
         w.tile = c + k * P;
         w.g0 = 0;
@@ -945,6 +971,8 @@ __global__ void __launch_bounds__(kEpiWarps * 32) tail_combine_kernel(const __gr
     constexpr int T = kEpiWarps * 32;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int tail = blockIdx.x >> 2, c = blockIdx.x & 3;
+    if (args.ls > 0 && (tail * args.G) / args.ls == ((tail + 1) * args.G - 1) / args.ls)
+        return;  // the tile lies in one CTA's range: stored whole by the GEMM
     const uint4 *src = reinterpret_cast<const uint4 *>(args.tail_part) +
                        static_cast<int64_t>(tail) * args.split * 16 * T + 4 * c * T + threadIdx.x;
     uint64_t acc[8];
@@ -1292,6 +1320,7 @@ GemmArgs make_args(const LinearWorkspace &ws, int64_t M, int64_t N, int64_t K, c
     a.per_row = 0;
     a.wide = 0;
     a.split = 1;
+    a.ls = 0;
     a.tail_tiles = 0;
     a.tail_part = ws.tail_part;
     a.a_side = ws.a_side;
@@ -1319,19 +1348,35 @@ GemmArgs make_args(const LinearWorkspace &ws, int64_t M, int64_t N, int64_t K, c
 // Split of the GEMM's last wave on this device (symmetric, group-64 fast
 // path): when the tiles left after whole waves fill at most half of one,
 // each of them is cut along K into `split` group ranges (at most
-// kMaxTailSplit, at least two groups each) for otherwise idle CTAs.
+// kMaxTailSplit, at least two groups each) for otherwise idle CTAs.  When
+// they fill more than half, the last two waves' group iterations are spread
+// evenly over the CTAs (two-wave form), but only where that shortens the
+// critical path by at least kMinStreamSaving group iterations: it costs
+// about the time of 25 (partial tiles written and read back, the combine
+// launch), measured on the LLaMA-2-7B o (saves 20: 3% slower) and down
+// (saves 54: 9% faster) projections.
 constexpr int kMaxTailSplit = 4;
+constexpr int kMinStreamSaving = 32;
 
-void tail_split(int64_t M, int64_t N, int64_t K, int mode, int *tail, int *split)
+void tail_split(int64_t M, int64_t N, int64_t K, int mode, int *tail, int *split, int *ls = nullptr)
 {
     *tail = 0;
     *split = 1;
+    if (ls) *ls = 0;
     const int sms = device_sms_or_zero();
     if (mode != QUARTZ_SYMMETRIC || sms <= 0 || M <= 0) return;
     const int64_t T = ((M + BM - 1) / BM) * ((N + BN - 1) / BN);
     const int64_t P = T < sms ? T : sms;
     const int64_t W = T / P, R = T % P, G = K / kGroupQ;
-    if (W < 1 || R == 0 || 2 * R > P) return;
+    if (W >= 1 && 2 * R > P) {
+        const int64_t Ts = P + R, U = Ts * G;
+        if (G * (P - R) < kMinStreamSaving * P || U >= (int64_t(1) << 30)) return;
+        *tail = static_cast<int>(Ts);
+        *split = 2;
+        if (ls) *ls = static_cast<int>((U + P - 1) / P);
+        return;
+    }
+    if (W < 1 || R == 0) return;
     int64_t S = P / R;
     if (S > kMaxTailSplit) S = kMaxTailSplit;
     if (S > G / 2) S = G / 2;
@@ -1380,7 +1425,7 @@ void linear_workspace_carve(void *base, int64_t M, int64_t N, int64_t K, int mod
     p += align256(static_cast<size_t>(nside) * G * ws->m_pad * 4);
     ws->w_side = reinterpret_cast<float *>(p);
     p += align256(static_cast<size_t>(nside) * G * ws->n_pad * 4);
-    tail_split(M, N, K, mode, &ws->tail_tiles, &ws->tail_split);
+    tail_split(M, N, K, mode, &ws->tail_tiles, &ws->tail_split, &ws->tail_ls);
     ws->tail_part = ws->tail_split > 1 ? reinterpret_cast<float *>(p) : nullptr;
 }
 
@@ -1457,11 +1502,12 @@ cudaError_t launch_gemm_tcgen05(const LinearWorkspace &ws, int64_t M, int64_t N,
     GemmArgs args = make_args(ws, M, N, K, bias, y, y_type, partials, partials_group, dev_err);
     args.per_row = per_row ? 1 : 0;
     args.wide = wide ? 1 : 0;
-    int tail = 0, split = 1;  // the workspace's split must still match this device's grid
+    int tail = 0, split = 1, ls = 0;  // the workspace's split must still match this device's grid
     if (mode == QUARTZ_SYMMETRIC && !partials && !per_row && ws.tail_split > 1 && ws.tail_part)
-        tail_split(M, N, K, mode, &tail, &split);
-    if (split > 1 && split == ws.tail_split && tail == ws.tail_tiles) {
+        tail_split(M, N, K, mode, &tail, &split, &ls);
+    if (split > 1 && split == ws.tail_split && tail == ws.tail_tiles && ls == ws.tail_ls) {
         args.split = ws.tail_split;
+        args.ls = ls;
         args.tail_tiles = ws.tail_tiles;
         args.full_tiles = args.num_tiles - ws.tail_tiles;
         cudaError_t e = launch_tc_out<QUARTZ_SYMMETRIC>(ta, tw, args, y_type, s);

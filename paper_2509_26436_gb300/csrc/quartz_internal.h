@@ -53,7 +53,8 @@ struct LinearWorkspace {
     float *tail_part;  // fp32 partial tiles of the split last wave (may be NULL)
     int64_t m_pad, n_pad;
     int nside;
-    int tail_tiles, tail_split;  // tiles of the split last wave and parts per tile (1 = no split)
+    int tail_tiles, tail_split;  // tiles of the split last wave(s) and parts per tile (1 = no split)
+    int tail_ls;                 // two-wave form: group iterations per CTA (0: one-wave form)
 };
 size_t linear_workspace_bytes(int64_t M, int64_t N, int64_t K, int mode);
 // Parts each tile of the symmetric tcgen05 GEMM's split last wave is cut

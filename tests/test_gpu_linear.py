@@ -183,22 +183,30 @@ def test_linear_split_last_wave(Q, M, N, K, out_dtype):
 
 
 def test_split_last_wave_launch_count(Q):
-    """The host takes the split exactly when the tiles after whole waves
-    fill at most half a wave and each part keeps at least two groups; the
-    launch count and the workspace report it."""
+    """The host splits the last wave when the tiles after whole waves fill at
+    most half a wave and each part keeps at least two groups, and spreads the
+    last two waves over all CTAs when they fill more than half and that saves
+    at least 32 group iterations on the critical path; the launch count and
+    the workspace report it."""
     sms = torch.cuda.get_device_properties(0).multi_processor_count
-    for M, N, K in SPLIT_SHAPES + [(2048, 4096, 4096), (1100, 4400, 128), (128, 256, 640)]:
+    shapes = SPLIT_SHAPES + [(2048, 4096, 4096), (2048, 4096, 11008), (1100, 4400, 128), (128, 256, 640)]
+    for M, N, K in shapes:
         T = -(-M // 128) * -(-N // 256)
         P = min(T, sms)
         W, R = divmod(T, P)
-        split = W >= 1 and 0 < R <= P // 2 and min(P // R, 4, K // 128) >= 2
-        if sms == 152 and (M, N, K) in SPLIT_SHAPES:
+        G = K // 64
+        if W >= 1 and 2 * R > P:
+            split, part_tiles = G * (P - R) >= 32 * P, 2 * (P + R)
+        else:
+            split = W >= 1 and R > 0 and min(P // R, 4, G // 2) >= 2
+            part_tiles = R * min(P // R, 4, G // 2) if split else 0
+        if sms == 152 and (M, N, K) in SPLIT_SHAPES + [(2048, 4096, 11008)]:
             assert split
         assert Q.linear_launch_count(M, N, K) == (3 if split else 2)
         assert Q.linear_launch_count(M, N, K, partials=True) == 2
         assert Q.linear_launch_count(M, N, K, algo=Q.ALGO_SIMT) == 2
-        parts = min(P // R, 4, K // 128) if split else 0
-        assert Q.linear_workspace_size(M, N, K) >= R * parts * 128 * 256 * 4
+        if split:
+            assert Q.linear_workspace_size(M, N, K) >= part_tiles * 128 * 256 * 4
 
 
 def test_bounded_wait_reports_timeout(Q):
