@@ -184,8 +184,12 @@ int32_t quartz_linear_launch_count(int64_t M, int64_t N, int64_t K, const quartz
  *   workspace  device scratch of at least quartz_linear_workspace_size bytes,
  *              16-byte aligned, owned by the caller; contents are scratch
  * Requirements: N % 8 == 0, K % 64 == 0, M >= 0.  The per-group partials
- * P_g are exact; the scaled sum is accumulated in binary32 and rounded once
- * to y_type.  Operands with 16-bit stage-1 codes (code_bits = 16, both
+ * P_g are exact; the scaled sum is accumulated in binary32 in group order
+ * and rounded once to y_type.  Where the symmetric TCGEN05 GEMM (no
+ * partials) splits its last wave(s) of tiles along K (see
+ * quartz_linear_launch_count), those tiles sum up to 4 consecutive runs of
+ * groups separately and then add the runs in order: no chain is longer than
+ * K/64 terms, and results are the same on every call on the same device.  Operands with 16-bit stage-1 codes (code_bits = 16, both
  * operands; decoded values up to 7 << 12, a group sum up to
  * 64 * 28672^2 > 2^31): QUARTZ_ALGO_SHIFT keeps P_g exact in 64-bit
  * integers; TCGEN05 (E5M2 operands) multiplies exactly but sums each group
@@ -204,8 +208,9 @@ int32_t quartz_linear(const quartz_encoded_t *a, const quartz_encoded_t *w, cons
  *   algo              quartz_algo_t: which GEMM kernel runs
  *   w_prepared        NULL, or prepared weights (below)
  *   gemm_event_begin  NULL, or a cudaEvent_t recorded on `stream` right before
- *   gemm_event_end    / right after the GEMM kernel (after operand expansion),
- *                     so a caller can time the GEMM kernel alone */
+ *   gemm_event_end    / right after the GEMM kernel and its tail combine, if
+ *                     any (after operand expansion), so a caller can time the
+ *                     GEMM alone */
 typedef struct {
     int32_t *partials;
     int32_t partials_group;
