@@ -17,6 +17,13 @@ time); the encode GB/s of the quantize kernel is reported beside it.  The
 inputs (~0.8 GB of fp16 activations per step) exceed the 129 MB L2, so no
 flush is needed between steps.  Multi-GPU runs are independent replicas
 (the path shards by token rows with no exchange): weak scaling.
+
+Secondary lines in the same JSON object (N = 1): `configs` times the single
+256 x 1152 layer, the quantize / decode sweep over 1M / 16M / 128M elements
+at G_s 8 / 16 / 32, the PixArt-Sigma and SDXL layers, and the paper's Table 1
+layer sizes (L2 flushed before every repetition); `peaks_measured` holds the
+fp32-pipe and FP8 tensor rates measured in the same run, the roofline
+denominators beside the derived and MEASURED_PEAKS.json figures.
 """
 from __future__ import annotations
 
@@ -55,6 +62,9 @@ def parse():
     p.add_argument("--no-attention", dest="attention", action="store_false",
                    help="skip the attention decode step leg (Appendix D, Table 6: heads x 128, "
                         "G_s 8/16/32, a 4096-token encoded cache, batch 16)")
+    p.add_argument("--no-configs", dest="configs", action="store_false",
+                   help="skip the secondary lines: configs 0-3 (single 1152 layer, encode/decode sweep, "
+                        "PixArt and SDXL layers) and the Table 1 layer sizes")
     p.add_argument("--no-llm", dest="llm", action="store_false",
                    help="skip the LLM-variant leg (Section 5: 16-bit codes straight to 4 bits, "
                         "G_s = 8, LLaMA-2-7B block linears)")
@@ -233,30 +243,80 @@ class ClockSampler:
 # --------------------------------------------------------------------------
 # CPU oracle baseline (a bounded sample of the same workload)
 # --------------------------------------------------------------------------
-def oracle_sample(layers, rows_per_layer, xs=None, ws=None, cols_per_layer=None, per_row=False):
-    """Time the oracle on `rows_per_layer` token rows of every layer (and the
-    first `cols_per_layer` output channels, or all): encode (Eq. 1 + Eq. 2)
-    of those rows plus the W4A4 linear for them.  Weights are encoded before
-    timing, like the GPU path.  Returns (seconds, ops)."""
+ORACLE_ROWS = 256
+
+
+def cpu_model():
+    """The host CPU's model name (/proc/cpuinfo, else lscpu, else the ISA)."""
+    try:
+        with open("/proc/cpuinfo") as fh:
+            for line in fh:
+                if line.lower().startswith("model name"):
+                    return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    import platform
+    return platform.machine()
+
+
+def oracle_setup(layers, rows_per_layer, xs=None, ws=None, per_row=False):
+    """Encode every layer's weights with the oracle (before timing, as the
+    GPU path does) and pick `rows_per_layer` evenly spaced token rows."""
     import numpy as np
 
     import oracle as O
     enc_w, xa_s = [], []
     for i, l in enumerate(layers):
         w = ws[i] if ws is not None else l.weights()
-        if cols_per_layer is not None:
-            w = np.ascontiguousarray(w[:cols_per_layer])
         enc_w.append(O.encode(w, l.K if per_row else GROUP_Q, GROUP_S))
         x = xs[i] if xs is not None else l.activations()
         sel = np.linspace(0, l.M - 1, rows_per_layer).astype(np.int64)
         xa_s.append(np.ascontiguousarray(x[sel]))
-    t0 = time.perf_counter()
-    ops = 0
-    for l, x, ew in zip(layers, xa_s, enc_w):
+    return enc_w, xa_s
+
+
+def oracle_step(layers, enc_w, xa_s, threads, per_row=False):
+    """One sampled step of the oracle: encode (Eq. 1 + Eq. 2) of the sampled
+    rows and the W4A4 linear for them, every output channel of every layer.
+    The rows of a layer are split into `threads` contiguous chunks run on
+    host threads (the oracle's C functions release the GIL).  Returns
+    (seconds, ops)."""
+    import concurrent.futures as cf
+
+    import numpy as np
+
+    import oracle as O
+
+    def work(l, x, ew):
         ea = O.encode(x, l.K if per_row else GROUP_Q, GROUP_S)
         O.linear(ea, ew)
-        ops += 2 * x.shape[0] * ew.rows * l.K
+
+    t0 = time.perf_counter()
+    ops = 0
+    with cf.ThreadPoolExecutor(max_workers=threads) as ex:
+        futs = []
+        for l, x, ew in zip(layers, xa_s, enc_w):
+            for chunk in np.array_split(np.arange(x.shape[0]), threads):
+                if chunk.size:
+                    futs.append(ex.submit(work, l, np.ascontiguousarray(x[chunk]), ew))
+            ops += 2 * x.shape[0] * ew.rows * l.K
+        for f in futs:
+            f.result()
     return time.perf_counter() - t0, ops
+
+
+def oracle_sample_desc(rows, threads):
+    return (f"{rows} evenly spaced token rows x all output channels of each of the 4 FLUX block linears "
+            f"per step (encode + linear), plain C oracle on {threads} host threads (rows split in "
+            "contiguous chunks; each thread's call decodes the layer's weights, as the oracle does), "
+            "weights encoded before timing")
 
 
 def run_reference(args):
@@ -265,30 +325,81 @@ def run_reference(args):
     if rank != 0:
         return
     layers = select_layers(inputs.CONFIG4, args.layers)
-    rows, cols = 1, 1024
-    xs = [l.activations() for l in layers]
-    ws = [l.weights() for l in layers]
+    threads = os.cpu_count() or 1
+    enc_w, xa_s = oracle_setup(layers, ORACLE_ROWS)
     times = []
     total_ops = 0
     for i in range(args.warmup + args.steps):
-        t, ops = oracle_sample(layers, rows, xs, ws, cols)
+        t, ops = oracle_step(layers, enc_w, xa_s, threads)
         if i >= args.warmup:
             times.append(t)
             total_ops = ops
     t_step = sum(times) / len(times)
     value = total_ops / t_step / 1e12
-    sample = (f"{rows} token row x the first {cols} output channels of each of the 4 FLUX block "
-              "linears per step (encode + linear), single-threaded plain C oracle, weights "
-              "encoded before timing")
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_step * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64/f64",
         "data": "synthetic", "config": layer_config(layers),
-        "cpu_baseline": {"value": value, "unit": "TOPS", "cores": 1, "kind": "oracle",
-                         "sample": sample},
+        "cpu_baseline": {"value": value, "unit": "TOPS", "cores": threads, "host_cores": os.cpu_count(),
+                         "cpu_model": cpu_model(), "kind": "oracle",
+                         "sample": oracle_sample_desc(ORACLE_ROWS, threads)},
         "e2e": {"value": value, "unit": "TOPS", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }), flush=True)
+
+
+# --------------------------------------------------------------------------
+# roofline denominators measured in this run
+# --------------------------------------------------------------------------
+def measure_peaks(torch, Q, dev, n_sm):
+    """Rates of the two pipes the GEMM uses, measured here (CUDA events, best
+    of several launches, nothing else running):
+      fp32_pipe   the paired fp32 multiply / fused multiply-add probe of
+                  libquartz (8 CTAs of 256 threads per SM), fp32 lane
+                  operations per second;
+      fp8_cublas  cuBLASLt FP8 E4M3 GEMM 8192^3 through torch._scaled_mm
+                  (the library peak, measured like the bf16 peak in
+                  MEASURED_PEAKS.json), FLOP/s;
+      fp8_tcgen05 libquartz's MMA probe: back-to-back tcgen05 kind::f8f6f4
+                  M128 N256 K32 from shared memory, one CTA per SM (the
+                  GEMM's own instruction and shape), FLOP/s."""
+    ev = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
+    stream = torch.cuda.current_stream()
+
+    def best(fn, reps):
+        fn()
+        torch.cuda.synchronize()
+        ts = []
+        for _ in range(reps):
+            e0, e1 = ev(), ev()
+            e0.record(stream)
+            work = fn()
+            e1.record(stream)
+            ts.append((e0, e1, work))
+        torch.cuda.synchronize()
+        return max(w / (a.elapsed_time(b) / 1e3) for a, b, w in ts)
+
+    out = {}
+    sink = torch.empty(n_sm * 8 * 256, dtype=torch.float32, device=dev)
+    out["fp32_pipe_tops"] = best(lambda: Q.probe_fp32_pipe(n_sm * 8, 20000, sink), 5) / 1e12
+    out["fp8_tcgen05_probe_tflops"] = best(lambda: Q.probe_mma_f8(n_sm, 20000), 5) / 1e12
+    assert Q.device_status() == 0
+    try:
+        n = 8192
+        g = torch.Generator(device=dev).manual_seed(1)
+        a = (torch.rand((n, n), generator=g, device=dev) - 0.5).to(torch.float8_e4m3fn)
+        b = (torch.rand((n, n), generator=g, device=dev) - 0.5).to(torch.float8_e4m3fn)
+        one = torch.ones((), dtype=torch.float32, device=dev)
+
+        def mm():
+            torch._scaled_mm(a, b.t(), one, one, out_dtype=torch.bfloat16)
+            return 2 * n ** 3
+        out["fp8_cublas_tflops"] = best(mm, 10) / 1e12
+        del a, b
+    except (RuntimeError, AttributeError, TypeError) as exc:
+        out["fp8_cublas_tflops"] = None
+        out["fp8_cublas_error"] = str(exc).splitlines()[0][:160]
+    return out
 
 
 # --------------------------------------------------------------------------
@@ -309,7 +420,13 @@ def run_ours(args):
         dist.init_process_group("nccl", device_id=dev)
     hbm_peak, bf16_peak, sm_mhz, peak_src = peaks()
     n_sm = torch.cuda.get_device_properties(dev).multi_processor_count
-    fp8_peak = bf16_peak * FP8_OVER_BF16                              # TFLOP/s
+    meas = measure_peaks(torch, Q, dev, n_sm)
+    if meas.get("fp8_cublas_tflops"):
+        fp8_peak = meas["fp8_cublas_tflops"]                          # TFLOP/s
+        fp8_src = "measured in this run: cuBLASLt FP8 E4M3 GEMM 8192^3 (torch._scaled_mm), best of 10"
+    else:
+        fp8_peak = bf16_peak * FP8_OVER_BF16
+        fp8_src = f"{peak_src} bf16 burst {bf16_peak} x {FP8_OVER_BF16} (nominal FP8 : BF16)"
     alu_peak = n_sm * FP32_LANES_PER_SM * sm_mhz * 1e6 / 1e12         # T fp32-pipe lane ops/s
     layers = select_layers(inputs.CONFIG4, args.layers)
 
@@ -408,10 +525,16 @@ def run_ours(args):
     alu_view = {"achieved": gemm_alu, "unit": "Top/s", "peak": alu_peak, "frac": gemm_alu / alu_peak,
                 "peak_source": f"derived: {n_sm} SMs x {FP32_LANES_PER_SM} fp32 lanes x "
                                f"{sm_mhz:.0f} MHz ({peak_src} max SM clock)",
+                "peak_measured": meas["fp32_pipe_tops"],
+                "frac_of_measured": gemm_alu / meas["fp32_pipe_tops"],
+                "peak_measured_source": "measured in this run: paired fp32 mul/fma probe "
+                                        "(quartz_probe_fp32_pipe), best of 5",
                 "work": ("1 fp32 add + 1 int32 add per output per 256 of K" if per_row else
                          "2 fp32 ops (multiply + fused multiply-add) per output per 64-wide group")}
     tensor_view = {"achieved": gemm_tflops, "unit": "TFLOP/s", "peak": fp8_peak, "frac": gemm_tflops / fp8_peak,
-                   "peak_source": f"{peak_src} bf16 burst {bf16_peak} x {FP8_OVER_BF16} (nominal FP8 : BF16)",
+                   "peak_source": fp8_src,
+                   "tcgen05_probe_peak": meas["fp8_tcgen05_probe_tflops"],
+                   "frac_of_tcgen05_probe": gemm_tflops / meas["fp8_tcgen05_probe_tflops"],
                    "work": "2 M N K FP8 MMA flops"}
     bound = "alu" if t_floor_alu >= t_floor_tensor else "tensor"
     main, other = (alu_view, tensor_view) if bound == "alu" else (tensor_view, alu_view)
@@ -467,8 +590,10 @@ def run_ours(args):
         assert Q.device_status() == 0
 
     # ---- LLM variant (optional) ---------------------------------------------
-    llm = run_llm_variant(args, Q, inputs, dev, n_sm, sm_mhz, peak_src, fp8_peak) if args.llm else None
+    llm = run_llm_variant(args, Q, inputs, dev, n_sm, sm_mhz, peak_src, fp8_peak, fp8_src) if args.llm else None
     attn = run_attention(args, Q, inputs, dev, hbm_peak, peak_src) if args.attention else None
+    configs = (run_configs(args, torch, Q, inputs, dev, hbm_peak, alu_peak, fp8_peak)
+               if args.configs and world == 1 and not per_row else None)
 
     # ---- end to end through the public API with host buffers ---------------
     # Each (step, layer) unit copies its activations from pinned host memory,
@@ -482,7 +607,7 @@ def run_ours(args):
         x_buf = [[torch.empty_like(x_dev[i]) for i in range(nl)] for _ in range(2)]
         y_buf = [[torch.empty_like(y_dev[i]) for i in range(nl)] for _ in range(2)]
         s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
-        e_steps = max(3, min(args.steps // 10, 20))
+        e_steps = max(20, min(args.steps, 50))
 
         def e2e_run(n_steps):
             loaded, consumed, computed, drained = {}, {}, {}, {}
@@ -511,25 +636,31 @@ def run_ours(args):
                     drained[u].record(s_out)
             stream.wait_event(drained[len(units) - 1])
 
-        e2e_run(1)
+        e2e_run(2)
         torch.cuda.synchronize()
-        barrier()
-        a0, a1 = ev(), ev()
-        a0.record(stream)
-        s_in.wait_stream(stream)
-        e2e_run(e_steps)
-        a1.record(stream)
-        torch.cuda.synchronize()
-        barrier()
-        te = a0.elapsed_time(a1) / 1e3 / e_steps
-        te = max_over_ranks(te, world, dev)
+        # three timed repetitions of e_steps steps each; the median is the
+        # value, the three are reported as the spread
+        reps = []
+        for _ in range(3):
+            barrier()
+            a0, a1 = ev(), ev()
+            a0.record(stream)
+            s_in.wait_stream(stream)
+            e2e_run(e_steps)
+            a1.record(stream)
+            torch.cuda.synchronize()
+            barrier()
+            reps.append(max_over_ranks(a0.elapsed_time(a1) / 1e3 / e_steps, world, dev))
+        te = statistics.median(reps)
         h2d = sum(x.numel() * 2 for x in x_host)
         d2h = sum(l.M * l.N * 2 for l in layers)
         link = host_link_gbs(torch, dev)
         floor = max(h2d / (link["h2d"] * 1e9), d2h / (link["d2h"] * 1e9), (h2d + d2h) / (link["both"] * 1e9))
         e2e = {"value": world * ops_step / te / 1e12, "unit": "TOPS",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": e_steps,
-               "ms_per_step": te * 1e3,
+               "ms_per_step": te * 1e3, "repetitions": len(reps),
+               "ms_per_step_reps": [r * 1e3 for r in reps],
+               "spread": (max(reps) - min(reps)) / te,
                "overlap": "H2D / compute / D2H on three streams, double-buffered",
                "roofline": {"bound": "host link", "link_gbs_measured": link,
                             "floor_ms": floor * 1e3, "frac": floor / te,
@@ -539,11 +670,15 @@ def run_ours(args):
     # ---- CPU oracle baseline (rank 0 only, N = 1) ---------------------------
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
-        rows = 128
-        t, ops = oracle_sample(layers, rows, xs, ws, per_row=per_row)
-        cpu = {"value": ops / t / 1e12, "unit": "TOPS", "cores": 1, "kind": "oracle",
-               "sample": f"{rows} token rows of each of the 4 layers (encode + linear), "
-                         f"{t:.1f} s single-threaded plain C"}
+        threads = os.cpu_count() or 1
+        enc_w_o, xa_o = oracle_setup(layers, ORACLE_ROWS, xs, ws, per_row=per_row)
+        tt, oo = 0.0, 0
+        for _ in range(3):
+            t, ops = oracle_step(layers, enc_w_o, xa_o, threads, per_row=per_row)
+            tt, oo = tt + t, oo + ops
+        cpu = {"value": oo / tt / 1e12, "unit": "TOPS", "cores": threads, "host_cores": os.cpu_count(),
+               "cpu_model": cpu_model(), "kind": "oracle",
+               "sample": oracle_sample_desc(ORACLE_ROWS, threads) + f"; 3 steps, {tt:.1f} s"}
 
     if world > 1:
         import torch.distributed as dist
@@ -565,10 +700,166 @@ def run_ours(args):
         "gemm_algos": algos,
         "llm_variant": llm,
         "attention": attn,
+        "configs": configs,
+        "peaks_measured": meas,
         "e2e": e2e,
         "cpu_baseline": cpu,
     }
     print(json.dumps(out), flush=True)
+
+
+# --------------------------------------------------------------------------
+# configs 0-3 and the paper's Table 1 layer sizes (secondary bench lines)
+# --------------------------------------------------------------------------
+L2_FLUSH_BYTES = 256 << 20   # written before every timed repetition (> 129 MB L2)
+CONFIG_REPS = 10
+
+
+def gemm_roofline(layers, gemm_ms, alu_peak, fp8_peak):
+    """Both floors of the tcgen05 GEMM for `layers` at the given per-layer
+    GEMM times: the fp32 pipe (2 ops per output and 64-group) and the FP8
+    tensor pipe (2 M N K)."""
+    t = sum(gemm_ms) / 1e3
+    epi = sum(2 * l.M * l.N * (l.K // GROUP_Q) for l in layers)
+    ops = sum(l.ops for l in layers)
+    alu, ten = epi / t / 1e12, ops / t / 1e12
+    return {"bound": "alu", "achieved": alu, "peak": alu_peak, "unit": "Top/s", "frac": alu / alu_peak,
+            "tensor": {"achieved": ten, "peak": fp8_peak, "unit": "TFLOP/s", "frac": ten / fp8_peak}}
+
+
+def time_linear_layers(torch, Q, dev, layers, xs, ws, flush, reps=CONFIG_REPS, group_s=GROUP_S):
+    """Per layer: quantize + linear (prepared weights), L2 flushed before each
+    repetition; CUDA events around the quantize kernel, the GEMM (+ tail
+    combine) and the whole layer.  Returns per-layer medians in ms."""
+    stream = torch.cuda.current_stream()
+    ev = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
+    out = []
+    for l, x, w in zip(layers, xs, ws):
+        xd = torch.from_numpy(x).to(dev)
+        ew = Q.encode_weights(torch.from_numpy(w).to(dev), group_s=group_s)
+        pw = Q.prepare_weights(ew)
+        ea = Q.empty_encoded(l.M, l.K, Q.Params(GROUP_Q, group_s), dev)
+        y = torch.empty((l.M, l.N), dtype=torch.float16, device=dev)
+        wsb = torch.empty(max(Q.linear_workspace_size(l.M, l.N, l.K, ea.params), 16), dtype=torch.uint8,
+                          device=dev)
+        for _ in range(3):
+            Q.quantize(xd, out=ea, group_s=group_s)
+            Q.linear(ea, ew, out=y, workspace=wsb, w_prepared=pw)
+        recs = []
+        for _ in range(reps):
+            flush()
+            e = [ev() for _ in range(5)]
+            e[0].record(stream)
+            Q.quantize(xd, out=ea, group_s=group_s)
+            e[1].record(stream)
+            Q.linear(ea, ew, out=y, workspace=wsb, w_prepared=pw, gemm_events=(e[2], e[3]))
+            e[4].record(stream)
+            recs.append(e)
+        torch.cuda.synchronize()
+        assert Q.device_status() == 0
+        med = lambda i, j: statistics.median(r[i].elapsed_time(r[j]) for r in recs)  # noqa: E731
+        out.append({"layer": l.name, "M": l.M, "N": l.N, "K": l.K, "ms": med(0, 4), "quantize_ms": med(0, 1),
+                    "gemm_ms": med(2, 3), "TOPS": l.ops / med(0, 4) / 1e9,
+                    "gemm_TOPS": l.ops / med(2, 3) / 1e9,
+                    "launches": 1 + Q.linear_launch_count(l.M, l.N, l.K, ea.params)})
+        del xd, ew, pw, ea, y, wsb
+    return out
+
+
+def run_encode_sweep(torch, Q, inputs, dev, hbm_peak, flush, reps=CONFIG_REPS):
+    """Config 1: quantize + LZS encode and decode (quartz_dequantize) of
+    1M / 16M / 128M fp16 elements ([256 | 4096 | 32768, 4096]; the smaller
+    tensors are the first rows of the 128M one) at G_s 8 / 16 / 32; L2
+    flushed before every repetition, CUDA events around the one kernel."""
+    stream = torch.cuda.current_stream()
+    ev = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
+    K = 4096
+    x_all = torch.from_numpy(inputs.mixture_activations(32768, K, seed=inputs.seed_for(1, 0))).to(dev)
+    res = []
+    for rows in (256, 4096, 32768):
+        x = x_all[:rows]
+        xhat = torch.empty_like(x)
+        n = rows * K
+        for gs in (8, 16, 32):
+            e = Q.empty_encoded(rows, K, Q.Params(GROUP_Q, gs), dev)
+            for _ in range(3):
+                Q.quantize(x, out=e, group_s=gs)
+                Q.dequantize(e, out=xhat)
+            te, td = [], []
+            for _ in range(reps):
+                flush()
+                a, b = ev(), ev()
+                a.record(stream)
+                Q.quantize(x, out=e, group_s=gs)
+                b.record(stream)
+                te.append((a, b))
+                flush()
+                a, b = ev(), ev()
+                a.record(stream)
+                Q.dequantize(e, out=xhat)
+                b.record(stream)
+                td.append((a, b))
+            torch.cuda.synchronize()
+            assert Q.device_status() == 0
+            ms_e = statistics.median(a.elapsed_time(b) for a, b in te)
+            ms_d = statistics.median(a.elapsed_time(b) for a, b in td)
+            enc_b = n * encode_bytes_per_elem(gs, GROUP_Q)
+            dec_b = n * (0.5 + 1.0 / gs + 2.0 / GROUP_Q + 2.0)
+            res.append({"elements": n, "shape": [rows, K], "group_s": gs,
+                        "encode_us": ms_e * 1e3, "encode_gbs": enc_b / ms_e / 1e6,
+                        "encode_frac": enc_b / ms_e / 1e6 / hbm_peak,
+                        "decode_us": ms_d * 1e3, "decode_gbs": dec_b / ms_d / 1e6,
+                        "decode_frac": dec_b / ms_d / 1e6 / hbm_peak,
+                        "note": "latency-bound (2.7 MB moved per launch)" if rows == 256 else "hbm-bound"})
+            del e
+    del x_all
+    return {"workload": "quantize+LZS encode / decode sweep, fp16 mixture 89% Laplace(0,0.05), "
+                        "10% N(0,0.3), 1% U(-8,8)",
+            "kernels": "quantize_sym_kernel / dequantize kernel", "peak_gbs": hbm_peak,
+            "encode_bytes": "2 + 1/2 + 1/G_s + 2/64 B per element",
+            "decode_bytes": "1/2 + 1/G_s + 2/64 + 2 B per element",
+            "l2": f"{L2_FLUSH_BYTES >> 20} MiB written before every repetition; median of {reps}",
+            "sizes": res}
+
+
+def run_configs(args, torch, Q, inputs, dev, hbm_peak, alu_peak, fp8_peak):
+    """Throughput of configs 0-3 and, as context for the paper's Table 1
+    (A100 latencies of 4096^2 / 5120^2 / 8192^2 layers at G_s 8 / 16 / 32, M
+    not stated), the same layers at M = 4096 tokens."""
+    buf = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    flush = buf.zero_
+    out = {"l2": f"{L2_FLUSH_BYTES >> 20} MiB written before every repetition; medians of {CONFIG_REPS}"}
+    for key, layers, desc in (("config0", inputs.CONFIG0, "single W4A4 linear 256 x 1152 -> 1152"),
+                              ("config2", inputs.CONFIG2, "PixArt-Sigma block linears, 8192 tokens"),
+                              ("config3", inputs.CONFIG3, "SDXL UNet 3x3 convs as im2col GEMMs, batch 2")):
+        xs = [l.activations() for l in layers]
+        ws = [l.weights() for l in layers]
+        per = time_linear_layers(torch, Q, dev, layers, xs, ws, flush)
+        t = sum(p["ms"] for p in per)
+        out[key] = {"workload": desc, "group_q": GROUP_Q, "group_s": GROUP_S, "mode": "symmetric", "out": "f16",
+                    "TOPS": sum(l.ops for l in layers) / t / 1e9, "ms_per_step": t,
+                    "layers": per,
+                    "roofline": gemm_roofline(layers, [p["gemm_ms"] for p in per], alu_peak, fp8_peak)}
+    out["config1"] = run_encode_sweep(torch, Q, inputs, dev, hbm_peak, flush)
+    # Table 1 context: the paper reports 0.189 / 0.184 / 0.176 ms (4096^2),
+    # 0.383 / 0.268 / 0.239 ms (5120^2) and 0.468 / 0.327 / 0.313 ms (8192^2)
+    # at g8 / g16 / g32 on an A100, M unstated
+    paper = {4096: (0.189, 0.184, 0.176), 5120: (0.383, 0.268, 0.239), 8192: (0.468, 0.327, 0.313)}
+    rows = []
+    M = 4096
+    for n, ref in paper.items():
+        x = inputs.laplace_activations(M, n, seed=inputs.seed_for(7, n % 97))
+        w = inputs.gaussian_weights(n, n, seed=inputs.seed_for(7, n % 97, 1))
+        for gs, ref_ms in zip((8, 16, 32), ref):
+            l = inputs.Layer(f"table1_{n}", M, n, n, 7, 0)
+            p = time_linear_layers(torch, Q, dev, [l], [x], [w], flush, group_s=gs)[0]
+            rows.append({"layer": f"{n}x{n}", "M": M, "group_s": gs, "ms": p["ms"], "gemm_ms": p["gemm_ms"],
+                         "TOPS": p["TOPS"], "paper_a100_ms": ref_ms})
+    out["table1_context"] = {"note": "paper: A100, s4 x s4 -> s32, M not stated (context, not a target); "
+                                     "here: one GB300, M = 4096 tokens, quantize + linear per call",
+                             "rows": rows}
+    del buf
+    return out
 
 
 LLM_GROUP_S = 8
@@ -624,7 +915,7 @@ def run_attention(args, Q, inputs, dev, hbm_peak, peak_src):
             "settings": out}
 
 
-def run_llm_variant(args, Q, inputs, dev, n_sm, sm_mhz, peak_src, fp8_peak):
+def run_llm_variant(args, Q, inputs, dev, n_sm, sm_mhz, peak_src, fp8_peak, fp8_src):
     """One step = encode (16-bit codes, G_s = 8) + linear of each of the four
     LLaMA-2-7B block linears at 2048 tokens; per-kernel CUDA-event times, for
     the tcgen05 GEMM (E5M2 operands) and the exact accumulator-shift GEMM."""
@@ -724,7 +1015,7 @@ def run_llm_variant(args, Q, inputs, dev, n_sm, sm_mhz, peak_src, fp8_peak):
                                    "unit": "Top/s", "frac": sh_ops / t_sh_gemm / 1e12 / alu_peak,
                                    "work": "2 dp4a + 1 shift + 1 add per output per 8-wide subgroup"}},
             "peak_source": f"alu: {n_sm} SMs x {FP32_LANES_PER_SM} lanes x {sm_mhz:.0f} MHz ({peak_src} "
-                           f"max SM clock); tensor: {peak_src} bf16 burst x {FP8_OVER_BF16}",
+                           f"max SM clock); tensor: {fp8_src}",
             "encode": {"kernel": "quantize_sym_kernel<8, wide>", "per_layer_ms": quant_ms,
                        "gbs": enc_bytes / (sum(quant_ms) / 1e3) / 1e9},
             "inputs": "seeded synthetic Laplace(0,0.05), 0.2% channels x100; weights N(0,0.02)"}

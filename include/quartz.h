@@ -348,6 +348,29 @@ int32_t quartz_device_status(void *stream);
  * the GEMM pipeline. */
 int32_t quartz_selftest_timeout(int64_t limit_ns, void *stream);
 
+/* ---------------------------------------------------------------------------
+ * Measurement aids.  The paper has no counterpart to these: they run one
+ * execution pipe of the SM at full rate so that a benchmark can state the
+ * linear layer's roofline against rates measured on the device at hand.
+ * Their results are timing only; time them with events on `stream`.
+ * ------------------------------------------------------------------------- */
+
+/* `blocks` CTAs of 256 threads; every thread runs `iters` rounds of 8
+ * independent fma.rn.f32x2 followed by 8 mul.rn.f32x2 (the paired fp32
+ * operations of the GEMM's dequant epilogue): blocks * 256 * iters * 32
+ * fp32 lane operations in total.  `sink` is a device float buffer of
+ * blocks * 256 elements that receives one value per thread (keeps the work
+ * observable).  1 <= blocks <= 2^20, 1 <= iters <= 2^32. */
+int32_t quartz_probe_fp32_pipe(int32_t blocks, int64_t iters, float *sink, void *stream);
+
+/* `blocks` CTAs (one per SM: each requests 200 KB of shared memory), each
+ * issuing 2 * iters back-to-back tcgen05.mma.cta_group::1.kind::f8f6f4
+ * M128 N256 K32 (E4M3 x E4M3 -> fp32 in TMEM) from one shared-memory stage:
+ * blocks * iters * 2 * (2 * 128 * 256 * 32) flops.  Every wait is bounded;
+ * a timeout is reported by quartz_device_status.  1 <= blocks <= 65535,
+ * 1 <= iters <= 2^24. */
+int32_t quartz_probe_mma_f8(int32_t blocks, int64_t iters, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

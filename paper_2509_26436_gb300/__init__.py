@@ -138,10 +138,12 @@ def quantize_static(x, scale, group_s: int = 16, group_q: int = 64, out: Encoded
     return e
 
 
-def dequantize(e: Encoded, stream=None):
-    """x_hat = s (v - z) as fp16 [rows, K]."""
+def dequantize(e: Encoded, stream=None, out=None):
+    """x_hat = s (v - z) as fp16 [rows, K] (into `out` if given)."""
     torch = _torch()
-    y = torch.empty((e.rows, e.K), dtype=torch.float16, device=e.codes.device)
+    y = out if out is not None else torch.empty((e.rows, e.K), dtype=torch.float16, device=e.codes.device)
+    if not (y.is_cuda and y.dtype == torch.float16 and y.is_contiguous() and y.numel() == e.rows * e.K):
+        raise ValueError("out must be a contiguous float16 CUDA tensor of rows x K elements")
     ec = e.c()
     N.check(N.load().quartz_dequantize(C.byref(ec), y.data_ptr(), _stream(stream)), "quartz_dequantize")
     return y
@@ -261,6 +263,25 @@ def device_status(stream=None) -> int:
 
 def selftest_timeout(limit_ns: int, stream=None) -> int:
     return int(N.load().quartz_selftest_timeout(limit_ns, _stream(stream)))
+
+
+# --- measurement aids (pipe-rate probes; no counterpart in the paper) -------
+
+def probe_fp32_pipe(blocks: int, iters: int, sink, stream=None) -> int:
+    """Launch the paired-fp32 probe; returns the fp32 lane operations it does
+    (blocks * 256 * iters * 32).  `sink`: float32 CUDA tensor of >= blocks * 256."""
+    if sink.numel() < blocks * 256 or not sink.is_cuda:
+        raise ValueError("sink must be a float32 CUDA tensor of at least blocks * 256 elements")
+    N.check(N.load().quartz_probe_fp32_pipe(blocks, iters, sink.data_ptr(), _stream(stream)),
+            "quartz_probe_fp32_pipe")
+    return blocks * 256 * iters * 32
+
+
+def probe_mma_f8(blocks: int, iters: int, stream=None) -> int:
+    """Launch the FP8 tcgen05 MMA probe; returns the flops it does
+    (blocks * iters * 2 MMAs of 2 * 128 * 256 * 32)."""
+    N.check(N.load().quartz_probe_mma_f8(blocks, iters, _stream(stream)), "quartz_probe_mma_f8")
+    return blocks * iters * 2 * 2 * 128 * 256 * 32
 
 
 # --- attention decode step (Appendix D, Table 6) ----------------------------

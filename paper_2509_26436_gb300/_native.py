@@ -81,6 +81,8 @@ SIGNATURES = {
                                        _P]),
     "quartz_device_status": (_I32, [_P]),
     "quartz_selftest_timeout": (_I32, [_I64, _P]),
+    "quartz_probe_fp32_pipe": (_I32, [_I32, _I64, _P, _P]),
+    "quartz_probe_mma_f8": (_I32, [_I32, _I64, _P]),
 }
 
 _lock = threading.Lock()

@@ -19,7 +19,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(PKG, "libquartz.so")
 BUILD_DIR = os.path.join(ROOT, "_build")
-SOURCES = ["api.cu", "quantize.cu", "linear.cu", "noalloc.cu", "attention.cu"]
+SOURCES = ["api.cu", "quantize.cu", "linear.cu", "noalloc.cu", "attention.cu", "probe.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

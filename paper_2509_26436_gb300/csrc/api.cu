@@ -96,7 +96,7 @@ const char *quartz_status_string(int32_t status)
     }
 }
 
-int32_t quartz_version(void) { return (1 << 16) | 6; }
+int32_t quartz_version(void) { return (1 << 16) | 7; }
 
 int32_t quartz_encoded_sizes(int64_t rows, int64_t K, const quartz_params_t *p, size_t out[5])
 {
@@ -391,6 +391,21 @@ int32_t quartz_selftest_timeout(int64_t limit_ns, void *stream)
     int *dev_err = device_error_word();
     if (!dev_err) return QUARTZ_ERR_CUDA;
     return map_cuda(launch_selftest_timeout(limit_ns, dev_err, static_cast<cudaStream_t>(stream)));
+}
+
+int32_t quartz_probe_fp32_pipe(int32_t blocks, int64_t iters, float *sink, void *stream)
+{
+    if (blocks < 1 || blocks > (1 << 20) || iters < 1 || iters > (int64_t(1) << 32) || !sink)
+        return QUARTZ_ERR_INVALID_ARG;
+    return map_cuda(launch_probe_fp32(blocks, iters, sink, static_cast<cudaStream_t>(stream)));
+}
+
+int32_t quartz_probe_mma_f8(int32_t blocks, int64_t iters, void *stream)
+{
+    if (blocks < 1 || blocks > (1 << 16) || iters < 1 || iters > (int64_t(1) << 24)) return QUARTZ_ERR_INVALID_ARG;
+    int *dev_err = device_error_word();
+    if (!dev_err) return QUARTZ_ERR_CUDA;
+    return map_cuda(launch_probe_mma_f8(blocks, iters, dev_err, static_cast<cudaStream_t>(stream)));
 }
 
 }  // extern "C"

@@ -94,5 +94,8 @@ cudaError_t launch_gemm_simt(const LinearWorkspace &ws, int64_t M, int64_t N, in
                              const void *bias, void *y, int y_type, int32_t *partials,
                              int partials_group, cudaStream_t s);
 cudaError_t launch_selftest_timeout(int64_t limit_ns, int *dev_err, cudaStream_t s);
+// Pipe-rate probes (probe.cu).
+cudaError_t launch_probe_fp32(int blocks, int64_t iters, float *sink, cudaStream_t s);
+cudaError_t launch_probe_mma_f8(int blocks, int64_t iters, int *dev_err, cudaStream_t s);
 
 }  // namespace quartz

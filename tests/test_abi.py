@@ -267,3 +267,13 @@ def test_missing_library_fails_loudly(tmp_path):
             N.load(str(tmp_path / "libquartz.so"))
     finally:
         N._lib = saved
+
+
+def test_probe_validation(lib):
+    """The pipe-rate probes reject bad sizes on the host (nothing launched)."""
+    assert lib.quartz_probe_fp32_pipe(0, 10, 0x1000, None) == N.QUARTZ_ERR_INVALID_ARG
+    assert lib.quartz_probe_fp32_pipe(4, 0, 0x1000, None) == N.QUARTZ_ERR_INVALID_ARG
+    assert lib.quartz_probe_fp32_pipe(4, 10, None, None) == N.QUARTZ_ERR_INVALID_ARG
+    assert lib.quartz_probe_mma_f8(0, 10, None) == N.QUARTZ_ERR_INVALID_ARG
+    assert lib.quartz_probe_mma_f8(4, 0, None) == N.QUARTZ_ERR_INVALID_ARG
+    assert lib.quartz_probe_mma_f8(1 << 17, 10, None) == N.QUARTZ_ERR_INVALID_ARG

@@ -182,6 +182,59 @@ def test_linear_split_last_wave(Q, M, N, K, out_dtype):
     _tol_check(y[torch.from_numpy(rows).cuda()].float().cpu().numpy(), ref, rabs, K // 64, out_dtype)
 
 
+# Shapes whose last wave is more than half full, so that the last P + R tiles'
+# group iterations are spread over all CTAs after one wave of whole tiles
+# (two-wave form), with 8-bit codes (exact P_g): 9 x 45 = 405 tiles = 2 x 152
+# + 101 with 96 groups, and 12 x 32 = 384 = 2 x 152 + 80 with 68 groups.  Both
+# mix whole tiles, whole tail tiles and tail tiles cut into two parts; M and
+# N are ragged, so the combine kernel stores partial edge tiles.
+TWO_WAVE_SHAPES = [(1100, 11400, 6144), (1500, 8000, 4352)]
+_two_wave_ref = {}
+
+
+def _two_wave_predicate(M, N, K, sms):
+    T = -(-M // 128) * -(-N // 256)
+    P = min(T, sms)
+    W, R = divmod(T, P)
+    return W >= 1 and 2 * R > P and (K // 64) * (P - R) >= 32 * P
+
+
+def _rows_every_m_tile(M):
+    rows = []
+    for m0 in range(0, M, 128):
+        m1 = min(m0 + 128, M)
+        rows += [m0, m0 + 1, m0 + 8, m0 + 37, m0 + 64, m1 - 9, m1 - 1]
+    return np.unique(np.clip(np.array(rows), 0, M - 1))
+
+
+@pytest.mark.parametrize("out_dtype", ["float16", "bfloat16", "float32"])
+@pytest.mark.parametrize("M,N,K", TWO_WAVE_SHAPES)
+def test_linear_two_wave_split_8bit(Q, M, N, K, out_dtype):
+    """Two-wave form on 8-bit codes against the oracle: all output columns of
+    rows sampled from every M tile, with a bias, three output types; the
+    prepared-weights call is bit-identical; the host really takes the form."""
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    if not _two_wave_predicate(M, N, K, sms):
+        pytest.skip(f"{sms} SMs: this shape does not take the two-wave form")
+    assert Q.linear_launch_count(M, N, K) == 3
+    xa = inputs.laplace_activations(M, K, seed=9200 + M)
+    xw = inputs.gaussian_weights(N, K, seed=9201 + N)
+    bias = np.random.default_rng(N + 1).normal(0, 0.1, N).astype(np.float16)
+    a = Q.quantize(torch.from_numpy(xa).cuda(), group_s=16)
+    w = Q.encode_weights(torch.from_numpy(xw).cuda(), group_s=16)
+    b = torch.from_numpy(bias).cuda()
+    y = Q.linear(a, w, b, out_dtype=getattr(torch, out_dtype))
+    y_again = Q.linear(a, w, b, out_dtype=getattr(torch, out_dtype), w_prepared=Q.prepare_weights(w))
+    assert Q.device_status() == 0
+    assert torch.equal(y, y_again)
+    rows = _rows_every_m_tile(M)
+    if (M, N, K) not in _two_wave_ref:
+        _two_wave_ref[(M, N, K)] = O.linear(O.encode(xa[rows], 64, 16), O.encode(xw, 64, 16), bias,
+                                            with_abs=True)
+    ref, rabs = _two_wave_ref[(M, N, K)]
+    _tol_check(y[torch.from_numpy(rows).cuda()].float().cpu().numpy(), ref, rabs, K // 64, out_dtype)
+
+
 def test_split_last_wave_launch_count(Q):
     """The host splits the last wave when the tiles after whole waves fill at
     most half a wave and each part keeps at least two groups, and spreads the

@@ -35,8 +35,17 @@ def _noalloc(Q, a, w, bias, y):
     return rc
 
 
-def test_noalloc_matches_workspace_entry_point(Q):
-    M, N, K = 200, 264, 640          # ragged M and N tiles, 10 groups
+# (200, 264, 640): ragged M and N tiles, 10 groups.  (1100, 4400, 640): on a
+# 152-SM GB300, 9 x 18 = 162 tiles, so the last 10 are cut into 4 parts each
+# whose partial tiles sit in the scratch array and are added by the combine
+# kernel.
+NOALLOC_SHAPES = [(200, 264, 640), (1100, 4400, 640)]
+SCRATCH_BYTES = 32 << 20   # QUARTZ_NOALLOC_SCRATCH_BYTES in quartz.h
+
+
+@pytest.mark.parametrize("M,N,K", NOALLOC_SHAPES)
+def test_noalloc_matches_workspace_entry_point(Q, M, N, K):
+    assert Q.linear_workspace_size(M, N, K) <= SCRATCH_BYTES
     w16 = inputs.gaussian_weights(N, K, seed=71)
     bias = torch.from_numpy(inputs.gaussian_weights(1, N, seed=72)[0]).cuda()
     w = Q.encode_weights(torch.from_numpy(w16).cuda(), group_s=16)
@@ -53,6 +62,7 @@ def test_noalloc_matches_workspace_entry_point(Q):
         # the results are in fact identical
         tol = 1e-5 * np.abs(exp) + (K // 64 + 4) * 2.0 ** -24 * np.abs(exp).max() + 2.0 ** -24
         assert (np.abs(got - exp) <= tol).all(), f"call {call}"
+        assert np.array_equal(got, exp), f"call {call}: same kernels, different result"
 
 
 def test_noalloc_rejects_oversized_problem(Q):
