@@ -96,21 +96,14 @@ struct PrepArgs {
 constexpr int kPrepThreads = 256;
 constexpr int kSideGroupsPerThread = 8;
 
-template <int GS, bool WIDE>
-__device__ __forceinline__ void run_expand(const ExpandJob &j, int64_t u)
+// kExpandUnits units per thread, a block apart (every load and store
+// instruction of a warp is contiguous); all loads are issued before any
+// decode so that several are in flight per thread.
+constexpr int kExpandUnits = 4;
+
+template <int GS>
+__device__ __forceinline__ void load_unit_flags(const ExpandJob &j, int64_t u, int &f0, int &f1)
 {
-    if (u >= j.units_pad) return;
-    int64_t dst = u;
-    if (j.permute) {
-        const int64_t r = u / j.units_per_row;
-        dst = perm16(r) * j.units_per_row + (u - r * j.units_per_row);
-    }
-    if (u >= j.units) {  // padding rows
-        j.out[dst] = make_uint4(0, 0, 0, 0);
-        return;
-    }
-    const uint2 c = j.codes[u];
-    int f0, f1;
     if (GS == 8) {
         if (j.packed_flags) {
             const uint32_t ff = j.flags[u];
@@ -124,15 +117,44 @@ __device__ __forceinline__ void run_expand(const ExpandJob &j, int64_t u)
     } else {
         f0 = f1 = load_flag(j.flags, (u * 16) / GS, j.packed_flags != 0);
     }
-    uint4 o;
-    if (WIDE) {
-        e5m2_from_codes8(c.x, f0, o.x, o.y);
-        e5m2_from_codes8(c.y, f1, o.z, o.w);
-    } else {
-        e4m3_from_codes8(c.x, f0, o.x, o.y);
-        e4m3_from_codes8(c.y, f1, o.z, o.w);
+}
+
+template <int GS, bool WIDE>
+__device__ __forceinline__ void run_expand(const ExpandJob &j, int64_t u0)
+{
+    uint2 c[kExpandUnits];
+    int f0[kExpandUnits], f1[kExpandUnits];
+#pragma unroll
+    for (int q = 0; q < kExpandUnits; ++q) {
+        const int64_t u = u0 + q * kPrepThreads;
+        c[q] = make_uint2(0u, 0u);
+        f0[q] = f1[q] = 0;
+        if (u < j.units) {
+            c[q] = __ldcs(j.codes + u);
+            load_unit_flags<GS>(j, u, f0[q], f1[q]);
+        }
     }
-    j.out[dst] = o;
+#pragma unroll
+    for (int q = 0; q < kExpandUnits; ++q) {
+        const int64_t u = u0 + q * kPrepThreads;
+        if (u >= j.units_pad) continue;
+        int64_t dst = u;
+        if (j.permute) {
+            const int64_t r = u / j.units_per_row;
+            dst = perm16(r) * j.units_per_row + (u - r * j.units_per_row);
+        }
+        uint4 o = make_uint4(0u, 0u, 0u, 0u);  // padding rows stay zero
+        if (u < j.units) {
+            if (WIDE) {
+                e5m2_from_codes8(c[q].x, f0[q], o.x, o.y);
+                e5m2_from_codes8(c[q].y, f1[q], o.z, o.w);
+            } else {
+                e4m3_from_codes8(c[q].x, f0[q], o.x, o.y);
+                e4m3_from_codes8(c[q].y, f1[q], o.z, o.w);
+            }
+        }
+        j.out[dst] = o;
+    }
 }
 
 __device__ __forceinline__ void run_side(const SideJob &j, int64_t t, int G, int nside)
@@ -161,9 +183,9 @@ __global__ void __launch_bounds__(kPrepThreads) prep_kernel(const __grid_constan
 {
     const int64_t bid = blockIdx.x;
     if (bid < args.block_end[0]) {
-        run_expand<GS, WIDE>(args.ex_a, bid * kPrepThreads + threadIdx.x);
+        run_expand<GS, WIDE>(args.ex_a, bid * (kPrepThreads * kExpandUnits) + threadIdx.x);
     } else if (bid < args.block_end[1]) {
-        run_expand<GS, WIDE>(args.ex_w, (bid - args.block_end[0]) * kPrepThreads + threadIdx.x);
+        run_expand<GS, WIDE>(args.ex_w, (bid - args.block_end[0]) * (kPrepThreads * kExpandUnits) + threadIdx.x);
     } else if (bid < args.block_end[2]) {
         run_side(args.sd_a, (bid - args.block_end[1]) * kPrepThreads + threadIdx.x, args.G, args.nside);
     } else {
@@ -1463,11 +1485,13 @@ cudaError_t launch_prepare(const quartz_encoded_t *a, const quartz_encoded_t *w,
         p.sd_a = {reinterpret_cast<const __half *>(a->scales), a->zeros, a->gsum, ws.a_side, a->rows, ws.m_pad, 1};
     p.sd_w = {reinterpret_cast<const __half *>(w->scales), w->zeros, w->gsum, ws.w_side, w->rows, ws.n_pad, 0};
     const int64_t side_chunks = (p.G + kSideGroupsPerThread - 1) / kSideGroupsPerThread;
-    const int64_t threads[4] = {expand ? p.ex_a.units_pad : 0, expand && !w_ready ? p.ex_w.units_pad : 0,
-                                a ? ws.m_pad * side_chunks : 0, w_ready ? 0 : ws.n_pad * side_chunks};
+    const int64_t items[4] = {expand ? p.ex_a.units_pad : 0, expand && !w_ready ? p.ex_w.units_pad : 0,
+                              a ? ws.m_pad * side_chunks : 0, w_ready ? 0 : ws.n_pad * side_chunks};
+    const int64_t per_block[4] = {kPrepThreads * kExpandUnits, kPrepThreads * kExpandUnits, kPrepThreads,
+                                  kPrepThreads};
     int64_t acc = 0;
     for (int i = 0; i < 4; ++i) {
-        acc += (threads[i] + kPrepThreads - 1) / kPrepThreads;
+        acc += (items[i] + per_block[i] - 1) / per_block[i];
         p.block_end[i] = acc;
     }
     if (acc == 0) return cudaSuccess;

@@ -605,29 +605,57 @@ __global__ void __launch_bounds__(kThreads) kv_append_kernel(const uint4 *__rest
 }
 
 // x_hat = s * (v - z), v = sgn(c) (|c| << FLAG); one thread per 8 elements.
+// Dequantiser: x_hat = s * (v - z), v = c << FLAG, in binary32, rounded once to
+// fp16.  Each thread takes kDeqChunksPerThread chunks of 8 elements (one
+// 32-bit code word in, one 16-byte fp16 vector out) spaced a block apart, so
+// that every load and store instruction of a warp is contiguous; all loads
+// are issued before any arithmetic, which keeps several of them in flight
+// per thread.  Subgroup and group indices are shifts (G_s and a 64-wide
+// group are powers of two); one scale per row (group_q = K, any K % 64 == 0)
+// divides by K.
+constexpr int kDeqChunksPerThread = 4;
+
+template <int GS>
 __global__ void __launch_bounds__(kThreads) dequantize_kernel(
     const uint32_t *__restrict__ codes, const uint8_t *__restrict__ flags,
-    const __half *__restrict__ scales, const int8_t *__restrict__ zeros, int group_s, int group_q,
+    const __half *__restrict__ scales, const int8_t *__restrict__ zeros, int64_t group_q,
     int packed, int64_t n_chunks, uint4 *__restrict__ out)
 {
-    const int64_t c = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x;
-    if (c >= n_chunks) return;
-    const uint32_t word = codes[c];
-    const int flag = load_flag(flags, (c * 8) / group_s, packed != 0);
-    const int64_t g = (c * 8) / group_q;
-    const float s = __half2float(scales[g]);
-    const int z = zeros ? zeros[g] : 0;
-    uint32_t o[4];
+    constexpr int kSubShift = GS == 8 ? 3 : GS == 16 ? 4 : GS == 32 ? 5 : 6;
+    const int64_t base = static_cast<int64_t>(blockIdx.x) * (kThreads * kDeqChunksPerThread) + threadIdx.x;
+    uint32_t word[kDeqChunksPerThread];
+    int flag[kDeqChunksPerThread], z[kDeqChunksPerThread];
+    float sc[kDeqChunksPerThread];
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const int c0 = static_cast<int>(word << (28 - 8 * i)) >> 28;
-        const int c1 = static_cast<int>(word << (24 - 8 * i)) >> 28;
-        const float y0 = __fmul_rn(s, static_cast<float>(c0 * (1 << flag) - z));
-        const float y1 = __fmul_rn(s, static_cast<float>(c1 * (1 << flag) - z));
-        const __half2 h = __floats2half2_rn(y0, y1);
-        o[i] = *reinterpret_cast<const uint32_t *>(&h);
+    for (int j = 0; j < kDeqChunksPerThread; ++j) {
+        const int64_t c = base + j * kThreads;
+        word[j] = 0u;
+        flag[j] = z[j] = 0;
+        sc[j] = 0.f;
+        if (c < n_chunks) {
+            word[j] = __ldcs(codes + c);
+            flag[j] = load_flag(flags, (c * 8) >> kSubShift, packed != 0);
+            const int64_t g = group_q == 64 ? (c >> 3) : (c * 8) / group_q;
+            sc[j] = __half2float(scales[g]);
+            if (zeros) z[j] = zeros[g];
+        }
     }
-    out[c] = make_uint4(o[0], o[1], o[2], o[3]);
+#pragma unroll
+    for (int j = 0; j < kDeqChunksPerThread; ++j) {
+        const int64_t c = base + j * kThreads;
+        if (c >= n_chunks) continue;
+        uint32_t o[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int c0 = static_cast<int>(word[j] << (28 - 8 * i)) >> 28;
+            const int c1 = static_cast<int>(word[j] << (24 - 8 * i)) >> 28;
+            const float y0 = __fmul_rn(sc[j], static_cast<float>(c0 * (1 << flag[j]) - z[j]));
+            const float y1 = __fmul_rn(sc[j], static_cast<float>(c1 * (1 << flag[j]) - z[j]));
+            const __half2 h = __floats2half2_rn(y0, y1);
+            o[i] = *reinterpret_cast<const uint32_t *>(&h);
+        }
+        __stcs(out + c, make_uint4(o[0], o[1], o[2], o[3]));
+    }
 }
 
 template <int GS, int MODE, bool WIDE = false>
@@ -769,12 +797,19 @@ cudaError_t launch_dequantize(const quartz_encoded_t *e, void *y, cudaStream_t s
 {
     const int64_t n_chunks = e->rows * e->K / 8;
     if (n_chunks == 0) return cudaSuccess;
-    const int64_t blocks = (n_chunks + kThreads - 1) / kThreads;
-    dequantize_kernel<<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(
-        reinterpret_cast<const uint32_t *>(e->codes), e->flags,
-        reinterpret_cast<const __half *>(e->scales),
-        e->p.mode == QUARTZ_ASYMMETRIC ? e->zeros : nullptr, e->p.group_s, e->p.group_q, e->p.flag_bits == 4, n_chunks,
-        static_cast<uint4 *>(y));
+    const int64_t per_block = kThreads * kDeqChunksPerThread;
+    const unsigned blocks = static_cast<unsigned>((n_chunks + per_block - 1) / per_block);
+    const uint32_t *codes = reinterpret_cast<const uint32_t *>(e->codes);
+    const __half *scales = reinterpret_cast<const __half *>(e->scales);
+    const int8_t *zeros = e->p.mode == QUARTZ_ASYMMETRIC ? e->zeros : nullptr;
+    const int packed = e->p.flag_bits == 4;
+    uint4 *out = static_cast<uint4 *>(y);
+    switch (e->p.group_s) {
+        case 8: dequantize_kernel<8><<<blocks, kThreads, 0, s>>>(codes, e->flags, scales, zeros, e->p.group_q, packed, n_chunks, out); break;
+        case 16: dequantize_kernel<16><<<blocks, kThreads, 0, s>>>(codes, e->flags, scales, zeros, e->p.group_q, packed, n_chunks, out); break;
+        case 32: dequantize_kernel<32><<<blocks, kThreads, 0, s>>>(codes, e->flags, scales, zeros, e->p.group_q, packed, n_chunks, out); break;
+        default: dequantize_kernel<64><<<blocks, kThreads, 0, s>>>(codes, e->flags, scales, zeros, e->p.group_q, packed, n_chunks, out); break;
+    }
     return cudaGetLastError();
 }
 
