@@ -538,9 +538,8 @@ def run_ours(args):
                    "work": "2 M N K FP8 MMA flops"}
     bound = "alu" if t_floor_alu >= t_floor_tensor else "tensor"
     main, other = (alu_view, tensor_view) if bound == "alu" else (tensor_view, alu_view)
-    roofline = {"bound": bound, "achieved": main["achieved"], "peak": main["peak"], "unit": main["unit"],
-                "frac": main["frac"], "traffic": None if per_row else gemm_traffic(),
-                "kernel": "gemm_tcgen05_kernel", "peak_source": main["peak_source"], "work": main["work"],
+    roofline = {"bound": bound, **main, "traffic": None if per_row else gemm_traffic(),
+                "kernel": "gemm_tcgen05_kernel",
                 "tensor" if bound == "alu" else "alu": other,
                 "floors_ms": {"alu": t_floor_alu * 1e3, "tensor": t_floor_tensor * 1e3},
                 "per_layer_ms": gemm_ms}
@@ -768,57 +767,99 @@ def time_linear_layers(torch, Q, dev, layers, xs, ws, flush, reps=CONFIG_REPS, g
 
 def run_encode_sweep(torch, Q, inputs, dev, hbm_peak, flush, reps=CONFIG_REPS):
     """Config 1: quantize + LZS encode and decode (quartz_dequantize) of
-    1M / 16M / 128M fp16 elements ([256 | 4096 | 32768, 4096]; the smaller
-    tensors are the first rows of the 128M one) at G_s 8 / 16 / 32; L2
-    flushed before every repetition, CUDA events around the one kernel."""
+    1M / 16M / 128M fp16 elements ([256 | 4096 | 32768, 4096]) at G_s 8 / 16 /
+    32.  Throughput: back-to-back launches over distinct row slices of one
+    128M-element tensor (and of one encoded tensor and one output tensor),
+    so that every launch reads and writes memory no earlier launch of the
+    cycle touched: 256 MB of inputs per cycle of slices (128 slices of 1M, 8
+    of 16M, the whole 128M), far above the 129 MB L2; CUDA events around
+    the whole sequence.  Latency: one launch after a 256 MiB L2 flush."""
     stream = torch.cuda.current_stream()
     ev = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
-    K = 4096
-    x_all = torch.from_numpy(inputs.mixture_activations(32768, K, seed=inputs.seed_for(1, 0))).to(dev)
+    K, R_ALL = 4096, 32768
+    x_all = torch.from_numpy(inputs.mixture_activations(R_ALL, K, seed=inputs.seed_for(1, 0))).to(dev)
+    xhat_all = torch.empty_like(x_all)
     res = []
-    for rows in (256, 4096, 32768):
-        x = x_all[:rows]
-        xhat = torch.empty_like(x)
-        n = rows * K
-        for gs in (8, 16, 32):
-            e = Q.empty_encoded(rows, K, Q.Params(GROUP_Q, gs), dev)
-            for _ in range(3):
-                Q.quantize(x, out=e, group_s=gs)
-                Q.dequantize(e, out=xhat)
-            te, td = [], []
+    for gs in (8, 16, 32):
+        e_all = Q.empty_encoded(R_ALL, K, Q.Params(GROUP_Q, gs), dev)
+
+        def enc_slice(i, rows):
+            sl = slice(i * rows, (i + 1) * rows)
+            return Q.Encoded(e_all.codes[sl], e_all.flags[sl], e_all.scales[sl], None, None, rows, K, e_all.params)
+
+        for rows in (256, 4096, 32768):
+            n_sl = R_ALL // rows
+            xs = [x_all[i * rows:(i + 1) * rows] for i in range(n_sl)]
+            hs = [xhat_all[i * rows:(i + 1) * rows] for i in range(n_sl)]
+            es = [enc_slice(i, rows) for i in range(n_sl)]
+            launches = max(20, n_sl)
+            for i in range(min(n_sl, 4)):
+                Q.quantize(xs[i], out=es[i], group_s=gs)
+                Q.dequantize(es[i], out=hs[i])
+            times = {}
+            for kind in ("encode", "decode"):
+                # the launches are captured in a CUDA graph so that the host's
+                # per-call cost does not starve the GPU between small kernels
+                g = torch.cuda.CUDAGraph()
+                side = torch.cuda.Stream(dev)
+                side.wait_stream(stream)
+                with torch.cuda.stream(side):
+                    with torch.cuda.graph(g, stream=side):
+                        for i in range(launches):
+                            if kind == "encode":
+                                Q.quantize(xs[i % n_sl], out=es[i % n_sl], group_s=gs)
+                            else:
+                                Q.dequantize(es[i % n_sl], out=hs[i % n_sl])
+                stream.wait_stream(side)
+                g.replay()
+                torch.cuda.synchronize()
+                reps_t = []
+                for _ in range(3):
+                    a, b = ev(), ev()
+                    a.record(stream)
+                    g.replay()
+                    b.record(stream)
+                    reps_t.append((a, b))
+                torch.cuda.synchronize()
+                times[kind] = statistics.median(a.elapsed_time(b) for a, b in reps_t) / launches
+                del g
+            lat = {"encode": [], "decode": []}
             for _ in range(reps):
-                flush()
-                a, b = ev(), ev()
-                a.record(stream)
-                Q.quantize(x, out=e, group_s=gs)
-                b.record(stream)
-                te.append((a, b))
-                flush()
-                a, b = ev(), ev()
-                a.record(stream)
-                Q.dequantize(e, out=xhat)
-                b.record(stream)
-                td.append((a, b))
+                for kind in ("encode", "decode"):
+                    flush()
+                    a, b = ev(), ev()
+                    a.record(stream)
+                    if kind == "encode":
+                        Q.quantize(xs[0], out=es[0], group_s=gs)
+                    else:
+                        Q.dequantize(es[0], out=hs[0])
+                    b.record(stream)
+                    lat[kind].append((a, b))
             torch.cuda.synchronize()
             assert Q.device_status() == 0
-            ms_e = statistics.median(a.elapsed_time(b) for a, b in te)
-            ms_d = statistics.median(a.elapsed_time(b) for a, b in td)
+            n = rows * K
             enc_b = n * encode_bytes_per_elem(gs, GROUP_Q)
             dec_b = n * (0.5 + 1.0 / gs + 2.0 / GROUP_Q + 2.0)
-            res.append({"elements": n, "shape": [rows, K], "group_s": gs,
+            ms_e, ms_d = times["encode"], times["decode"]
+            res.append({"elements": n, "shape": [rows, K], "group_s": gs, "launches": launches,
                         "encode_us": ms_e * 1e3, "encode_gbs": enc_b / ms_e / 1e6,
                         "encode_frac": enc_b / ms_e / 1e6 / hbm_peak,
                         "decode_us": ms_d * 1e3, "decode_gbs": dec_b / ms_d / 1e6,
                         "decode_frac": dec_b / ms_d / 1e6 / hbm_peak,
+                        "encode_latency_us": statistics.median(a.elapsed_time(b) for a, b in lat["encode"]) * 1e3,
+                        "decode_latency_us": statistics.median(a.elapsed_time(b) for a, b in lat["decode"]) * 1e3,
                         "note": "latency-bound (2.7 MB moved per launch)" if rows == 256 else "hbm-bound"})
-            del e
-    del x_all
+        del e_all
+    del x_all, xhat_all
+    res.sort(key=lambda r: (r["elements"], r["group_s"]))
     return {"workload": "quantize+LZS encode / decode sweep, fp16 mixture 89% Laplace(0,0.05), "
                         "10% N(0,0.3), 1% U(-8,8)",
-            "kernels": "quantize_sym_kernel / dequantize kernel", "peak_gbs": hbm_peak,
+            "kernels": "quantize_sym_kernel / dequantize_kernel", "peak_gbs": hbm_peak,
             "encode_bytes": "2 + 1/2 + 1/G_s + 2/64 B per element",
             "decode_bytes": "1/2 + 1/G_s + 2/64 + 2 B per element",
-            "l2": f"{L2_FLUSH_BYTES >> 20} MiB read before every repetition; median of {reps}",
+            "l2": "throughput: back-to-back launches (one CUDA graph, replayed 3 times, median) over "
+                  "distinct slices, 256 MB of inputs per cycle (> 129 MB L2); latency: one launch after "
+                  f"a 256 MiB read of another buffer, median of {reps}",
             "sizes": res}
 
 
