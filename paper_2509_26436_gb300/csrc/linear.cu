@@ -1288,7 +1288,8 @@ cudaError_t launch_tc(const CUtensorMap &ta, const CUtensorMap &tw, const GemmAr
     }
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
-    const int grid = args.num_tiles < num_sms() ? args.num_tiles : num_sms();
+    int grid = args.num_tiles < num_sms() ? args.num_tiles : num_sms();
+    if (args.split > 1 && args.ls == 0 && args.full_tiles == 0) grid = args.tail_tiles * args.split;
     kern<<<grid, kThreads, smem, s>>>(ta, tw, args);
     return cudaGetLastError();
 }
@@ -1370,7 +1371,9 @@ GemmArgs make_args(const LinearWorkspace &ws, int64_t M, int64_t N, int64_t K, c
 // Split of the GEMM's last wave on this device (symmetric, group-64 fast
 // path): when the tiles left after whole waves fill at most half of one,
 // each of them is cut along K into `split` group ranges (at most
-// kMaxTailSplit, at least two groups each) for otherwise idle CTAs.  When
+// kMaxTailSplit, at least two groups each) for otherwise idle CTAs; with
+// fewer tiles than SMs (a first wave that is also the last), every tile is
+// cut that way and the grid has tiles x split CTAs.  When
 // they fill more than half, the last two waves' group iterations are spread
 // evenly over the CTAs (two-wave form), but only where that shortens the
 // critical path by at least kMinStreamSaving group iterations: it costs
@@ -1396,6 +1399,15 @@ void tail_split(int64_t M, int64_t N, int64_t K, int mode, int *tail, int *split
         *tail = static_cast<int>(Ts);
         *split = 2;
         if (ls) *ls = static_cast<int>((U + P - 1) / P);
+        return;
+    }
+    if (T < sms) {  // fewer tiles than SMs: every tile is cut along K for the idle SMs
+        int64_t S = sms / T;
+        if (S > kMaxTailSplit) S = kMaxTailSplit;
+        if (S > G / 2) S = G / 2;
+        if (S < 2) return;
+        *tail = static_cast<int>(T);
+        *split = static_cast<int>(S);
         return;
     }
     if (W < 1 || R == 0) return;

@@ -182,6 +182,33 @@ def test_linear_split_last_wave(Q, M, N, K, out_dtype):
     _tol_check(y[torch.from_numpy(rows).cuda()].float().cpu().numpy(), ref, rabs, K // 64, out_dtype)
 
 
+# Fewer tiles than SMs: every tile is cut along K into up to 4 parts (one
+# CTA each): 2 x 5 tiles of 18 groups (the 256 x 1152 single layer, 4
+# parts), 1 tile of 10 groups (4 parts), 3 x 3 ragged tiles of 5 groups (2
+# parts), 40 tiles of 3 groups (stays whole: parts keep at least two groups).
+SMALL_SHAPES = [(256, 1152, 1152), (100, 200, 640), (300, 520, 320), (1000, 1200, 192)]
+
+
+@pytest.mark.parametrize("out_dtype", ["float16", "bfloat16", "float32"])
+@pytest.mark.parametrize("M,N,K", SMALL_SHAPES)
+def test_linear_split_small_problems(Q, M, N, K, out_dtype):
+    """Split along K of every tile when the problem has fewer tiles than SMs:
+    all outputs against the oracle, with a bias; the prepared-weights call is
+    bit-identical."""
+    xa = inputs.laplace_activations(M, K, seed=9300 + M)
+    xw = inputs.gaussian_weights(N, K, seed=9301 + N)
+    bias = np.random.default_rng(N + 2).normal(0, 0.1, N).astype(np.float16)
+    a = Q.quantize(torch.from_numpy(xa).cuda(), group_s=16)
+    w = Q.encode_weights(torch.from_numpy(xw).cuda(), group_s=16)
+    b = torch.from_numpy(bias).cuda()
+    y = Q.linear(a, w, b, out_dtype=getattr(torch, out_dtype))
+    y_again = Q.linear(a, w, b, out_dtype=getattr(torch, out_dtype), w_prepared=Q.prepare_weights(w))
+    assert Q.device_status() == 0
+    assert torch.equal(y, y_again)
+    ref, rabs = O.linear(O.encode(xa, 64, 16), O.encode(xw, 64, 16), bias, with_abs=True)
+    _tol_check(y.float().cpu().numpy(), ref, rabs, K // 64, out_dtype)
+
+
 # Shapes whose last wave is more than half full, so that the last P + R tiles'
 # group iterations are spread over all CTAs after one wave of whole tiles
 # (two-wave form), with 8-bit codes (exact P_g): 9 x 45 = 405 tiles = 2 x 152
@@ -242,13 +269,17 @@ def test_split_last_wave_launch_count(Q):
     at least 32 group iterations on the critical path; the launch count and
     the workspace report it."""
     sms = torch.cuda.get_device_properties(0).multi_processor_count
-    shapes = SPLIT_SHAPES + [(2048, 4096, 4096), (2048, 4096, 11008), (1100, 4400, 128), (128, 256, 640)]
+    shapes = SPLIT_SHAPES + SMALL_SHAPES + [(2048, 4096, 4096), (2048, 4096, 11008), (1100, 4400, 128),
+                                            (128, 256, 640), (128, 256, 64)]
     for M, N, K in shapes:
         T = -(-M // 128) * -(-N // 256)
         P = min(T, sms)
         W, R = divmod(T, P)
         G = K // 64
-        if W >= 1 and 2 * R > P:
+        if T < sms:
+            split = min(sms // T, 4, G // 2) >= 2
+            part_tiles = T * min(sms // T, 4, G // 2) if split else 0
+        elif W >= 1 and 2 * R > P:
             split, part_tiles = G * (P - R) >= 32 * P, 2 * (P + R)
         else:
             split = W >= 1 and R > 0 and min(P // R, 4, G // 2) >= 2
@@ -493,9 +524,12 @@ def test_prepared_weights_identical(Q, algo, mode):
     prep = Q.prepare_weights(w)
     y0, p0 = Q.linear(a, w, b, algo=ALGOS[algo], partials_group=3)
     y1, p1 = Q.linear(a, w, b, algo=ALGOS[algo], w_prepared=prep, partials_group=3)
+    # without partials the tcgen05 launch cuts these 4 tiles along K (another
+    # summation order): compare like with like
     y2 = Q.linear(a, w, b, algo=ALGOS[algo], w_prepared=prep)   # reusable
+    y3 = Q.linear(a, w, b, algo=ALGOS[algo])
     assert Q.device_status() == 0
-    assert torch.equal(y0, y1) and torch.equal(y0, y2) and torch.equal(p0, p1)
+    assert torch.equal(y0, y1) and torch.equal(y2, y3) and torch.equal(p0, p1)
 
 
 @pytest.mark.parametrize("kind", ["per_row", "wide", "packed"])

@@ -3,9 +3,10 @@
 The persistent GEMM runs P = min(T, SMs) CTAs over T tiles of 128 x 256
 outputs, each a sequence of G 64-wide K groups (Section 4.4, Appendix C).
 When the tiles left after whole waves would leave CTAs idle, the host cuts
-them along K (linear.cu: tail_split) and every CTA role walks the same work
-list (work_items / work_item); tail_combine_kernel adds the parts of a cut
-tile and returns at once for a tail tile that one CTA ran whole.
+them along K (linear.cu: tail_split; with fewer tiles than SMs every tile is
+cut and the grid has tiles x parts CTAs) and every CTA role walks the same
+work list (work_items / work_item); tail_combine_kernel adds the parts of a
+cut tile and returns at once for a tail tile that one CTA ran whole.
 
 This file restates those three pieces of integer arithmetic in Python and
 checks, over a grid of tile counts, SM counts and group counts, that
@@ -30,6 +31,14 @@ MAX_TAIL_SPLIT = 4
 MIN_STREAM_SAVING = 32
 
 
+def grid_size(T, sms, tail, split, ls):
+    """CTAs of the launch: one per tile up to the SM count, or tiles x split
+    when every tile is cut (fewer tiles than SMs)."""
+    if split > 1 and ls == 0 and tail == T:
+        return tail * split
+    return min(T, sms)
+
+
 def tail_split(T, sms, G):
     """(tail_tiles, split, ls) as the host chooses them (symmetric mode)."""
     P = min(T, sms)
@@ -40,6 +49,9 @@ def tail_split(T, sms, G):
         if G * (P - R) < MIN_STREAM_SAVING * P or U >= 1 << 30:
             return 0, 1, 0
         return Ts, 2, (U + P - 1) // P
+    if T < sms:
+        S = min(sms // T, MAX_TAIL_SPLIT, G // 2)
+        return (T, S, 0) if S >= 2 else (0, 1, 0)
     if W < 1 or R == 0:
         return 0, 1, 0
     S = min(P // R, MAX_TAIL_SPLIT, G // 2)
@@ -88,7 +100,8 @@ def combine_skips(tail_index, G, ls):
 
 def check_plan(T, sms, G):
     tail, split, ls = tail_split(T, sms, G)
-    P = min(T, sms)
+    P = grid_size(T, sms, tail, split, ls)
+    assert P <= sms
     cover = {}
     busiest = 0
     for c in range(P):
@@ -124,8 +137,10 @@ def check_plan(T, sms, G):
             ti = tile - (T - tail)
             assert combine_skips(ti, G, ls) == (len(pieces) == 1), f"combine test wrong for tail tile {ti}"
     # the plan's critical path (group iterations of the busiest CTA)
-    W = T // P
-    if split > 1 and ls > 0:
+    W = T // min(T, sms)
+    if split > 1 and ls == 0 and tail == T:
+        assert busiest == -(-G // split)
+    elif split > 1 and ls > 0:
         assert busiest <= (W - 1) * G + ls
         assert busiest <= (W + 1) * G - MIN_STREAM_SAVING
     elif split > 1:
@@ -170,6 +185,11 @@ def test_split_plan_forms_reached_at_152_sms():
     assert split == 2 and ls > 0 and tail == 256
     # a last wave more than half full whose cut would save too little stays whole
     assert plan(2048, 4096, 4096)[1] == 1
+    # fewer tiles than SMs: 256 x 1152 x 1152 (2 x 5 tiles, 18 groups) in 4 parts
+    # each; one tile of 10 groups in 4; one tile of a single group stays whole
+    assert plan(256, 1152, 1152) == (10, 4, 0)
+    assert plan(128, 256, 640) == (1, 4, 0)
+    assert plan(128, 256, 64)[1] == 1
 
 
 def test_split_plan_exhaustive_small():
