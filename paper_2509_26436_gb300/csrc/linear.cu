@@ -226,6 +226,7 @@ static_assert(kEpiWarps * 32 * kRegsEpilogue + 128 * kRegsControl <= kThreads * 
               "register split exceeds the launch allocation");
 constexpr uint32_t kTmemCols = 512;   // two fp32 accumulators of 256 columns
 constexpr int kRasterM = 8;
+constexpr int kRowRasterMaxN = 16;  // see tile_coords
 // Per-row scales (group_q = K): the MMA accumulates kPerRowChunk stages (256
 // of K) into one TMEM accumulator before the epilogue takes it; each such sum
 // is an integer below 256 * 112^2 < 2^22, exact in fp32 and convertible with
@@ -238,6 +239,7 @@ struct GemmArgs {
     int64_t m_pad, n_pad;
     int M, N, G;
     int tiles_m, tiles_n, num_tiles;
+    int raster_m;         // M-tiles per band of the visiting order: kRasterM or 1 (see tile_coords)
     const __half *bias;
     void *y;
     int y_type;
@@ -277,15 +279,24 @@ struct Smem {
     static constexpr int kAlloc = kTotal + 1024;  // slack to align the base to 1024 bytes
 };
 
-// Tile visiting order: bands of kRasterM M-tiles, N-tiles inside a band, so
-// the CTAs resident at one time share few A row-blocks and W column-blocks
-// and both stay in L2.
+// Tile visiting order: bands of RM M-tiles, N-tiles inside a band (M
+// fastest), so the CTAs resident at one time share few A row-blocks and W
+// column-blocks and both stay in L2.  RM is kRasterM, or 1 (whole rows of
+// tiles, one M-tile after the other) for layers at most kRowRasterMaxN
+// tiles wide on the symmetric fast path: there a band of 8 M-tiles holds
+// fewer tiles than one wave of CTAs, so the waves would cut bands and read
+// an A row-block again in the next wave (measured 2.3x A reads for a
+// 12-tile-wide, 192-group layer), while a row keeps each A row-block's
+// consumers in one wave and the whole narrow W stays in L2.  RM is a
+// template argument of the GEMM (a runtime band size measured 1.4% slower
+// on the wide layers); a.raster_m holds it for the combine kernel.
+template <int RM>
 __device__ __forceinline__ void tile_coords(int tile, const GemmArgs &a, int &mt, int &nt)
 {
-    const int band = tile / (kRasterM * a.tiles_n);
-    const int m0 = band * kRasterM;
-    const int gm = min(kRasterM, a.tiles_m - m0);
-    const int r = tile - band * kRasterM * a.tiles_n;
+    const int band = tile / (RM * a.tiles_n);
+    const int m0 = band * RM;
+    const int gm = min(RM, a.tiles_m - m0);
+    const int r = tile - band * RM * a.tiles_n;
     mt = m0 + r % gm;
     nt = r / gm;
 }
@@ -386,12 +397,12 @@ __device__ __forceinline__ float4 add_bias4(const GemmArgs &args, int64_t n, flo
 // acc[c][4h + i] holds output column 16c + tq + i of this warp's slice, rows
 // trow + 16h (low half) and trow + 16h + 8 (high half) of its quarter; the
 // bias is added in fp32, then one rounding to the output type.
-template <int OUT>
+template <int OUT, int RM>
 __device__ __forceinline__ void store_tile_sym(const GemmArgs &args, int tile, int quarter, int slot, int trow,
                                                int tq, const uint64_t (&acc)[4][8])
 {
     int mt, nt;
-    tile_coords(tile, args, mt, nt);
+    tile_coords<RM>(tile, args, mt, nt);
 #pragma unroll
     for (int h = 0; h < 2; ++h)
 #pragma unroll
@@ -504,7 +515,7 @@ __device__ __forceinline__ void lds_b64x2(uint32_t addr, uint64_t &a, uint64_t &
     asm volatile("ld.shared.v2.b64 {%0, %1}, [%2];" : "=l"(a), "=l"(b) : "r"(addr) : "memory");
 }
 
-template <int MODE, int OUT, bool DUMP, bool PERROW>
+template <int MODE, int OUT, bool DUMP, bool PERROW, int RM = kRasterM>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tmap_a,
                         const __grid_constant__ CUtensorMap tmap_w, const GemmArgs args)
@@ -573,7 +584,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int k = 0; k < n_items && ok; ++k) {
                 const WorkItem wi = work_item(args, k);
                 int mt, nt;
-                tile_coords(wi.tile, args, mt, nt);
+                tile_coords<RM>(wi.tile, args, mt, nt);
                 for (int g = wi.g0; g < wi.g1; ++g, ++it) {
                     const int s = it % kStages;
                     if (it >= kStages &&
@@ -613,7 +624,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int k = 0; k < n_items && ok; ++k) {
                 const WorkItem wi = work_item(args, k);
                 int mt, nt;
-                tile_coords(wi.tile, args, mt, nt);
+                tile_coords<RM>(wi.tile, args, mt, nt);
                 for (int g = wi.g0; g < wi.g1; ++g, ++it) {
                     const int ss = it % S;
                     if (it >= S && !mbar_wait_bounded(side_empty_bar(ss), ((it / S) - 1) & 1, abort_flag,
@@ -752,7 +763,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 if (!ok) break;
                 int mt, nt;
-                tile_coords(tile, args, mt, nt);
+                tile_coords<RM>(tile, args, mt, nt);
 #pragma unroll
                 for (int h = 0; h < 2; ++h)
 #pragma unroll
@@ -852,7 +863,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                                         static_cast<uint32_t>(acc64[c][2 * j + 1] >> 32));
                     continue;
                 }
-                store_tile_sym<OUT>(args, wi.tile, quarter, slot, trow, tq, acc64);
+                store_tile_sym<OUT, RM>(args, wi.tile, quarter, slot, trow, tq, acc64);
             }
         } else {
             float2 acc[2][16];
@@ -913,7 +924,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 float2 p = make_float2(__uint_as_float(r[8 * h + 2 * i]), __uint_as_float(r[8 * h + 2 * i + 1]));
                                 if (DUMP && g == args.partials_group) {
                                     int mt, nt;
-                                    tile_coords(tile, args, mt, nt);
+                                    tile_coords<RM>(tile, args, mt, nt);
                                     const int64_t m = static_cast<int64_t>(mt) * BM + quarter * 32 + 16 * h + trow;
                                     const int64_t n = static_cast<int64_t>(nt) * BN + slot * kColsPerWarp + 16 * chunk + tq + i;
                                     if (n < args.N) {
@@ -942,7 +953,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 if (!ok) break;
                 int mt, nt;
-                tile_coords(tile, args, mt, nt);
+                tile_coords<RM>(tile, args, mt, nt);
                 // ---- store: 4 rows x 4 chunks of 4 consecutive columns per thread ----
 #pragma unroll
                 for (int h = 0; h < 2; ++h)
@@ -1014,7 +1025,10 @@ __global__ void __launch_bounds__(kEpiWarps * 32) tail_combine_kernel(const __gr
         }
     }
     int mt, nt;
-    tile_coords(args.full_tiles + tail, args, mt, nt);
+    if (args.raster_m == 1)
+        tile_coords<1>(args.full_tiles + tail, args, mt, nt);
+    else
+        tile_coords<kRasterM>(args.full_tiles + tail, args, mt, nt);
     const int quarter = warp & 3, slot = warp >> 2, trow = lane >> 2, tq = 4 * (lane & 3);
     const int64_t n = static_cast<int64_t>(nt) * BN + slot * kColsPerWarp + 16 * c + tq;
     if (n >= args.N) return;
@@ -1282,6 +1296,9 @@ cudaError_t launch_tc(const CUtensorMap &ta, const CUtensorMap &tw, const GemmAr
     auto kern = args.partials ? gemm_tcgen05_kernel<MODE, OUT, true, false>
                               : gemm_tcgen05_kernel<MODE, OUT, false, false>;
     if constexpr (MODE == QUARTZ_SYMMETRIC) {
+        if (!args.partials && !args.per_row && args.raster_m == 1) kern = gemm_tcgen05_kernel<MODE, OUT, false, false, 1>;
+    }
+    if constexpr (MODE == QUARTZ_SYMMETRIC) {
         if (args.per_row)
             kern = args.partials ? gemm_tcgen05_kernel<MODE, OUT, true, true>
                                  : gemm_tcgen05_kernel<MODE, OUT, false, true>;
@@ -1356,6 +1373,7 @@ GemmArgs make_args(const LinearWorkspace &ws, int64_t M, int64_t N, int64_t K, c
     a.tiles_n = static_cast<int>((N + BN - 1) / BN);
     a.tiles_m = static_cast<int>((M + BM - 1) / BM);
     a.num_tiles = a.tiles_m * a.tiles_n;
+    a.raster_m = kRasterM;
     a.full_tiles = a.num_tiles;
     a.bias = static_cast<const __half *>(bias);
     a.y = y;
@@ -1538,6 +1556,7 @@ cudaError_t launch_gemm_tcgen05(const LinearWorkspace &ws, int64_t M, int64_t N,
     GemmArgs args = make_args(ws, M, N, K, bias, y, y_type, partials, partials_group, dev_err);
     args.per_row = per_row ? 1 : 0;
     args.wide = wide ? 1 : 0;
+    if (mode == QUARTZ_SYMMETRIC && !partials && !per_row && args.tiles_n <= kRowRasterMaxN) args.raster_m = 1;
     int tail = 0, split = 1, ls = 0;  // the workspace's split must still match this device's grid
     if (mode == QUARTZ_SYMMETRIC && !partials && !per_row && ws.tail_split > 1 && ws.tail_part)
         tail_split(M, N, K, mode, &tail, &split, &ls);
