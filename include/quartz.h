@@ -158,9 +158,14 @@ int32_t quartz_dequantize(const quartz_encoded_t *e, void *x_hat_f16, void *stre
 /* Workspace bytes quartz_linear needs for an [M, K] x [N, K]^T product
  * (the operands expanded to the tensor-core input format, transposed group
  * scales and, where the symmetric tcgen05 GEMM splits its last wave of
- * tiles along K, the fp32 partial tiles of that wave).  The last part
- * depends on the current device's SM count: query it on the device that
- * will run the call.  Returns 0 for invalid arguments. */
+ * tiles along K, the fp32 partial tiles of that wave: 128 KB per part and
+ * tile, up to 4 parts per tail tile; when the last two waves are spread
+ * over all SMs, 2 parts are reserved for each of their tiles although only
+ * the tiles cut by a CTA's range boundary, fewer than the SM count, use
+ * them, e.g. 64 MiB of which at most 37.75 MiB is written for a
+ * 2048 x 11008 -> 4096 layer).  The last part depends on the current
+ * device's SM count: query it on the device that will run the call.
+ * Returns 0 for invalid arguments. */
 size_t quartz_linear_workspace_size(int64_t M, int64_t N, int64_t K, const quartz_params_t *p);
 
 /* Kernels one quartz_linear_ex call with these sizes, algorithm and
