@@ -221,60 +221,84 @@ __device__ __forceinline__ UnitCodes encode_unit_sym_scaled(const uint4 lo, cons
 
 // The LLM variant of Section 5 on one unit (symmetric): Eq. 1 with 32767
 // levels (16-bit codes), then Eq. 2 straight to 4 bits with FLAG =
-// max(29 - clz(m), 0) in 0..12, m the OR of the subgroup's |q|.  The same
-// binary32 operations as the per-chunk encoder, so the codes, FLAGs and
+// max(29 - clz(m), 0) in 0..12, m the OR of the subgroup's |q|.  The OR has
+// the bit length of the subgroup's largest |q|, and |q| = rne(min(|x| r,
+// 32767)) grows with |x|, so the FLAG comes from the subgroup's largest
+// |x| (one conversion per subgroup, as in the 8-bit encoder) and each code
+// is bits F .. F+2 of |q|, taken from the 1.5 * 2^23 rounding sum, with the
+// sign of x applied in 4-bit two's complement.  The binary32 operations
+// that produce q are those of the per-chunk encoder, so codes, FLAGs and
 // scales are bit-identical to quartz_quantize's.  All 32 lanes call it
 // together (4 lanes per group).
+__device__ __forceinline__ int lzs_flag_wide(float amax_sub, float r)
+{
+    const int qmax = min(__float2int_rn(__fmul_rn(amax_sub, r)), 32767);
+    return max(29 - __clz(qmax), 0);
+}
+
+// Codes of 8 elements (four fp16 pairs `w`, sign-cleared copies `a`) for
+// 16-bit stage-1 codes: |q| = rne(|x| r) (capped at 32767 when CAP), c =
+// sgn(x) (|q| >> flag), element k in bits 4k..4k+3.
+template <bool CAP>
+__device__ __forceinline__ uint32_t lzs_word8_wide(const uint32_t *w, const uint32_t *a, float r, int flag)
+{
+    uint32_t u[4][2];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const float2 f = __half22float2(*reinterpret_cast<const __half2 *>(&a[i]));
+        float2 t = mul2_rn(f, make_float2(r, r));
+        if (CAP) {
+            t.x = fminf(t.x, 32767.0f);
+            t.y = fminf(t.y, 32767.0f);
+        }
+        // scalar additions (see lzs_word8); the low 22 bits of the sum are
+        // |q|, and |q| >> flag <= 7 lands in the low byte
+        u[i][0] = __float_as_uint(__fadd_rn(t.x, kRoundAddend)) >> flag;
+        u[i][1] = __float_as_uint(__fadd_rn(t.y, kRoundAddend)) >> flag;
+    }
+    const uint32_t ev = prmt(prmt(u[0][0], u[1][0], 0x0040u), prmt(u[2][0], u[3][0], 0x0040u), 0x5410u);
+    const uint32_t od = prmt(prmt(u[0][1], u[1][1], 0x0040u), prmt(u[2][1], u[3][1], 0x0040u), 0x5410u);
+    const uint32_t sev = prmt(prmt(w[0], w[1], 0x00D9u), prmt(w[2], w[3], 0x00D9u), 0x5410u);
+    const uint32_t sod = prmt(prmt(w[0], w[1], 0x00FBu), prmt(w[2], w[3], 0x00FBu), 0x5410u);
+    const uint32_t cev = signed_nibbles(ev & 0x07070707u, sev);
+    const uint32_t cod = signed_nibbles(od & 0x07070707u, sod);
+    return cev | (cod << 4);
+}
+
 template <int GS>
 __device__ __forceinline__ UnitCodes encode_unit_wide(const uint4 lo, const uint4 hi)
 {
     const uint32_t w[8] = {lo.x, lo.y, lo.z, lo.w, hi.x, hi.y, hi.z, hi.w};
-    float x[16];
+    uint32_t a[8];
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-        const float2 f = __half22float2(*reinterpret_cast<const __half2 *>(&w[i]));
-        x[2 * i] = f.x;
-        x[2 * i + 1] = f.y;
-    }
-    float amax = 0.f;
-#pragma unroll
-    for (int i = 0; i < 16; ++i) amax = fmaxf(amax, fabsf(x[i]));
-    amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, 1));
-    amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, 2));
+    for (int i = 0; i < 8; ++i) a[i] = w[i] & 0x7FFF7FFFu;
+    __half2 m0 = __hmax2(__hmax2(*reinterpret_cast<const __half2 *>(&a[0]), *reinterpret_cast<const __half2 *>(&a[1])),
+                         __hmax2(*reinterpret_cast<const __half2 *>(&a[2]), *reinterpret_cast<const __half2 *>(&a[3])));
+    __half2 m1 = __hmax2(__hmax2(*reinterpret_cast<const __half2 *>(&a[4]), *reinterpret_cast<const __half2 *>(&a[5])),
+                         __hmax2(*reinterpret_cast<const __half2 *>(&a[6]), *reinterpret_cast<const __half2 *>(&a[7])));
+    const float2 f0 = __half22float2(m0), f1 = __half22float2(m1);
+    const float sub0 = fmaxf(f0.x, f0.y), sub1 = fmaxf(f1.x, f1.y);
+    const float unit_max = fmaxf(sub0, sub1);
+    const float pair_max = fmaxf(unit_max, __shfl_xor_sync(0xffffffffu, unit_max, 1));
+    const float amax = fmaxf(pair_max, __shfl_xor_sync(0xffffffffu, pair_max, 2));
+
     UnitCodes u;
     u.s16 = __float2half_rn(__fdiv_rn(amax, 32767.0f));
     const float s = __half2float(u.s16);
     const float r = (s > 0.f) ? __frcp_rn(s) : 0.f;
-
-    int q[16];
-    uint32_t m0 = 0, m1 = 0;
-#pragma unroll
-    for (int i = 0; i < 16; ++i) {
-        const float t = fminf(fmaxf(__fmul_rn(x[i], r), -65536.0f), 65536.0f);
-        q[i] = min(max(__float2int_rn(t), -32767), 32767);
-        if (i < 8)
-            m0 |= static_cast<uint32_t>(abs(q[i]));
-        else
-            m1 |= static_cast<uint32_t>(abs(q[i]));
+    if (GS == 8) {
+        u.flag0 = lzs_flag_wide(sub0, r);
+        u.flag1 = lzs_flag_wide(sub1, r);
+    } else {
+        const float m = GS == 16 ? unit_max : GS == 32 ? pair_max : amax;
+        u.flag0 = u.flag1 = lzs_flag_wide(m, r);
     }
-    if (GS >= 16) {
-        m0 |= m1;
-        if (GS >= 32) m0 |= __shfl_xor_sync(0xffffffffu, m0, 1);
-        if (GS >= 64) m0 |= __shfl_xor_sync(0xffffffffu, m0, 2);
-        m1 = m0;
-    }
-    u.flag0 = max(29 - __clz(static_cast<int>(m0)), 0);
-    u.flag1 = max(29 - __clz(static_cast<int>(m1)), 0);
-    u.c0 = u.c1 = 0;
-#pragma unroll
-    for (int i = 0; i < 16; ++i) {
-        const int f = i < 8 ? u.flag0 : u.flag1;
-        const int mag = abs(q[i]) >> f;  // truncation toward zero
-        const uint32_t c = static_cast<uint32_t>(q[i] < 0 ? -mag : mag) & 0xFu;
-        if (i < 8)
-            u.c0 |= c << (4 * i);
-        else
-            u.c1 |= c << (4 * (i - 8));
+    if (__float2int_rn(__fmul_rn(amax, r)) > 32767) {  // only when the fp16 scale rounded down
+        u.c0 = lzs_word8_wide<true>(w, a, r, u.flag0);
+        u.c1 = lzs_word8_wide<true>(w + 4, a + 4, r, u.flag1);
+    } else {
+        u.c0 = lzs_word8_wide<false>(w, a, r, u.flag0);
+        u.c1 = lzs_word8_wide<false>(w + 4, a + 4, r, u.flag1);
     }
     u.flag_next = 0;
     if (GS >= 16) u.flag_next = __shfl_down_sync(0xffffffffu, u.flag0, kUnitsPerSub<GS>());
