@@ -189,6 +189,7 @@ static_assert(kAttnThreads * 33 * 4 <= kAttnDynSmem, "slot reduction fits the co
 template <int GS>
 __global__ void __launch_bounds__(kAttnThreads, 5) attn_decode_kernel(const __grid_constant__ AttnArgs a)
 {
+    griddep_wait();
     constexpr int S = kD / GS;            // subgroups per row
     constexpr int kWordsPerSub = GS / 8;  // code words per subgroup
     extern __shared__ __align__(128) uint8_t s_ring[];  // [kStages][K, V][kTileBytes]
@@ -380,6 +381,7 @@ __global__ void __launch_bounds__(kAttnThreads, 5) attn_decode_kernel(const __gr
 template <int OUT>
 __global__ void __launch_bounds__(kD) attn_combine_kernel(const float *__restrict__ part, int n_split, void *out)
 {
+    griddep_wait();
     const int64_t bh = blockIdx.x;
     const int d = threadIdx.x;
     const float *p = part + bh * n_split * kPartStride;
@@ -435,7 +437,7 @@ cudaError_t launch_decode(int64_t BH, AttnArgs &a, cudaStream_t s)
     if (sms <= 0) sms = 1;
     a.n_split = attn_splits(BH, a.L, static_cast<int64_t>(sms) * occ, &a.chunk);
     const dim3 grid(static_cast<unsigned>(a.n_split), static_cast<unsigned>(BH));
-    attn_decode_kernel<GS><<<grid, kAttnThreads, kAttnDynSmem, s>>>(a);
+    launch_pdl(attn_decode_kernel<GS>, dim3(grid), dim3(kAttnThreads), kAttnDynSmem, s, a);
     return cudaGetLastError();
 }
 
@@ -480,9 +482,9 @@ cudaError_t launch_attention_decode(const quartz_encoded_t *q, const quartz_enco
     }
     if (e != cudaSuccess) return e;
     const unsigned cb = static_cast<unsigned>(BH);
-    if (o_type == QUARTZ_OUT_F16) attn_combine_kernel<QUARTZ_OUT_F16><<<cb, kD, 0, s>>>(a.part, a.n_split, o);
-    else if (o_type == QUARTZ_OUT_BF16) attn_combine_kernel<QUARTZ_OUT_BF16><<<cb, kD, 0, s>>>(a.part, a.n_split, o);
-    else attn_combine_kernel<QUARTZ_OUT_F32><<<cb, kD, 0, s>>>(a.part, a.n_split, o);
+    if (o_type == QUARTZ_OUT_F16) launch_pdl(attn_combine_kernel<QUARTZ_OUT_F16>, dim3(cb), dim3(kD), 0, s, a.part, a.n_split, o);
+    else if (o_type == QUARTZ_OUT_BF16) launch_pdl(attn_combine_kernel<QUARTZ_OUT_BF16>, dim3(cb), dim3(kD), 0, s, a.part, a.n_split, o);
+    else launch_pdl(attn_combine_kernel<QUARTZ_OUT_F32>, dim3(cb), dim3(kD), 0, s, a.part, a.n_split, o);
     return cudaGetLastError();
 }
 

@@ -200,6 +200,7 @@ __device__ __forceinline__ void run_side(const SideJob &j, int64_t t, int G, int
 template <int GS, bool WIDE>
 __global__ void __launch_bounds__(kPrepThreads) prep_kernel(const __grid_constant__ PrepArgs args)
 {
+    griddep_wait();
     const int64_t bid = blockIdx.x;
     if (bid < args.block_end[0]) {
         run_expand<GS, WIDE>(args.ex_a, bid * (kPrepThreads * kExpandPairs) + threadIdx.x);
@@ -539,6 +540,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tmap_a,
                         const __grid_constant__ CUtensorMap tmap_w, const GemmArgs args)
 {
+    griddep_wait();
     constexpr int NSIDE = (MODE == QUARTZ_ASYMMETRIC) ? 3 : 1;
     using L = Smem<NSIDE>;
     extern __shared__ uint8_t smem_raw[];
@@ -1020,6 +1022,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 template <int OUT>
 __global__ void __launch_bounds__(kEpiWarps * 32) tail_combine_kernel(const __grid_constant__ GemmArgs args)
 {
+    griddep_wait();
     constexpr int T = kEpiWarps * 32;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int tail = blockIdx.x >> 2, c = blockIdx.x & 3;
@@ -1074,6 +1077,7 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const __nv_fp8_e4m3 *__r
                                                         const __nv_fp8_e4m3 *__restrict__ w_op,
                                                         const GemmArgs args, int K)
 {
+    griddep_wait();
     __shared__ int16_t sa[64][kGroupQ + 2];
     __shared__ int16_t sw[64][kGroupQ + 2];
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
@@ -1156,6 +1160,7 @@ __global__ void __launch_bounds__(256) gemm_shift_kernel(const uint32_t *__restr
                                                          const uint8_t *__restrict__ w_flags,
                                                          const GemmArgs args, int K, int a_packed, int w_packed)
 {
+    griddep_wait();
     constexpr int kSub = kGroupQ / GS;            // subgroups per group
     constexpr int kWordsPerSub = GS / 4;          // int8x4 words per subgroup
     __shared__ uint32_t sa[64][2 * kGroupQ / 8 + 1];
@@ -1326,7 +1331,7 @@ cudaError_t launch_tc(const CUtensorMap &ta, const CUtensorMap &tw, const GemmAr
     if (e != cudaSuccess) return e;
     int grid = args.num_tiles < num_sms() ? args.num_tiles : num_sms();
     if (args.split > 1 && args.ls == 0 && args.full_tiles == 0) grid = args.tail_tiles * args.split;
-    kern<<<grid, kThreads, smem, s>>>(ta, tw, args);
+    launch_pdl(kern, dim3(grid), dim3(kThreads), smem, s, ta, tw, args);
     return cudaGetLastError();
 }
 
@@ -1345,9 +1350,9 @@ cudaError_t launch_tail_combine(const GemmArgs &args, int y_type, cudaStream_t s
 {
     const unsigned grid = static_cast<unsigned>(args.tail_tiles) * 4;
     switch (y_type) {
-        case QUARTZ_OUT_F16: tail_combine_kernel<QUARTZ_OUT_F16><<<grid, kEpiWarps * 32, 0, s>>>(args); break;
-        case QUARTZ_OUT_BF16: tail_combine_kernel<QUARTZ_OUT_BF16><<<grid, kEpiWarps * 32, 0, s>>>(args); break;
-        default: tail_combine_kernel<QUARTZ_OUT_F32><<<grid, kEpiWarps * 32, 0, s>>>(args); break;
+        case QUARTZ_OUT_F16: launch_pdl(tail_combine_kernel<QUARTZ_OUT_F16>, dim3(grid), dim3(kEpiWarps * 32), 0, s, args); break;
+        case QUARTZ_OUT_BF16: launch_pdl(tail_combine_kernel<QUARTZ_OUT_BF16>, dim3(grid), dim3(kEpiWarps * 32), 0, s, args); break;
+        default: launch_pdl(tail_combine_kernel<QUARTZ_OUT_F32>, dim3(grid), dim3(kEpiWarps * 32), 0, s, args); break;
     }
     return cudaGetLastError();
 }
@@ -1356,7 +1361,7 @@ template <int MODE, int OUT>
 cudaError_t launch_simt(const LinearWorkspace &ws, const GemmArgs &args, int K, cudaStream_t s)
 {
     dim3 grid(static_cast<unsigned>((args.N + 63) / 64), static_cast<unsigned>((args.M + 63) / 64));
-    gemm_simt_kernel<MODE, OUT><<<grid, 256, 0, s>>>(static_cast<const __nv_fp8_e4m3 *>(ws.a_op),
+    launch_pdl(gemm_simt_kernel<MODE, OUT>, dim3(grid), dim3(256), 0, s, static_cast<const __nv_fp8_e4m3 *>(ws.a_op),
                                                      static_cast<const __nv_fp8_e4m3 *>(ws.w_op), args, K);
     return cudaGetLastError();
 }
@@ -1547,18 +1552,18 @@ cudaError_t launch_prepare(const quartz_encoded_t *a, const quartz_encoded_t *w,
     const unsigned blocks = static_cast<unsigned>(acc);
     if (w->p.code_bits == 16) {  // 16-bit stage-1 codes: E5M2 operands
         switch (w->p.group_s) {
-            case 8: prep_kernel<8, true><<<blocks, kPrepThreads, 0, s>>>(p); break;
-            case 16: prep_kernel<16, true><<<blocks, kPrepThreads, 0, s>>>(p); break;
-            case 32: prep_kernel<32, true><<<blocks, kPrepThreads, 0, s>>>(p); break;
-            default: prep_kernel<64, true><<<blocks, kPrepThreads, 0, s>>>(p); break;
+            case 8: launch_pdl(prep_kernel<8, true>, dim3(blocks), dim3(kPrepThreads), 0, s, p); break;
+            case 16: launch_pdl(prep_kernel<16, true>, dim3(blocks), dim3(kPrepThreads), 0, s, p); break;
+            case 32: launch_pdl(prep_kernel<32, true>, dim3(blocks), dim3(kPrepThreads), 0, s, p); break;
+            default: launch_pdl(prep_kernel<64, true>, dim3(blocks), dim3(kPrepThreads), 0, s, p); break;
         }
         return cudaGetLastError();
     }
     switch (w->p.group_s) {
-        case 8: prep_kernel<8, false><<<blocks, kPrepThreads, 0, s>>>(p); break;
-        case 16: prep_kernel<16, false><<<blocks, kPrepThreads, 0, s>>>(p); break;
-        case 32: prep_kernel<32, false><<<blocks, kPrepThreads, 0, s>>>(p); break;
-        default: prep_kernel<64, false><<<blocks, kPrepThreads, 0, s>>>(p); break;
+        case 8: launch_pdl(prep_kernel<8, false>, dim3(blocks), dim3(kPrepThreads), 0, s, p); break;
+        case 16: launch_pdl(prep_kernel<16, false>, dim3(blocks), dim3(kPrepThreads), 0, s, p); break;
+        case 32: launch_pdl(prep_kernel<32, false>, dim3(blocks), dim3(kPrepThreads), 0, s, p); break;
+        default: launch_pdl(prep_kernel<64, false>, dim3(blocks), dim3(kPrepThreads), 0, s, p); break;
     }
     return cudaGetLastError();
 }
@@ -1610,7 +1615,7 @@ cudaError_t launch_shift(const quartz_encoded_t *a, const quartz_encoded_t *w, c
                          cudaStream_t s)
 {
     dim3 grid(static_cast<unsigned>((args.N + 63) / 64), static_cast<unsigned>((args.M + 63) / 64));
-    gemm_shift_kernel<GS, MODE, OUT, WIDE><<<grid, 256, 0, s>>>(
+    launch_pdl(gemm_shift_kernel<GS, MODE, OUT, WIDE>, dim3(grid), dim3(256), 0, s, 
         reinterpret_cast<const uint32_t *>(a->codes), a->flags, reinterpret_cast<const uint32_t *>(w->codes),
         w->flags, args, static_cast<int>(a->K), a->p.flag_bits == 4, w->p.flag_bits == 4);
     return cudaGetLastError();

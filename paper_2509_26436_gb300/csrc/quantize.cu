@@ -342,6 +342,7 @@ __global__ void __launch_bounds__(kThreads) quantize_sym_kernel(const uint4 *__r
                                                                 uint8_t *__restrict__ flags,
                                                                 __half *__restrict__ scales, int packed)
 {
+    griddep_wait();
     const int lane = threadIdx.x & 31;
     const int64_t base = static_cast<int64_t>(blockIdx.x) * (kThreads * kUnitsPerThread) + threadIdx.x;
     uint4 raw[kUnitsPerThread][2];
@@ -373,6 +374,7 @@ __global__ void __launch_bounds__(kThreads) quantize_row_sym_kernel(const uint4 
                                                                     uint8_t *__restrict__ flags,
                                                                     __half *__restrict__ scales, int packed)
 {
+    griddep_wait();
     __shared__ float warp_max[kThreads / 32];
     const int lane = threadIdx.x & 31;
     const int64_t row = blockIdx.x;
@@ -431,6 +433,7 @@ __global__ void __launch_bounds__(kThreads) encode_operand_kernel(
     uint4 *__restrict__ a_op, float *__restrict__ a_side, uint2 *__restrict__ codes,
     uint8_t *__restrict__ flags, __half *__restrict__ scales, int packed)
 {
+    griddep_wait();
     const int lane = threadIdx.x & 31;
     const int64_t base = static_cast<int64_t>(blockIdx.x) * (kThreads * kUnitsPerThread) + threadIdx.x;
     uint4 raw[kUnitsPerThread][2];
@@ -582,6 +585,7 @@ __global__ void __launch_bounds__(kThreads) quantize_kernel(const uint4 *__restr
                                                             int8_t *__restrict__ zeros,
                                                             int32_t *__restrict__ gsum, int packed)
 {
+    griddep_wait();
     const int lane = threadIdx.x & 31;
     const int64_t base = static_cast<int64_t>(blockIdx.x) * (kThreads * kChunksPerThread) + threadIdx.x;
     uint4 raw[kChunksPerThread];
@@ -609,6 +613,7 @@ __global__ void __launch_bounds__(kThreads) kv_append_kernel(const uint4 *__rest
                                                              uint8_t *__restrict__ flags,
                                                              __half *__restrict__ scales, int packed)
 {
+    griddep_wait();
     const int lane = threadIdx.x & 31;
     const int64_t base = static_cast<int64_t>(blockIdx.x) * (kThreads * kChunksPerThread) + threadIdx.x;
     uint4 raw[kChunksPerThread];
@@ -645,6 +650,7 @@ __global__ void __launch_bounds__(kThreads) dequantize_kernel(
     const __half *__restrict__ scales, const int8_t *__restrict__ zeros, int64_t group_q,
     int packed, int64_t n_chunks, uint4 *__restrict__ out)
 {
+    griddep_wait();
     constexpr int kSubShift = GS == 8 ? 3 : GS == 16 ? 4 : GS == 32 ? 5 : 6;
     const int64_t base = static_cast<int64_t>(blockIdx.x) * (kThreads * kDeqChunksPerThread) + threadIdx.x;
     uint32_t word[kDeqChunksPerThread];
@@ -689,7 +695,7 @@ cudaError_t launch_q(const void *x, const quartz_encoded_t *e, cudaStream_t s)
         const int64_t n_units = e->rows * e->K / 16;
         const int64_t per_block = kThreads * kUnitsPerThread;
         const int64_t blocks = (n_units + per_block - 1) / per_block;
-        quantize_sym_kernel<GS, WIDE><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(
+        launch_pdl(quantize_sym_kernel<GS, WIDE>, dim3(static_cast<unsigned>(blocks)), dim3(kThreads), 0, s, 
             static_cast<const uint4 *>(x), n_units, reinterpret_cast<uint2 *>(e->codes), e->flags,
             reinterpret_cast<__half *>(e->scales), e->p.flag_bits == 4);
         return cudaGetLastError();
@@ -697,7 +703,7 @@ cudaError_t launch_q(const void *x, const quartz_encoded_t *e, cudaStream_t s)
         const int64_t n_chunks = e->rows * e->K / 8;
         const int64_t per_block = kThreads * kChunksPerThread;
         const int64_t blocks = (n_chunks + per_block - 1) / per_block;
-        quantize_kernel<GS, MODE><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(
+        launch_pdl(quantize_kernel<GS, MODE>, dim3(static_cast<unsigned>(blocks)), dim3(kThreads), 0, s, 
             static_cast<const uint4 *>(x), n_chunks, reinterpret_cast<uint32_t *>(e->codes), e->flags,
             reinterpret_cast<__half *>(e->scales), e->zeros, e->gsum, e->p.flag_bits == 4);
         return cudaGetLastError();
@@ -729,7 +735,7 @@ template <int GS>
 cudaError_t launch_row(const void *x, const quartz_encoded_t *e, int use_static, unsigned short s16,
                        cudaStream_t s)
 {
-    quantize_row_sym_kernel<GS><<<static_cast<unsigned>(e->rows), kThreads, 0, s>>>(
+    launch_pdl(quantize_row_sym_kernel<GS>, dim3(static_cast<unsigned>(e->rows)), dim3(kThreads), 0, s, 
         static_cast<const uint4 *>(x), e->K, e->p.group_q, use_static, s16, reinterpret_cast<uint2 *>(e->codes),
         e->flags, reinterpret_cast<__half *>(e->scales), e->p.flag_bits == 4);
     return cudaGetLastError();
@@ -761,10 +767,10 @@ cudaError_t launch_kv_append(const void *x, int64_t BH, int64_t T, const quartz_
     __half *scales = reinterpret_cast<__half *>(cache->scales);
     const int packed = cache->p.flag_bits == 4;
     switch (cache->p.group_s) {
-        case 8: kv_append_kernel<8><<<blocks, kThreads, 0, s>>>(xv, n_chunks, cpr, T, L_max, t0, codes, cache->flags, scales, packed); break;
-        case 16: kv_append_kernel<16><<<blocks, kThreads, 0, s>>>(xv, n_chunks, cpr, T, L_max, t0, codes, cache->flags, scales, packed); break;
-        case 32: kv_append_kernel<32><<<blocks, kThreads, 0, s>>>(xv, n_chunks, cpr, T, L_max, t0, codes, cache->flags, scales, packed); break;
-        default: kv_append_kernel<64><<<blocks, kThreads, 0, s>>>(xv, n_chunks, cpr, T, L_max, t0, codes, cache->flags, scales, packed); break;
+        case 8: launch_pdl(kv_append_kernel<8>, dim3(blocks), dim3(kThreads), 0, s, xv, n_chunks, cpr, T, L_max, t0, codes, cache->flags, scales, packed); break;
+        case 16: launch_pdl(kv_append_kernel<16>, dim3(blocks), dim3(kThreads), 0, s, xv, n_chunks, cpr, T, L_max, t0, codes, cache->flags, scales, packed); break;
+        case 32: launch_pdl(kv_append_kernel<32>, dim3(blocks), dim3(kThreads), 0, s, xv, n_chunks, cpr, T, L_max, t0, codes, cache->flags, scales, packed); break;
+        default: launch_pdl(kv_append_kernel<64>, dim3(blocks), dim3(kThreads), 0, s, xv, n_chunks, cpr, T, L_max, t0, codes, cache->flags, scales, packed); break;
     }
     return cudaGetLastError();
 }
@@ -801,18 +807,18 @@ cudaError_t launch_encode_operand(const void *x, int64_t M, int64_t K, const qua
     const int packed = enc && enc->p.flag_bits == 4;
     if (p->code_bits == 16) {  // Section 5 LLM variant: E5M2 operand
         switch (p->group_s) {
-            case 8: encode_operand_kernel<8, true><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
-            case 16: encode_operand_kernel<16, true><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
-            case 32: encode_operand_kernel<32, true><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
-            default: encode_operand_kernel<64, true><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
+            case 8: launch_pdl(encode_operand_kernel<8, true>, dim3(blocks), dim3(kThreads), 0, s, xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
+            case 16: launch_pdl(encode_operand_kernel<16, true>, dim3(blocks), dim3(kThreads), 0, s, xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
+            case 32: launch_pdl(encode_operand_kernel<32, true>, dim3(blocks), dim3(kThreads), 0, s, xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
+            default: launch_pdl(encode_operand_kernel<64, true>, dim3(blocks), dim3(kThreads), 0, s, xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
         }
         return cudaGetLastError();
     }
     switch (p->group_s) {
-        case 8: encode_operand_kernel<8, false><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
-        case 16: encode_operand_kernel<16, false><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
-        case 32: encode_operand_kernel<32, false><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
-        default: encode_operand_kernel<64, false><<<blocks, kThreads, 0, s>>>(xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
+        case 8: launch_pdl(encode_operand_kernel<8, false>, dim3(blocks), dim3(kThreads), 0, s, xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
+        case 16: launch_pdl(encode_operand_kernel<16, false>, dim3(blocks), dim3(kThreads), 0, s, xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
+        case 32: launch_pdl(encode_operand_kernel<32, false>, dim3(blocks), dim3(kThreads), 0, s, xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
+        default: launch_pdl(encode_operand_kernel<64, false>, dim3(blocks), dim3(kThreads), 0, s, xv, n_units, n_units_pad, upr, ws.m_pad, op, ws.a_side, codes, flags, scales, packed); break;
     }
     return cudaGetLastError();
 }
@@ -829,10 +835,10 @@ cudaError_t launch_dequantize(const quartz_encoded_t *e, void *y, cudaStream_t s
     const int packed = e->p.flag_bits == 4;
     uint4 *out = static_cast<uint4 *>(y);
     switch (e->p.group_s) {
-        case 8: dequantize_kernel<8><<<blocks, kThreads, 0, s>>>(codes, e->flags, scales, zeros, e->p.group_q, packed, n_chunks, out); break;
-        case 16: dequantize_kernel<16><<<blocks, kThreads, 0, s>>>(codes, e->flags, scales, zeros, e->p.group_q, packed, n_chunks, out); break;
-        case 32: dequantize_kernel<32><<<blocks, kThreads, 0, s>>>(codes, e->flags, scales, zeros, e->p.group_q, packed, n_chunks, out); break;
-        default: dequantize_kernel<64><<<blocks, kThreads, 0, s>>>(codes, e->flags, scales, zeros, e->p.group_q, packed, n_chunks, out); break;
+        case 8: launch_pdl(dequantize_kernel<8>, dim3(blocks), dim3(kThreads), 0, s, codes, e->flags, scales, zeros, e->p.group_q, packed, n_chunks, out); break;
+        case 16: launch_pdl(dequantize_kernel<16>, dim3(blocks), dim3(kThreads), 0, s, codes, e->flags, scales, zeros, e->p.group_q, packed, n_chunks, out); break;
+        case 32: launch_pdl(dequantize_kernel<32>, dim3(blocks), dim3(kThreads), 0, s, codes, e->flags, scales, zeros, e->p.group_q, packed, n_chunks, out); break;
+        default: launch_pdl(dequantize_kernel<64>, dim3(blocks), dim3(kThreads), 0, s, codes, e->flags, scales, zeros, e->p.group_q, packed, n_chunks, out); break;
     }
     return cudaGetLastError();
 }
