@@ -610,11 +610,13 @@ def run_ours(args):
         s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
         e_steps = max(20, min(args.steps, 50))
 
-        def e2e_run(n_steps):
+        def e2e_run(n_steps, compute=True):
             # unit u = (step, layer) uses buffer set u % 2 of its layer, last
             # used by unit u - 2 nl: its H2D waits only for that unit's encode
             # and its compute only for that unit's D2H, so compute can run up
-            # to 2 nl - 1 units ahead of the slower D2H stream
+            # to 2 nl - 1 units ahead of the slower D2H stream.  compute=False
+            # issues the same copies and events without the kernels (the
+            # control that shows what the host link alone allows)
             loaded, consumed, computed, drained = {}, {}, {}, {}
             units = [(k, i) for k in range(n_steps) for i in range(nl)]
             back = 2 * nl
@@ -627,12 +629,14 @@ def run_ours(args):
                     loaded[u] = torch.cuda.Event()
                     loaded[u].record(s_in)
                 stream.wait_event(loaded[u])
-                Q.quantize(x_buf[p][i], out=enc_a[i], group_s=GROUP_S, group_q=gq[i])
+                if compute:
+                    Q.quantize(x_buf[p][i], out=enc_a[i], group_s=GROUP_S, group_q=gq[i])
                 consumed[u] = torch.cuda.Event()
                 consumed[u].record(stream)
                 if u >= back:
                     stream.wait_event(drained[u - back])
-                Q.linear(enc_a[i], enc_w[i], out=y_buf[p][i], workspace=workspace, w_prepared=prep_w[i])
+                if compute:
+                    Q.linear(enc_a[i], enc_w[i], out=y_buf[p][i], workspace=workspace, w_prepared=prep_w[i])
                 computed[u] = torch.cuda.Event()
                 computed[u].record(stream)
                 with torch.cuda.stream(s_out):
@@ -643,21 +647,32 @@ def run_ours(args):
             stream.wait_event(drained[len(units) - 1])
 
         e2e_run(2)
+        e2e_run(2, compute=False)
         torch.cuda.synchronize()
-        # three timed repetitions of e_steps steps each; the median is the
-        # value, the three are reported as the spread
-        reps = []
-        for _ in range(3):
+
+        def timed_rep(compute):
             barrier()
             a0, a1 = ev(), ev()
             a0.record(stream)
             s_in.wait_stream(stream)
-            e2e_run(e_steps)
+            e2e_run(e_steps, compute)
             a1.record(stream)
             torch.cuda.synchronize()
             barrier()
-            reps.append(max_over_ranks(a0.elapsed_time(a1) / 1e3 / e_steps, world, dev))
+            return max_over_ranks(a0.elapsed_time(a1) / 1e3 / e_steps, world, dev)
+
+        # five timed repetitions of e_steps steps each, every one followed by
+        # the same copies without the kernels; the median is the value.  The
+        # host link itself alternates between two rates from one repetition
+        # to the next (copies alone: about 5.8 or 6.8-7.0 ms per FLUX step),
+        # so the spread of the repetitions is the link's; the ratio to the
+        # copies alone is what the pipeline adds.
+        reps, copy_reps = [], []
+        for _ in range(5):
+            reps.append(timed_rep(True))
+            copy_reps.append(timed_rep(False))
         te = statistics.median(reps)
+        tc = statistics.median(copy_reps)
         h2d = sum(x.numel() * 2 for x in x_host)
         d2h = sum(l.M * l.N * 2 for l in layers)
         link = host_link_gbs(torch, dev)
@@ -667,6 +682,10 @@ def run_ours(args):
                "ms_per_step": te * 1e3, "repetitions": len(reps),
                "ms_per_step_reps": [r * 1e3 for r in reps],
                "spread": (max(reps) - min(reps)) / te,
+               "copies_alone": {"ms_per_step": tc * 1e3, "ms_per_step_reps": [r * 1e3 for r in copy_reps],
+                                "e2e_over_copies": te / tc,
+                                "what": "the same H2D / D2H copies and events with no kernels, timed after "
+                                        "each end-to-end repetition"},
                "overlap": "H2D / compute / D2H on three streams, two buffer sets per layer (compute up to "
                           "2 x layers - 1 units ahead of the D2H stream)",
                "roofline": {"bound": "host link", "link_gbs_measured": link,
