@@ -610,3 +610,54 @@ def test_back_to_back_calls_share_buffers(Q):
         assert torch.equal(r, g), f"call {i} differs when issued back to back"
     for i in range(len(Ns)):
         assert torch.equal(ref[2 * i], ref[2 * i + 1])  # two-call and fused paths agree
+
+
+def test_three_stream_pipeline_matches_synchronous(Q):
+    """Host-to-device copies on one stream, quantize + linear on another and
+    device-to-host copies on a third, ordered only by events, with each
+    device buffer reused two units later (the end-to-end pattern of the
+    benchmark): every host output equals the one a synchronous run gives."""
+    M, K = 700, 1152
+    Ns = [1152, 4608, 3456]
+    xs = [torch.from_numpy(inputs.laplace_activations(M, K, seed=8600 + i)).pin_memory() for i in range(len(Ns))]
+    ws = [Q.encode_weights(torch.from_numpy(inputs.gaussian_weights(n, K, seed=8700 + i)).cuda(), group_s=16)
+          for i, n in enumerate(Ns)]
+    preps = [Q.prepare_weights(w) for w in ws]
+    work = torch.empty(max(Q.linear_workspace_size(M, n, K) for n in Ns), dtype=torch.uint8, device="cuda")
+    enc = Q.empty_encoded(M, K, Q.Params(64, 16), "cuda")
+    steps = 3
+    units = [(k, i) for k in range(steps) for i in range(len(Ns))]
+
+    ref = []
+    for k, i in units:
+        a = Q.quantize(xs[i].cuda(), group_s=16)
+        ref.append(Q.linear(a, ws[i], w_prepared=preps[i]).cpu())
+
+    x_buf = [torch.empty((M, K), dtype=torch.float16, device="cuda") for _ in range(2)]
+    y_buf = [[torch.empty((M, n), dtype=torch.float16, device="cuda") for n in Ns] for _ in range(2)]
+    y_host = [torch.empty((M, Ns[i]), dtype=torch.float16).pin_memory() for _, i in units]
+    s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
+    main = torch.cuda.current_stream()
+    loaded, consumed, computed, drained = {}, {}, {}, {}
+    for u, (k, i) in enumerate(units):
+        p = u % 2
+        with torch.cuda.stream(s_in):
+            if u >= 2:
+                s_in.wait_event(consumed[u - 2])
+            x_buf[p].copy_(xs[i], non_blocking=True)
+            loaded[u] = torch.cuda.Event(); loaded[u].record(s_in)
+        main.wait_event(loaded[u])
+        Q.quantize(x_buf[p], out=enc, group_s=16)
+        consumed[u] = torch.cuda.Event(); consumed[u].record(main)
+        if u >= 2:
+            main.wait_event(drained[u - 2])
+        Q.linear(enc, ws[i], out=y_buf[p][i], workspace=work, w_prepared=preps[i])
+        computed[u] = torch.cuda.Event(); computed[u].record(main)
+        with torch.cuda.stream(s_out):
+            s_out.wait_event(computed[u])
+            y_host[u].copy_(y_buf[p][i], non_blocking=True)
+            drained[u] = torch.cuda.Event(); drained[u].record(s_out)
+    torch.cuda.synchronize()
+    assert Q.device_status() == 0
+    for u in range(len(units)):
+        assert torch.equal(y_host[u], ref[u]), f"unit {u} differs"
