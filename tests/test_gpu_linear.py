@@ -661,3 +661,46 @@ def test_three_stream_pipeline_matches_synchronous(Q):
     assert Q.device_status() == 0
     for u in range(len(units)):
         assert torch.equal(y_host[u], ref[u]), f"unit {u} differs"
+
+
+def test_graph_replay_matches_eager(Q):
+    """quantize + linear and the fused path captured into one CUDA graph
+    (kernels with programmatic dependent launch keep their ordering inside
+    a graph) and replayed twice give the eager results bit for bit."""
+    M, K = 1100, 640
+    Ns = [4400, 4096]  # split last wave / whole tiles
+    xs = [torch.from_numpy(inputs.laplace_activations(M, K, seed=8800 + i)).cuda() for i in range(len(Ns))]
+    ws = [Q.encode_weights(torch.from_numpy(inputs.gaussian_weights(n, K, seed=8900 + i)).cuda(), group_s=16)
+          for i, n in enumerate(Ns)]
+    preps = [Q.prepare_weights(w) for w in ws]
+    work = torch.empty(max(Q.linear_workspace_size(M, n, K) for n in Ns), dtype=torch.uint8, device="cuda")
+    enc = Q.empty_encoded(M, K, Q.Params(64, 16), "cuda")
+    ys = [torch.empty((M, n), dtype=torch.float16, device="cuda") for n in Ns]
+    yf = [torch.empty((M, n), dtype=torch.float16, device="cuda") for n in Ns]
+
+    def body(stream):
+        for i in range(len(Ns)):
+            Q.quantize(xs[i], out=enc, group_s=16, stream=stream)
+            Q.linear(enc, ws[i], out=ys[i], workspace=work, w_prepared=preps[i], stream=stream)
+            Q.linear_f16(xs[i], ws[i], out=yf[i], workspace=work, w_prepared=preps[i], stream=stream)
+
+    body(None)
+    torch.cuda.synchronize()
+    ref = [y.clone() for y in ys] + [y.clone() for y in yf]
+    for y in ys + yf:
+        y.zero_()
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(side):
+        with torch.cuda.graph(g, stream=side):
+            body(side)
+    torch.cuda.current_stream().wait_stream(side)
+    for _ in range(2):
+        g.replay()
+        torch.cuda.synchronize()
+        assert Q.device_status() == 0
+        for r, y in zip(ref, ys + yf):
+            assert torch.equal(r, y)
+        for y in ys + yf:
+            y.zero_()
