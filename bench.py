@@ -319,6 +319,38 @@ def oracle_sample_desc(rows, threads):
             "weights encoded before timing")
 
 
+def oracle_configs(inputs, threads):
+    """The oracle on configs 0-3, context for their GPU lines: config 0 in
+    full and config 1's encode (1M and 16M elements) on one host thread,
+    configs 2 and 3 on ORACLE_ROWS evenly spaced rows per layer on `threads`
+    host threads (encode + linear, weights encoded before timing)."""
+    import oracle as O
+    out = {}
+    l0 = inputs.CONFIG0
+    enc_w, xa = oracle_setup(l0, l0[0].M)
+    t, ops = oracle_step(l0, enc_w, xa, 1)
+    out["config0"] = {"TOPS": ops / t / 1e12, "seconds": t, "threads": 1,
+                      "sample": "the whole layer (256 x 1152 -> 1152), encode + linear"}
+    for key, layers in (("config2", inputs.CONFIG2), ("config3", inputs.CONFIG3)):
+        enc_w, xa = oracle_setup(layers, ORACLE_ROWS)
+        t, ops = oracle_step(layers, enc_w, xa, threads)
+        out[key] = {"TOPS": ops / t / 1e12, "seconds": t, "threads": threads,
+                    "sample": f"{ORACLE_ROWS} evenly spaced rows x all output channels of every layer, "
+                              "encode + linear"}
+    enc = []
+    for rows in (256, 4096):
+        x = inputs.mixture_activations(rows, 4096, seed=inputs.seed_for(1, 0))
+        t0 = time.perf_counter()
+        O.encode(x, GROUP_Q, GROUP_S)
+        t = time.perf_counter() - t0
+        n = rows * 4096
+        enc.append({"elements": n, "seconds": t,
+                    "gbs": n * (2 + 0.5 + 1 / GROUP_S + 2 / GROUP_Q) / t / 1e9})
+    out["config1"] = {"threads": 1, "group_s": GROUP_S, "encode": enc,
+                      "sample": "quantize + LZS encode of the sweep's 1M and 16M-element tensors"}
+    return out
+
+
 def run_reference(args):
     from paper_2509_26436_gb300 import inputs
     rank, world, _ = dist_env()
@@ -705,6 +737,9 @@ def run_ours(args):
         cpu = {"value": oo / tt / 1e12, "unit": "TOPS", "cores": threads, "host_cores": os.cpu_count(),
                "cpu_model": cpu_model(), "kind": "oracle",
                "sample": oracle_sample_desc(ORACLE_ROWS, threads) + f"; 3 steps, {tt:.1f} s"}
+        if args.configs and not per_row:
+            from paper_2509_26436_gb300 import inputs as inp
+            cpu["configs"] = oracle_configs(inp, threads)
 
     if world > 1:
         import torch.distributed as dist
