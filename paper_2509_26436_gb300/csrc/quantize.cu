@@ -226,10 +226,11 @@ __device__ __forceinline__ UnitCodes encode_unit_sym_scaled(const uint4 lo, cons
 // 32767)) grows with |x|, so the FLAG comes from the subgroup's largest
 // |x| (one conversion per subgroup, as in the 8-bit encoder) and each code
 // is bits F .. F+2 of |q|, taken from the 1.5 * 2^23 rounding sum, with the
-// sign of x applied in 4-bit two's complement.  The binary32 operations
-// that produce q are those of the per-chunk encoder, so codes, FLAGs and
-// scales are bit-identical to quartz_quantize's.  All 32 lanes call it
-// together (4 lanes per group).
+// sign of x applied in 4-bit two's complement.  q comes from the binary32
+// operations of the definition (x r with r = RN(1/s), round half to even,
+// the 32767 cap), so codes, FLAGs and scales are exactly Eq. 1 + Eq. 2's
+// (compared bit for bit in the GPU tests).  All 32 lanes call it together
+// (4 lanes per group).
 __device__ __forceinline__ int lzs_flag_wide(float amax_sub, float r)
 {
     const int qmax = min(__float2int_rn(__fmul_rn(amax_sub, r)), 32767);
