@@ -184,10 +184,17 @@ constexpr int kTileBytes = kTile * kD / 2;     // 8 KB of codes per tile and cac
 constexpr int kAttnDynSmem = kStages * 2 * kTileBytes;
 static_assert(kAttnThreads * 33 * 4 <= kAttnDynSmem, "slot reduction fits the code ring");
 
-// At least 5 CTAs per SM: more resident warps to cover the memory latency
-// (measured 8-10% faster than the unbounded 120-register build, no spills).
+// Resident CTAs per SM the register allocation is bounded for: more warps
+// cover the memory latency.  5 (at most 102 registers, no spills) measured
+// 8-10% faster than the unbounded 120-register build.  At G_s = 32 the
+// shared memory of 6 CTAs fits and the kernel compiles to 80 registers
+// without spills: 3-4% faster; at G_s = 8 shared memory allows only 5, and
+// at G_s = 16 the 80-register build spills and is slower, so both keep 5.
 template <int GS>
-__global__ void __launch_bounds__(kAttnThreads, 5) attn_decode_kernel(const __grid_constant__ AttnArgs a)
+constexpr int attn_min_ctas() { return GS == 32 ? 6 : 5; }
+
+template <int GS>
+__global__ void __launch_bounds__(kAttnThreads, attn_min_ctas<GS>()) attn_decode_kernel(const __grid_constant__ AttnArgs a)
 {
     griddep_wait();
     constexpr int S = kD / GS;            // subgroups per row
