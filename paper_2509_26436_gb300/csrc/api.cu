@@ -1,6 +1,7 @@
 // Host side of the C ABI declared in include/quartz.h: argument validation,
 // workspace carving and kernel launches.  Nothing here allocates device
 // memory or synchronises, except quartz_device_status.
+#include <atomic>
 #include <cstring>
 
 #include "quartz_internal.h"
@@ -11,7 +12,8 @@ namespace {
 __device__ int g_device_error;
 
 constexpr int kMaxDevices = 64;
-int *g_error_ptr[kMaxDevices] = {};
+// per device, looked up on first use (any host thread; they all store the same value)
+std::atomic<int *> g_error_ptr[kMaxDevices] = {};
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
@@ -68,12 +70,14 @@ int *device_error_word()
 {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
-    if (!g_error_ptr[dev]) {
+    int *ptr = g_error_ptr[dev].load(std::memory_order_acquire);
+    if (!ptr) {
         void *p = nullptr;
         if (cudaGetSymbolAddress(&p, g_device_error) != cudaSuccess) return nullptr;
-        g_error_ptr[dev] = static_cast<int *>(p);
+        ptr = static_cast<int *>(p);
+        g_error_ptr[dev].store(ptr, std::memory_order_release);
     }
-    return g_error_ptr[dev];
+    return ptr;
 }
 
 }  // namespace quartz

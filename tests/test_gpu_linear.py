@@ -704,3 +704,45 @@ def test_graph_replay_matches_eager(Q):
             assert torch.equal(r, y)
         for y in ys + yf:
             y.zero_()
+
+
+def test_two_host_threads(Q):
+    """Two host threads, each with its own stream, workspace and buffers,
+    issue quantize + linear and the fused path concurrently (the ctypes
+    calls release the GIL): every result equals the one a single thread
+    gives."""
+    import threading
+
+    M, K = 700, 1152
+    Ns = [4608, 1152]
+    xs = [torch.from_numpy(inputs.laplace_activations(M, K, seed=9000 + i)).cuda() for i in range(2)]
+    ws = [Q.encode_weights(torch.from_numpy(inputs.gaussian_weights(n, K, seed=9100 + i)).cuda(), group_s=16)
+          for i, n in enumerate(Ns)]
+    preps = [Q.prepare_weights(w) for w in ws]
+    torch.cuda.synchronize()
+
+    def job(i, stream, out):
+        work = torch.empty(Q.linear_workspace_size(M, Ns[i], K), dtype=torch.uint8, device="cuda")
+        with torch.cuda.stream(stream):
+            for _ in range(5):
+                a = Q.quantize(xs[i], group_s=16, stream=stream)
+                out.append(Q.linear(a, ws[i], workspace=work, w_prepared=preps[i], stream=stream))
+                out.append(Q.linear_f16(xs[i], ws[i], workspace=work, w_prepared=preps[i], stream=stream))
+        stream.synchronize()
+
+    ref = [[], []]
+    for i in range(2):
+        job(i, torch.cuda.Stream(), ref[i])
+    got = [[], []]
+    streams = [torch.cuda.Stream(), torch.cuda.Stream()]
+    threads = [threading.Thread(target=job, args=(i, streams[i], got[i])) for i in range(2)]
+    for t in threads:
+        t.start()
+    for t in threads:
+        t.join()
+    torch.cuda.synchronize()
+    assert Q.device_status() == 0
+    for i in range(2):
+        assert len(got[i]) == len(ref[i])
+        for r, g in zip(ref[i], got[i]):
+            assert torch.equal(r, g)
