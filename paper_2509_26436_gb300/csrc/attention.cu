@@ -36,6 +36,8 @@
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
+#include <atomic>
+
 #include "lzs_e4m3.cuh"
 #include "quartz_internal.h"
 
@@ -428,15 +430,19 @@ int attn_splits(int64_t BH, int64_t L, int64_t slots, int *chunk)
 template <int GS>
 cudaError_t launch_decode(int64_t BH, AttnArgs &a, cudaStream_t s)
 {
-    static int occ = 0;  // resident CTAs per SM of this instance
+    // resident CTAs per SM of this instance, looked up on first use (any
+    // host thread; they all store the same value)
+    static std::atomic<int> occ_cache{0};
     cudaError_t e = cudaFuncSetAttribute(attn_decode_kernel<GS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          kAttnDynSmem);
     if (e != cudaSuccess) return e;
+    int occ = occ_cache.load(std::memory_order_relaxed);
     if (occ == 0) {
         int n = 0;
         e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attn_decode_kernel<GS>, kAttnThreads, kAttnDynSmem);
         if (e != cudaSuccess) return e;
         occ = n > 0 ? n : 1;
+        occ_cache.store(occ, std::memory_order_relaxed);
     }
     int dev = 0, sms = 0;
     cudaGetDevice(&dev);
