@@ -163,7 +163,9 @@ int32_t quartz_dequantize(const quartz_encoded_t *e, void *x_hat_f16, void *stre
  * over all SMs, 2 parts are reserved for each of their tiles although only
  * the tiles cut by a CTA's range boundary, fewer than the SM count, use
  * them, e.g. 64 MiB of which at most 37.75 MiB is written for a
- * 2048 x 11008 -> 4096 layer).  The last part depends on the current
+ * 2048 x 11008 -> 4096 layer; when more than half but not all of the SMs
+ * hold a tile and every tile's groups are spread over all SMs, 3 parts
+ * are reserved per tile).  The last part depends on the current
  * device's SM count: query it on the device that will run the call.
  * Returns 0 for invalid arguments. */
 size_t quartz_linear_workspace_size(int64_t M, int64_t N, int64_t K, const quartz_params_t *p);

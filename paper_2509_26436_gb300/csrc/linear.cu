@@ -272,10 +272,13 @@ struct GemmArgs {
     // (the same count each); each of the remaining tail_tiles is cut along K
     // into `split` group ranges taken by CTAs 0 .. tail_tiles * split - 1,
     // which leave fp32 partial tiles in tail_part; tail_combine_kernel adds
-    // them in part order and writes the outputs.  Two-wave form (ls > 0):
-    // the last tail_tiles tiles' tail_tiles * G group iterations are cut into
-    // one contiguous range of ls per CTA; a tile met by two ranges leaves
-    // parts 0 (groups from 0) and 1 (groups to G), the others are stored whole.
+    // them in part order and writes the outputs.  Range forms (ls > 0): the
+    // last tail_tiles tiles' tail_tiles * G group iterations (after at least
+    // one wave of whole tiles, or every tile's when more than half but not
+    // all of the SMs hold one) are cut into one contiguous range of ls per
+    // CTA, one CTA per SM; a tile met by r ranges leaves parts 0 .. r - 1 in
+    // group order (r <= 2 after whole tiles, where ls >= G; r <= 3 otherwise,
+    // where ls >= G / 2), a tile inside one range is stored whole.
     int full_tiles, tail_tiles, split;
     int ls;
     float *tail_part;     // [tail_tiles][split][16][kEpiWarps * 32] float4 (fp32 pairs)
@@ -355,7 +358,7 @@ __device__ __forceinline__ WorkItem work_item(const GemmArgs &a, int k)
             w.part = -1;
             w.tail = 0;
         } else {
-            w.part = w.g0 == 0 ? 0 : 1;
+            w.part = c - t0 / a.ls;  // ranges before this one that meet the tile
             w.tail = t;
         }
         return w;
@@ -1026,8 +1029,11 @@ __global__ void __launch_bounds__(kEpiWarps * 32) tail_combine_kernel(const __gr
     constexpr int T = kEpiWarps * 32;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int tail = blockIdx.x >> 2, c = blockIdx.x & 3;
-    if (args.ls > 0 && (tail * args.G) / args.ls == ((tail + 1) * args.G - 1) / args.ls)
-        return;  // the tile lies in one CTA's range: stored whole by the GEMM
+    // parts of this tile: every one of the split equal parts, or (range
+    // forms) one per CTA range the tile's groups meet
+    const int parts = args.ls > 0 ? ((tail + 1) * args.G - 1) / args.ls - (tail * args.G) / args.ls + 1
+                                  : args.split;
+    if (parts == 1) return;  // the tile lies in one CTA's range: stored whole by the GEMM
     const uint4 *src = reinterpret_cast<const uint4 *>(args.tail_part) +
                        static_cast<int64_t>(tail) * args.split * 16 * T + 4 * c * T + threadIdx.x;
     uint64_t acc[8];
@@ -1037,7 +1043,7 @@ __global__ void __launch_bounds__(kEpiWarps * 32) tail_combine_kernel(const __gr
         acc[2 * j] = (static_cast<uint64_t>(v.y) << 32) | v.x;
         acc[2 * j + 1] = (static_cast<uint64_t>(v.w) << 32) | v.z;
     }
-    for (int p = 1; p < args.split; ++p) {
+    for (int p = 1; p < parts; ++p) {
         const uint4 *sp = src + static_cast<int64_t>(p) * 16 * T;
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
@@ -1335,6 +1341,7 @@ cudaError_t launch_tc(const CUtensorMap &ta, const CUtensorMap &tw, const GemmAr
     if (e != cudaSuccess) return e;
     int grid = args.num_tiles < num_sms() ? args.num_tiles : num_sms();
     if (args.split > 1 && args.ls == 0 && args.full_tiles == 0) grid = args.tail_tiles * args.split;
+    if (args.ls > 0) grid = num_sms();  // one group range per SM
     launch_pdl(kern, dim3(grid), dim3(kThreads), smem, s, ta, tw, args);
     return cudaGetLastError();
 }
@@ -1445,6 +1452,17 @@ void tail_split(int64_t M, int64_t N, int64_t K, int mode, int *tail, int *split
         *tail = static_cast<int>(Ts);
         *split = 2;
         if (ls) *ls = static_cast<int>((U + P - 1) / P);
+        return;
+    }
+    if (T < sms && 2 * T > sms) {
+        // more than half the SMs hold a tile: the tiles' T * G group
+        // iterations are cut into one contiguous range per SM (ls >= G / 2,
+        // so a tile meets at most 3 ranges: 3 part slots per tile)
+        const int64_t U = T * G;
+        if (G * (sms - T) < kMinStreamSaving * sms || U >= (int64_t(1) << 30)) return;
+        *tail = static_cast<int>(T);
+        *split = 3;
+        if (ls) *ls = static_cast<int>((U + sms - 1) / sms);
         return;
     }
     if (T < sms) {  // fewer tiles than SMs: every tile is cut along K for the idle SMs

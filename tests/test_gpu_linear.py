@@ -262,6 +262,47 @@ def test_linear_two_wave_split_8bit(Q, M, N, K, out_dtype):
     _tol_check(y[torch.from_numpy(rows).cuda()].float().cpu().numpy(), ref, rabs, K // 64, out_dtype)
 
 
+# More than half but not all of the 152 SMs hold a tile: every tile's group
+# iterations are spread in one range per SM, a tile in up to 3 parts.
+# 90 tiles (ragged M and N, 100 groups, ls 60) and SDXL's 3x3 conv on 1280
+# channels at 32x32 (80 tiles, 180 groups, ls 95).
+RANGE_SHAPES = [(1200, 2296, 6400), (2048, 1280, 11520)]
+
+
+def _range_predicate(M, N, K, sms):
+    T = -(-M // 128) * -(-N // 256)
+    return T < sms < 2 * T and (K // 64) * (sms - T) >= 32 * sms
+
+
+@pytest.mark.parametrize("out_dtype", ["float16", "bfloat16", "float32"])
+@pytest.mark.parametrize("M,N,K", RANGE_SHAPES)
+def test_linear_range_split_fewer_tiles_than_sms(Q, M, N, K, out_dtype):
+    """Range plan over all tiles (up to three parts per tile, added by the
+    combine kernel in group order): rows sampled from every M tile, all
+    columns, with a bias, three output types; prepared weights give the
+    same bits."""
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    if not _range_predicate(M, N, K, sms):
+        pytest.skip("this device's SM count does not take the range plan here")
+    assert Q.linear_launch_count(M, N, K) == 3
+    xa = inputs.laplace_activations(M, K, seed=M + K + 3)
+    xw = inputs.gaussian_weights(N, K, seed=N + K + 4)
+    bias = np.random.default_rng(N + 5).normal(0, 0.1, N).astype(np.float16)
+    a = Q.quantize(torch.from_numpy(xa).cuda(), group_s=16)
+    w = Q.encode_weights(torch.from_numpy(xw).cuda(), group_s=16)
+    b = torch.from_numpy(bias).cuda()
+    y = Q.linear(a, w, b, out_dtype=getattr(torch, out_dtype))
+    y_again = Q.linear(a, w, b, out_dtype=getattr(torch, out_dtype), w_prepared=Q.prepare_weights(w))
+    assert Q.device_status() == 0
+    assert torch.equal(y, y_again)
+    rows = _rows_every_m_tile(M)
+    if (M, N, K) not in _two_wave_ref:
+        _two_wave_ref[(M, N, K)] = O.linear(O.encode(xa[rows], 64, 16), O.encode(xw, 64, 16), bias,
+                                            with_abs=True)
+    ref, rabs = _two_wave_ref[(M, N, K)]
+    _tol_check(y[torch.from_numpy(rows).cuda()].float().cpu().numpy(), ref, rabs, K // 64, out_dtype)
+
+
 def test_split_last_wave_launch_count(Q):
     """The host splits the last wave when the tiles after whole waves fill at
     most half a wave and each part keeps at least two groups, and spreads the
@@ -269,14 +310,17 @@ def test_split_last_wave_launch_count(Q):
     at least 32 group iterations on the critical path; the launch count and
     the workspace report it."""
     sms = torch.cuda.get_device_properties(0).multi_processor_count
-    shapes = SPLIT_SHAPES + SMALL_SHAPES + [(2048, 4096, 4096), (2048, 4096, 11008), (1100, 4400, 128),
-                                            (128, 256, 640), (128, 256, 64)]
+    shapes = SPLIT_SHAPES + SMALL_SHAPES + RANGE_SHAPES + [(2048, 4096, 4096), (2048, 4096, 11008),
+                                                           (1100, 4400, 128), (128, 256, 640), (128, 256, 64),
+                                                           (1200, 2296, 640)]
     for M, N, K in shapes:
         T = -(-M // 128) * -(-N // 256)
         P = min(T, sms)
         W, R = divmod(T, P)
         G = K // 64
-        if T < sms:
+        if T < sms and 2 * T > sms:
+            split, part_tiles = G * (sms - T) >= 32 * sms, 3 * T
+        elif T < sms:
             split = min(sms // T, 4, G // 2) >= 2
             part_tiles = T * min(sms // T, 4, G // 2) if split else 0
         elif W >= 1 and 2 * R > P:

@@ -3,17 +3,21 @@
 The persistent GEMM runs P = min(T, SMs) CTAs over T tiles of 128 x 256
 outputs, each a sequence of G 64-wide K groups (Section 4.4, Appendix C).
 When the tiles left after whole waves would leave CTAs idle, the host cuts
-them along K (linear.cu: tail_split; with fewer tiles than SMs every tile is
-cut and the grid has tiles x parts CTAs) and every CTA role walks the same
-work list (work_items / work_item); tail_combine_kernel adds the parts of a
-cut tile and returns at once for a tail tile that one CTA ran whole.
+them along K (linear.cu: tail_split; with at most half as many tiles as
+SMs every tile is cut into equal parts and the grid has tiles x parts CTAs;
+with more than half, every tile's groups are spread in one range per SM)
+and every CTA role walks the same work list (work_items / work_item);
+tail_combine_kernel adds the parts of a cut tile and returns at once for a
+tail tile that one CTA ran whole.
 
 This file restates those three pieces of integer arithmetic in Python and
 checks, over a grid of tile counts, SM counts and group counts, that
   * every (tile, group) pair is computed by exactly one CTA;
   * a tile is either whole (part -1, all G groups on one CTA) or cut into
-    parts numbered 0 .. split-1 (one-wave form) or 0 and 1 (two-wave form),
-    whose group ranges are contiguous, ordered by part and cover [0, G);
+    parts numbered 0 .. split-1 (equal parts) or 0 .. r-1 for the r CTA
+    ranges it meets (range forms: r <= 2 after a wave of whole tiles, r <= 3
+    with fewer tiles than SMs), whose group ranges are contiguous, ordered
+    by part and cover [0, G);
   * every part's partial-tile slot index is inside the workspace that the
     host sizes (tail_tiles x split slots);
   * the combine kernel's test for "this tail tile was cut" agrees with the
@@ -32,10 +36,13 @@ MIN_STREAM_SAVING = 32
 
 
 def grid_size(T, sms, tail, split, ls):
-    """CTAs of the launch: one per tile up to the SM count, or tiles x split
-    when every tile is cut (fewer tiles than SMs)."""
+    """CTAs of the launch: one per tile up to the SM count, tiles x split
+    when every tile is cut into equal parts (fewer tiles than SMs), one per
+    SM when group ranges are spread over the SMs."""
     if split > 1 and ls == 0 and tail == T:
         return tail * split
+    if ls > 0:
+        return sms
     return min(T, sms)
 
 
@@ -50,6 +57,13 @@ def tail_split(T, sms, G):
             return 0, 1, 0
         return Ts, 2, (U + P - 1) // P
     if T < sms:
+        if 2 * T > sms:
+            # more than half the SMs hold a tile: one contiguous range of the
+            # tiles' group iterations per SM (a tile in up to 3 parts)
+            U = T * G
+            if G * (sms - T) < MIN_STREAM_SAVING * sms or U >= 1 << 30:
+                return 0, 1, 0
+            return T, 3, (U + sms - 1) // sms
         S = min(sms // T, MAX_TAIL_SPLIT, G // 2)
         return (T, S, 0) if S >= 2 else (0, 1, 0)
     if W < 1 or R == 0:
@@ -85,7 +99,7 @@ def work_item(c, P, T, G, tail, split, ls, k):
         g0, g1 = max(b - t0, 0), min(e - t0, G)
         if g0 == 0 and g1 == G:
             return full + t, 0, G, -1, 0
-        return full + t, g0, g1, (0 if g0 == 0 else 1), t
+        return full + t, g0, g1, c - t0 // ls, t
     if split <= 1 or k < full // P:
         return c + k * P, 0, G, -1, 0
     ti = c // split
@@ -93,9 +107,15 @@ def work_item(c, P, T, G, tail, split, ls, k):
     return full + ti, part * G // split, (part + 1) * G // split, part, ti
 
 
+def range_parts(tail_index, G, ls):
+    """Parts of tail tile `tail_index` when group ranges of ls are spread
+    over the SMs: the ranges its G group iterations meet."""
+    return ((tail_index + 1) * G - 1) // ls - (tail_index * G) // ls + 1
+
+
 def combine_skips(tail_index, G, ls):
-    """tail_combine_kernel returns at once for this tail tile (two-wave form)."""
-    return ls > 0 and (tail_index * G) // ls == ((tail_index + 1) * G - 1) // ls
+    """tail_combine_kernel returns at once for this tail tile (range forms)."""
+    return ls > 0 and range_parts(tail_index, G, ls) == 1
 
 
 def check_plan(T, sms, G):
@@ -130,7 +150,9 @@ def check_plan(T, sms, G):
         else:
             assert -1 not in parts
             if ls > 0:
-                assert parts == [0, 1], f"tile {tile}: two-wave parts {parts}"
+                ti = tile - (T - tail)
+                assert parts == list(range(range_parts(ti, G, ls))), f"tile {tile}: range parts {parts}"
+                assert len(parts) <= split, f"tile {tile}: {len(parts)} parts, {split} slots"
             else:
                 assert parts == list(range(split)), f"tile {tile}: parts {parts}"
         if split > 1 and tile >= T - tail:
@@ -140,6 +162,8 @@ def check_plan(T, sms, G):
     W = T // min(T, sms)
     if split > 1 and ls == 0 and tail == T:
         assert busiest == -(-G // split)
+    elif split > 1 and ls > 0 and T < sms:
+        assert busiest <= ls and busiest <= G - MIN_STREAM_SAVING
     elif split > 1 and ls > 0:
         assert busiest <= (W - 1) * G + ls
         assert busiest <= (W + 1) * G - MIN_STREAM_SAVING
@@ -190,6 +214,11 @@ def test_split_plan_forms_reached_at_152_sms():
     assert plan(256, 1152, 1152) == (10, 4, 0)
     assert plan(128, 256, 640) == (1, 4, 0)
     assert plan(128, 256, 64)[1] == 1
+    # more than half the SMs hold a tile: one range per SM, tiles in up to 3
+    # parts (SDXL 3x3 conv on 1280 channels at 32x32: 16 x 5 = 80 tiles, 180 groups)
+    assert plan(2048, 1280, 11520) == (80, 3, 95)
+    assert plan(1200, 2296, 6400) == (90, 3, 60)
+    assert plan(1200, 2296, 640)[1] == 1   # saving too small
 
 
 def test_split_plan_exhaustive_small():
