@@ -254,6 +254,29 @@ def test_linear16_tcgen05_llama_layers_sampled(Q, layer):
                   layer.K // 64, "float16")
 
 
+def test_linear16_tcgen05_range_split(Q):
+    """16-bit codes through the range plan (90 tiles on 152 SMs, 100 groups,
+    tiles in up to 3 parts added by the combine kernel): rows sampled from
+    every M tile, a bias, against the oracle with the E5M2 sum bound."""
+    M, N, K = 1200, 2296, 6400
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    T = -(-M // 128) * -(-N // 256)
+    if not (T < sms < 2 * T and (K // 64) * (sms - T) >= 32 * sms):
+        pytest.skip("this device's SM count does not take the range plan here")
+    assert Q.linear_launch_count(M, N, K, Q.Params(64, 8, code_bits=16)) == 3
+    xa = inputs.laplace_activations(M, K, seed=5900, outlier_frac=0.002, outlier_scale=100.0)
+    xw = inputs.gaussian_weights(N, K, seed=5901)
+    bias = np.random.default_rng(5902).normal(0, 0.1, N).astype(np.float16)
+    a = Q.quantize(torch.from_numpy(xa).cuda(), group_s=8, code_bits=16)
+    w = Q.encode_weights(torch.from_numpy(xw).cuda(), group_s=8, code_bits=16)
+    y = Q.linear(a, w, torch.from_numpy(bias).cuda(), algo=Q.ALGO_TCGEN05)
+    assert Q.device_status() == 0
+    rows = np.unique([min(m0 + d, M - 1) for m0 in range(0, M, 128) for d in (0, 5, 63, 127)])
+    rt = torch.from_numpy(rows).cuda()
+    _tc_tol_check(y[rt].float().cpu().numpy(), O.encode16(xa[rows], 64, 8), O.encode16(xw, 64, 8), bias,
+                  K // 64, "float16")
+
+
 # --- fused activation path with 16-bit codes ---------------------------------
 
 @pytest.mark.parametrize("flag_bits", [8, 4])
