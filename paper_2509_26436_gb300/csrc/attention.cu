@@ -48,8 +48,6 @@ constexpr int kD = 128;              // head dimension
 constexpr int kWords = kD / 8;       // 32-bit code words per token row
 constexpr int kTile = 128;           // tokens per tile = threads per CTA
 constexpr int kAttnThreads = 128;
-constexpr int kChunksPerRow = 4;               // 16-byte code chunks (32 codes) per token row
-constexpr int kSlots = kAttnThreads / kChunksPerRow;  // token slots of the value phase
 constexpr int kPfStride = kTile + 2;           // s_pf row stride: conflict-free reads and writes
 constexpr int kPartStride = kD + 4;  // o[128], m, l (+ pad) per split
 constexpr int kMaxSplits = 64;
@@ -184,16 +182,24 @@ __device__ __forceinline__ void load_side(const AttnArgs &a, int64_t row, bool v
 constexpr int kStages = 2;                     // code tiles in flight per CTA
 constexpr int kTileBytes = kTile * kD / 2;     // 8 KB of codes per tile and cache
 constexpr int kAttnDynSmem = kStages * 2 * kTileBytes;
-static_assert(kAttnThreads * 33 * 4 <= kAttnDynSmem, "slot reduction fits the code ring");
+// Value phase layout: each thread takes kValDims dimensions (one piece of
+// a token row's codes) of tile_tokens / slots tokens.  16 dimensions (an
+// 8-byte piece, 16 accumulators) at G_s = 8 and 16: fewer registers, which
+// lets G_s = 16 run 6 CTAs per SM (2-3% faster at G_s = 8 and 16); 32 (a
+// 16-byte chunk) at G_s = 32 and 64, 1% faster there.
+template <int GS>
+constexpr int val_dims() { return GS <= 16 ? 16 : 32; }
+static_assert(kAttnThreads * (16 + 1) * 4 <= kAttnDynSmem && kAttnThreads * (32 + 1) * 4 <= kAttnDynSmem,
+              "slot reduction fits the code ring");
 
 // Resident CTAs per SM the register allocation is bounded for: more warps
 // cover the memory latency.  5 (at most 102 registers, no spills) measured
-// 8-10% faster than the unbounded 120-register build.  At G_s = 32 the
-// shared memory of 6 CTAs fits and the kernel compiles to 80 registers
-// without spills: 3-4% faster; at G_s = 8 shared memory allows only 5, and
-// at G_s = 16 the 80-register build spills and is slower, so both keep 5.
+// 8-10% faster than the unbounded 120-register build.  At G_s = 16 and 32
+// the shared memory of 6 CTAs fits and the kernel compiles to at most 80
+// registers without spills (G_s = 16 with the 16-dimension value layout):
+// 3-4% faster; at G_s = 8 shared memory allows only 5.
 template <int GS>
-constexpr int attn_min_ctas() { return GS == 32 ? 6 : 5; }
+constexpr int attn_min_ctas() { return GS == 16 || GS == 32 ? 6 : 5; }
 
 template <int GS>
 __global__ void __launch_bounds__(kAttnThreads, attn_min_ctas<GS>()) attn_decode_kernel(const __grid_constant__ AttnArgs a)
@@ -264,11 +270,15 @@ __global__ void __launch_bounds__(kAttnThreads, attn_min_ctas<GS>()) attn_decode
     __syncthreads();
     const uint32_t sq_addr = static_cast<uint32_t>(__cvta_generic_to_shared(s_q));
 
-    const int vc = tid % kChunksPerRow;  // value phase: 16-byte code chunk (dims 32 vc ..)
-    const int slot = tid / kChunksPerRow; // value phase: token slot
-    float acc[32];
+    constexpr int kValDims = val_dims<GS>();          // value phase: dimensions per thread
+    constexpr int kPieces = kD / kValDims;             // code pieces per token row
+    constexpr int kSlots = kAttnThreads / kPieces;     // token slots
+    constexpr int kWordsPerPiece = kValDims / 8;       // 32-bit code words per piece
+    const int vc = tid % kPieces;   // value phase: code piece (dims kValDims vc ..)
+    const int slot = tid / kPieces; // value phase: token slot
+    float acc[kValDims];
 #pragma unroll
-    for (int k = 0; k < 32; ++k) acc[k] = 0.f;
+    for (int k = 0; k < kValDims; ++k) acc[k] = 0.f;
     float m_run = -INFINITY;  // running maximum (log2 domain)
     float l_thr = 0.f;        // this thread's share of the running sum
 
@@ -331,7 +341,7 @@ __global__ void __launch_bounds__(kAttnThreads, attn_min_ctas<GS>()) attn_decode
             s_pf[j][tid] = p * scale_pow2((j * GS) / 64 ? cur.sv.y : cur.sv.x, row_flag(cur.vf, j, a.v_packed != 0));
         if (m_new != m_run) {  // CTA-uniform: rescale only when the maximum grew
 #pragma unroll
-            for (int k = 0; k < 32; ++k) acc[k] *= alpha;
+            for (int k = 0; k < kValDims; ++k) acc[k] *= alpha;
         }
         m_run = m_new;
         __syncthreads();
@@ -340,12 +350,18 @@ __global__ void __launch_bounds__(kAttnThreads, attn_min_ctas<GS>()) attn_decode
 #pragma unroll
         for (int i = 0; i < kTile / kSlots; ++i) {
             const int ti = slot + i * kSlots;
-            const uint4 ch = lds_u4(vst + tile_off(ti, vc));
-            const uint32_t words[4] = {ch.x, ch.y, ch.z, ch.w};
+            uint32_t words[kWordsPerPiece];
+            if constexpr (kWordsPerPiece == 4) {
+                const uint4 ch = lds_u4(vst + tile_off(ti, vc));
+                words[0] = ch.x, words[1] = ch.y, words[2] = ch.z, words[3] = ch.w;
+            } else {
+                asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(words[0]), "=r"(words[1])
+                             : "r"(vst + tile_off(ti, vc >> 1) + 8 * (vc & 1)));
+            }
 #pragma unroll
-            for (int w = 0; w < 4; ++w) {
-                // word 4 vc + w of the row; its subgroup's factor (0 past the end)
-                const int sub = (4 * vc + w) / kWordsPerSub;
+            for (int w = 0; w < kWordsPerPiece; ++w) {
+                // word kWordsPerPiece vc + w of the row; its subgroup's factor (0 past the end)
+                const int sub = (kWordsPerPiece * vc + w) / kWordsPerSub;
                 const float pf = s_pf[sub][ti];
                 const uint32_t ev = (words[w] & 0x0F0F0F0Fu) ^ 0x08080808u;         // codes 0, 2, 4, 6 as c + 8
                 const uint32_t od = ((words[w] >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u;  // codes 1, 3, 5, 7
@@ -361,13 +377,13 @@ __global__ void __launch_bounds__(kAttnThreads, attn_min_ctas<GS>()) attn_decode
     cp_async_wait<0>();
 
     // ---- reduce over token slots, write this split's partial result -------
-    // (the code ring is free now: thread (slot, vc) stores its 32 sums at
-    // (4 slot + vc) * 33, which keeps both the stores and the column reads
-    // below free of bank conflicts)
+    // (the code ring is free now: thread (slot, vc) stores its kValDims sums
+    // at (kPieces slot + vc) * (kValDims + 1), which keeps both the stores and
+    // the column reads below free of bank conflicts)
     __syncthreads();
     float *s_red = reinterpret_cast<float *>(s_ring);
 #pragma unroll
-    for (int k = 0; k < 32; ++k) s_red[(slot * kChunksPerRow + vc) * 33 + k] = acc[k];
+    for (int k = 0; k < kValDims; ++k) s_red[(slot * kPieces + vc) * (kValDims + 1) + k] = acc[k];
     float ws = l_thr;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) ws += __shfl_xor_sync(0xffffffffu, ws, o);
@@ -375,7 +391,8 @@ __global__ void __launch_bounds__(kAttnThreads, attn_min_ctas<GS>()) attn_decode
     __syncthreads();
     float od = 0.f;
 #pragma unroll 8
-    for (int sl = 0; sl < kSlots; ++sl) od += s_red[(sl * kChunksPerRow + tid / 32) * 33 + (tid & 31)];
+    for (int sl = 0; sl < kSlots; ++sl)
+        od += s_red[(sl * kPieces + tid / kValDims) * (kValDims + 1) + (tid % kValDims)];
     float *part = a.part + (bh * a.n_split + split) * kPartStride;
     part[tid] = od;
     if (tid == 0) {
