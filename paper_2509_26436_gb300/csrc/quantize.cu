@@ -238,22 +238,25 @@ __device__ __forceinline__ int lzs_flag_wide(float amax_sub, float r)
 }
 
 // Codes of 8 elements (four fp16 pairs `w`, sign-cleared copies `a`) for
-// 16-bit stage-1 codes: |q| = rne(|x| r) (capped at 32767 when CAP), c =
-// sgn(x) (|q| >> flag), element k in bits 4k..4k+3.
-template <bool CAP>
+// 16-bit stage-1 codes: c = sgn(x) (min(rne(|x| r), 32767) >> flag), element
+// k in bits 4k..4k+3.  Branch-free cap: the fp16 scale can round down (by up
+// to half of it for the smallest subnormal scales), so rne(|x| r) reaches
+// up to 49151 for the elements nearest the group maximum.  Such an element
+// lies in a subgroup with FLAG 12 (its capped maximum is 32767), where its
+// shifted magnitude is 8..11 against the capped value's 7, while every
+// shifted magnitude in a subgroup with a lower FLAG is at most 7; so each
+// packed magnitude byte b <= 15 becomes (b & 7) | 7 * (bit 3 of b).  (A
+// branch on the cap, as the 8-bit encoder has, diverges here: with 32767
+// levels the fp16 rounding of the scale takes it in about half the groups.)
 __device__ __forceinline__ uint32_t lzs_word8_wide(const uint32_t *w, const uint32_t *a, float r, int flag)
 {
     uint32_t u[4][2];
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
         const float2 f = __half22float2(*reinterpret_cast<const __half2 *>(&a[i]));
-        float2 t = mul2_rn(f, make_float2(r, r));
-        if (CAP) {
-            t.x = fminf(t.x, 32767.0f);
-            t.y = fminf(t.y, 32767.0f);
-        }
+        const float2 t = mul2_rn(f, make_float2(r, r));
         // scalar additions (see lzs_word8); the low 22 bits of the sum are
-        // |q|, and |q| >> flag <= 7 lands in the low byte
+        // rne(|x| r), and its value >> flag (at most 11) lands in the low byte
         u[i][0] = __float_as_uint(__fadd_rn(t.x, kRoundAddend)) >> flag;
         u[i][1] = __float_as_uint(__fadd_rn(t.y, kRoundAddend)) >> flag;
     }
@@ -261,8 +264,10 @@ __device__ __forceinline__ uint32_t lzs_word8_wide(const uint32_t *w, const uint
     const uint32_t od = prmt(prmt(u[0][1], u[1][1], 0x0040u), prmt(u[2][1], u[3][1], 0x0040u), 0x5410u);
     const uint32_t sev = prmt(prmt(w[0], w[1], 0x00D9u), prmt(w[2], w[3], 0x00D9u), 0x5410u);
     const uint32_t sod = prmt(prmt(w[0], w[1], 0x00FBu), prmt(w[2], w[3], 0x00FBu), 0x5410u);
-    const uint32_t cev = signed_nibbles(ev & 0x07070707u, sev);
-    const uint32_t cod = signed_nibbles(od & 0x07070707u, sod);
+    const uint32_t mev = (ev & 0x07070707u) | (((ev >> 3) & 0x01010101u) * 7u);  // bytes 8..15 -> 7
+    const uint32_t mod = (od & 0x07070707u) | (((od >> 3) & 0x01010101u) * 7u);
+    const uint32_t cev = signed_nibbles(mev, sev);
+    const uint32_t cod = signed_nibbles(mod, sod);
     return cev | (cod << 4);
 }
 
@@ -294,13 +299,8 @@ __device__ __forceinline__ UnitCodes encode_unit_wide(const uint4 lo, const uint
         const float m = GS == 16 ? unit_max : GS == 32 ? pair_max : amax;
         u.flag0 = u.flag1 = lzs_flag_wide(m, r);
     }
-    if (__float2int_rn(__fmul_rn(amax, r)) > 32767) {  // only when the fp16 scale rounded down
-        u.c0 = lzs_word8_wide<true>(w, a, r, u.flag0);
-        u.c1 = lzs_word8_wide<true>(w + 4, a + 4, r, u.flag1);
-    } else {
-        u.c0 = lzs_word8_wide<false>(w, a, r, u.flag0);
-        u.c1 = lzs_word8_wide<false>(w + 4, a + 4, r, u.flag1);
-    }
+    u.c0 = lzs_word8_wide(w, a, r, u.flag0);
+    u.c1 = lzs_word8_wide(w + 4, a + 4, r, u.flag1);
     u.flag_next = 0;
     if (GS >= 16) u.flag_next = __shfl_down_sync(0xffffffffu, u.flag0, kUnitsPerSub<GS>());
     return u;

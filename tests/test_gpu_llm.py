@@ -78,6 +78,25 @@ def test_encode16_edge_values(Q):
     assert ref.flags.max() == 12
 
 
+def test_encode16_cap_every_fp16_maximum(Q):
+    """The 32767 cap at every scale: one 64-element group per positive finite
+    fp16 maximum (31743 rows, normal and subnormal scales), holding that
+    maximum and the 63 fp16 values just below it with seeded signs.  The
+    fp16 scale rounds down for about half of the maxima, so rne(|x| r)
+    passes 32767 (up to about 1.5 x 32767 for the smallest subnormal scales)
+    for the values nearest the maximum; codes, FLAGs and scales must still be
+    Eq. 1 + Eq. 2's with the cap, at every G_s."""
+    top = np.arange(1, 0x7C00, dtype=np.int64)
+    bits = np.clip(top[:, None] - np.arange(64)[None, :], 0, None).astype(np.uint16)
+    x = bits.view(np.float16).copy()
+    signs = np.random.default_rng(2509).integers(0, 2, size=x.shape).astype(bool)
+    x[signs] = -x[signs]
+    for gs in (8, 16, 32, 64):
+        ref = O.encode16(x, 64, gs)
+        _assert_equal(_enc(Q, x, gs), ref)
+    assert ref.flags.max() == 12
+
+
 @pytest.mark.parametrize("gs", [8, 16, 64])
 @pytest.mark.parametrize("shape", [(1, 64), (3, 576), (129, 4096)])
 def test_encode16_packed_flags(Q, gs, shape):
